@@ -1,0 +1,506 @@
+#!/usr/bin/env python3
+"""Benchmark of the HSA hot path on GB300 (prints one JSON line on rank 0).
+
+Step = one pass of the prefill hot path over one batch of the long-context
+workload (B=2, L=32768, S=64, Hq=32, Hkv=4, d=128, top-k=8): chunk pool ->
+top-k selection -> inverse index -> forward -> backward, all through the C ABI.
+The decode sub-benchmark runs hsa_decode against a resident 2^26-token memory
+(64 queries x 8 heads, top-k 8). Inputs are seeded synthetic tensors generated
+on the device.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl hsa|reference]
+
+N > 1 runs under torch.distributed.run: every rank processes its own batch
+(weak scaling, no data-path collective); the max time over ranks is used.
+--impl reference times the CPU oracle on the same workload and metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "HSA fwd+bwd tokens/s (L=32K,S=64,k=8); decode q/s @64M memory; % roofline"
+UNIT = "tokens/s"
+PREFILL = synth.WORKLOADS[3]
+DECODE = synth.WORKLOADS[5]
+
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of the dominant
+# kernel from one ncu capture, keyed by the source file it was compiled from
+# and that file's sha256 at capture time (reported as null once the source
+# has changed).
+NCU_TRAFFIC = {}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            j = json.load(f)
+        return dict(hbm=float(j["hbm_gbs"]), bf16=float(j["bf16_tflops"]),
+                    bf16_sus=float(j.get("bf16_tflops_sustained", j["bf16_tflops"])), source="measured")
+    except (OSError, KeyError, ValueError):
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+def source_sha(rel):
+    import hashlib
+
+    with open(os.path.join(ROOT, rel), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+# ----------------------------------------------------------------------------- algorithmic work
+
+def slot_heads(w):
+    """Number of (token, query head, selected chunk) triples."""
+    t = np.arange(w.L)
+    keff = np.minimum(w.topk, np.minimum(t // w.S, w.Nc))
+    return int(keff.sum()) * w.Hq * w.B
+
+
+def visible_pairs(w):
+    t = np.arange(w.L)
+    return int(np.minimum(t // w.S, w.Nc).sum()) * w.B * w.Hkv
+
+
+def work_model(w):
+    """Algorithmic FLOPs and compulsory HBM bytes per call (one batch)."""
+    bf, f4 = 2, 4
+    q = w.B * w.L * w.Hq * w.d
+    kv = w.B * w.L * w.Hkv * w.d
+    kb = w.B * w.Nc * w.Hkv * w.d
+    sel = w.B * w.L * w.Hkv * w.topk
+    u = slot_heads(w)
+    return {
+        "hsa_chunk_pool": dict(flops=kv, bytes=kv * bf + kb * (f4 + bf)),
+        "hsa_select_topk": dict(flops=2 * w.d * visible_pairs(w) + q, bytes=q * bf + kb * f4 + sel * (4 + f4)),
+        "hsa_build_index": dict(flops=0, bytes=sel * 4 * 3 + w.B * w.Hkv * w.Nc * 4),
+        "hsa_forward": dict(flops=4 * w.S * w.d * u, bytes=q * bf * 2 + 2 * kv * bf + sel * (4 + f4 + f4)),
+        "hsa_backward": dict(flops=10 * w.S * w.d * u,
+                             bytes=3 * q * bf + 2 * kv * bf + kb * f4 + q * f4 + 2 * kv * f4 + sel * (4 + f4)),
+    }
+
+
+def bound_of(flops, nbytes, pk):
+    t_tensor = flops / (pk["bf16_sus"] * 1e12)
+    t_hbm = nbytes / (pk["hbm"] * 1e9)
+    return ("tensor", t_tensor) if t_tensor >= t_hbm else ("hbm", t_hbm)
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        self.f.close()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        try:
+            rows = open(self.path).read().strip().splitlines()
+        except OSError:
+            rows = []
+        for r in rows:
+            parts = [p.strip() for p in r.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        loaded = [s for s in sm if s >= 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2504_16795_gb300 as hsa
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    if not os.path.exists(hsa.lib_path()):
+        if rank == 0:
+            hsa.build()
+        if world > 1:
+            dist.barrier()
+    hsa.load()
+    pk = peaks()
+    w = PREFILL
+    shape = hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk)
+    log(f"[rank {rank}] generating inputs for {w.name}")
+    X = {n: synth.device_tensor(w, n, dev) for n in ("q", "K", "V", "dO")}
+    wss = hsa.Workspaces(shape, dev)
+    f32, i32, bf = torch.float32, torch.int32, torch.bfloat16
+    sel = (w.B, w.L, w.Hkv, w.topk)
+    Y = dict(kbar32=torch.empty((w.B, w.Nc, w.Hkv, w.d), dtype=f32, device=dev),
+             kbar16=torch.empty((w.B, w.Nc, w.Hkv, w.d), dtype=bf, device=dev),
+             idx=torch.empty(sel, dtype=i32, device=dev), s_sel=torch.empty(sel, dtype=f32, device=dev),
+             offsets=torch.empty(w.B * w.Hkv * w.Nc + 1, dtype=i32, device=dev),
+             entries=torch.empty(w.B * w.L * w.Hkv * w.topk, dtype=i32, device=dev),
+             O=torch.empty_like(X["q"]), w=torch.empty(sel, dtype=f32, device=dev),
+             dq=torch.empty(X["q"].shape, dtype=f32, device=dev),
+             dK=torch.empty(X["K"].shape, dtype=f32, device=dev),
+             dV=torch.empty(X["V"].shape, dtype=f32, device=dev))
+    calls = ["hsa_chunk_pool", "hsa_select_topk", "hsa_build_index", "hsa_forward", "hsa_backward"]
+
+    def step(ev=None):
+        def mark(i):
+            if ev is not None:
+                ev[i].record()
+        mark(0)
+        hsa.chunk_pool(shape, X["K"], Y["kbar32"], Y["kbar16"])
+        mark(1)
+        hsa.select_topk(shape, X["q"], Y["kbar32"], Y["idx"], Y["s_sel"])
+        mark(2)
+        hsa.build_index(shape, Y["idx"], Y["offsets"], Y["entries"], ws=wss.index)
+        mark(3)
+        hsa.forward(shape, X["q"], X["K"], X["V"], Y["idx"], Y["s_sel"], Y["offsets"], Y["entries"], Y["O"],
+                    Y["w"], ws=wss.forward)
+        mark(4)
+        hsa.backward(shape, X["q"], X["K"], X["V"], Y["kbar32"], Y["idx"], Y["w"], Y["O"], X["dO"], Y["offsets"],
+                     Y["entries"], Y["dq"], Y["dK"], Y["dV"], ws=wss.backward)
+        mark(5)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    K = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(K)]
+    launches0 = hsa.kernel_launches()
+    with ClockSampler(local_rank) as clk:
+        barrier()
+        wall0 = time.perf_counter()
+        for i in range(K):
+            step(evs[i])
+        barrier()
+        wall = time.perf_counter() - wall0
+    launches = hsa.kernel_launches() - launches0
+    clocks = clk.summary()
+    ms_total = sum(evs[i][0].elapsed_time(evs[i][5]) for i in range(K))
+    per_call = {c: statistics.mean(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K))
+                for j, c in enumerate(calls)}
+    ms_total = max_over_ranks(ms_total)
+    ms_step = ms_total / K
+    tokens = w.B * w.L
+    value = world * tokens * K / (ms_total / 1e3)
+    log(f"[rank {rank}] {ms_step:.3f} ms/step, wall {wall / K * 1e3:.3f} ms/step, per call (ms): "
+        + ", ".join(f"{c} {v:.3f}" for c, v in per_call.items()))
+
+    # roofline per call; the dominant call is the headline
+    model = work_model(w)
+    kernels = {}
+    for c in calls:
+        m = model[c]
+        bound, t_min = bound_of(m["flops"], m["bytes"], pk)
+        sec = per_call[c] / 1e3
+        if bound == "tensor":
+            ach, peak, unit = m["flops"] / sec / 1e12, pk["bf16_sus"], "TFLOP/s"
+        else:
+            ach, peak, unit = m["bytes"] / sec / 1e9, pk["hbm"], "GB/s"
+        kernels[c] = {"ms": round(per_call[c], 4), "bound": bound, "achieved": round(ach, 2), "peak": peak,
+                      "unit": unit, "frac": round(ach / peak, 4), "algorithmic_flops": m["flops"],
+                      "algorithmic_bytes": m["bytes"], "roofline_ms": round(t_min * 1e3, 4)}
+    dom = max(calls, key=lambda c: per_call[c])
+    tr = NCU_TRAFFIC.get(dom)
+    traffic = None
+    if tr and source_sha(tr["source"]) == tr["sha256"]:
+        traffic = tr["bytes_per_launch"]
+    roof = {k: kernels[dom][k] for k in ("bound", "achieved", "peak", "unit", "frac")}
+    roof.update({"kernel": dom, "traffic": traffic,
+                 "peak_source": f"{pk['source']} ({'bf16 sustained' if roof['bound'] == 'tensor' else 'hbm copy'})"})
+
+    # end to end through host buffers: H2D inputs, the path, D2H outputs, every step
+    e2e = None
+    if not args.no_e2e:
+        host_in = {n: torch.empty(X[n].shape, dtype=X[n].dtype, pin_memory=True) for n in ("q", "K", "V", "dO")}
+        for n in host_in:
+            host_in[n].copy_(X[n])
+        host_out = {n: torch.empty(Y[n].shape, dtype=Y[n].dtype, pin_memory=True) for n in ("O", "dq", "dK", "dV")}
+        h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+        d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+
+        def e2e_step():
+            for n, t in host_in.items():
+                X[n].copy_(t, non_blocking=True)
+            step()
+            for n, t in host_out.items():
+                t.copy_(Y[n], non_blocking=True)
+
+        for _ in range(max(1, min(args.warmup, 2))):
+            e2e_step()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(K):
+            e2e_step()
+        e1.record()
+        barrier()
+        ms_e2e = max_over_ranks(e0.elapsed_time(e1))
+        e2e = {"value": world * tokens * K / (ms_e2e / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e / K}
+        del host_in, host_out
+
+    del X, Y, wss
+    torch.cuda.empty_cache()
+
+    decode = None
+    if not args.no_decode:
+        decode = run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa)
+
+    return dict(value=value, ms_step=ms_step, kernels=kernels, roofline=roof, e2e=e2e, clocks=clocks,
+                launches=launches, decode=decode, wall_ms_step=wall / K * 1e3)
+
+
+def run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa):
+    import torch
+
+    w = DECODE
+    T, Nc = w.L, w.Nc
+    log(f"generating the {T}-token decode memory")
+    Kmem = synth.device_tensor(w, "K", dev)
+    Vmem = synth.device_tensor(w, "V", dev)
+    q = synth.device_tensor(w, "q", dev)
+    pshape = hsa.Shape(B=1, L=T, Hq=w.Hq, Hkv=w.Hkv, d=w.d, topk=w.topk)
+    kbar32 = torch.empty((1, Nc, w.Hkv, w.d), dtype=torch.float32, device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    hsa.chunk_pool(pshape, Kmem.view(1, T, w.Hkv, w.d), kbar32, None, want_bf16=False)
+    e1.record()
+    barrier()
+    pool_ms = e0.elapsed_time(e1)
+    dshape = hsa.DecodeShape(Bq=w.Bq, Hq=w.Hq, Hkv=w.Hkv, d=w.d, n_chunks=Nc, topk=w.topk)
+    kb = kbar32.view(Nc, w.Hkv, w.d)
+    O = torch.empty_like(q)
+    out = (w.Bq, w.Hkv, w.topk)
+    idx = torch.empty(out, dtype=torch.int32, device=dev)
+    s_sel = torch.empty(out, dtype=torch.float32, device=dev)
+    wts = torch.empty(out, dtype=torch.float32, device=dev)
+    ws = torch.empty(hsa.decode_workspace_size(dshape), dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        hsa.decode(dshape, q, Kmem, Vmem, kb, O, idx, s_sel, wts, ws)
+    barrier()
+    steps = max(args.steps, 10)
+    e0.record()
+    for _ in range(steps):
+        hsa.decode(dshape, q, Kmem, Vmem, kb, O, idx, s_sel, wts, ws)
+    e1.record()
+    barrier()
+    ms = max_over_ranks(e0.elapsed_time(e1)) / steps
+    needles = synth.needle_chunk_ids(w)
+    got = idx.cpu().numpy()
+    found = int(sum(int(needles[b]) in got[b, 0] for b in range(w.Bq)))
+    scan_bytes = Nc * w.Hkv * w.d * 4
+    gather_bytes = w.Bq * w.Hkv * w.topk * 2 * w.S * w.d * 2
+    nbytes = scan_bytes + gather_bytes + 2 * w.Bq * w.Hq * w.d * 2
+    flops = 2 * w.Bq * w.Hkv * Nc * w.d
+    achieved = nbytes / (ms / 1e3) / 1e9
+    del Kmem, Vmem
+    torch.cuda.empty_cache()
+    return {"value": world * w.Bq / (ms / 1e3), "unit": "queries/s", "ms_per_call": ms,
+            "memory_tokens": T, "chunks": Nc, "queries": w.Bq, "Hq": w.Hq, "Hkv": w.Hkv, "d": w.d, "topk": w.topk,
+            "needles_found": f"{found}/{w.Bq}", "pool_ms_once": pool_ms,
+            "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm"], "unit": "GB/s",
+                         "frac": round(achieved / pk["hbm"], 4), "algorithmic_bytes": nbytes,
+                         "scan": "fp32 chunk summaries", "flops": flops}}
+
+
+# ----------------------------------------------------------------------------- CPU oracle (baseline / reference arm)
+
+def oracle_sample(T, b=0):
+    """Host inputs for the last T tokens of batch b (all groups), as fp64 [1, L, ...] arrays."""
+    w = PREFILL
+    t0 = w.L - T
+    q = np.zeros((1, w.L, w.Hq, w.d))
+    dO = np.zeros((1, w.L, w.Hq, w.d))
+    q[:, t0:] = synth.bf16_to_f64(synth.host_tensor(w, "q", (b, t0, 0, 0), (b + 1, w.L, w.Hq, w.d)))
+    dO[:, t0:] = synth.bf16_to_f64(synth.host_tensor(w, "dO", (b, t0, 0, 0), (b + 1, w.L, w.Hq, w.d)))
+    K = synth.bf16_to_f64(synth.host_tensor(w, "K", (b, 0, 0, 0), (b + 1, w.L, w.Hkv, w.d)))
+    V = synth.bf16_to_f64(synth.host_tensor(w, "V", (b, 0, 0, 0), (b + 1, w.L, w.Hkv, w.d)))
+    mask = np.zeros((1, w.L), np.uint8)
+    mask[0, t0:] = 1
+    return q, K, V, dO, mask
+
+
+def oracle_step(data):
+    """Time the oracle's fwd+bwd on the sampled tokens; pooling is charged pro rata."""
+    import oracle
+
+    w = PREFILL
+    q, K, V, dO, mask = data
+    T = int(mask.sum())
+    t0 = time.perf_counter()
+    kbar32 = oracle.pool(K, w.S, f32=True)
+    kbar64 = oracle.pool(K, w.S)
+    t_pool = time.perf_counter() - t0
+    t1 = time.perf_counter()
+    idx, s_sel, _ = oracle.select(q, kbar32, w.S, w.topk, f32=True, token_mask=mask)
+    oracle.forward(q, K, V, idx, s_sel, w.S, token_mask=mask)
+    oracle.backward(q, K, V, kbar64, idx, s_sel, dO, w.S, token_mask=mask)
+    t_rest = time.perf_counter() - t1
+    return t_rest + t_pool * T / w.L
+
+
+def cpu_baseline(target_s=15.0):
+    import oracle
+
+    oracle.build()
+    T = 128
+    sec = oracle_step(oracle_sample(T))
+    T2 = int(min(4096, max(T, T * target_s / max(sec, 1e-3))))
+    T2 = max(64, (T2 // 64) * 64)
+    sec2 = oracle_step(oracle_sample(T2))
+    return {"value": T2 / sec2, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+            "sample": (f"fwd+bwd of the last {T2} tokens of batch 0 (all 4 groups, 32 heads) of the "
+                       f"B=2 L=32768 workload; selection over all visible chunks; chunk pooling charged "
+                       f"pro rata; {sec2:.1f} s of CPU time")}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    import oracle
+
+    oracle.build()
+    T = 128
+    data = oracle_sample(T)
+    for _ in range(args.warmup):
+        oracle_step(data)
+    times = [oracle_step(data) for _ in range(args.steps)]
+    sec = sum(times)
+    value = T * args.steps / sec
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_obj(),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+                             "sample": f"each step: fwd+bwd of the last {T} tokens of batch 0 (all groups)"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def config_obj():
+    w = PREFILL
+    return {"workload": f"{w.name} HSA fwd+bwd: B={w.B} L={w.L} S={w.S} Hq={w.Hq} Hkv={w.Hkv} d={w.d} k={w.topk}",
+            "B": w.B, "L": w.L, "S": w.S, "Hq": w.Hq, "Hkv": w.Hkv, "d": w.d, "topk": w.topk,
+            "global_batch": w.B, "seq_len": w.L, "parallelism": "replicas (one batch per GPU)",
+            "l2": "inputs larger than L2 (q, dO, O 512 MiB each; no flush)",
+            "decode_workload": f"{DECODE.name}: memory {DECODE.L} tokens, {DECODE.Bq} queries x Hq={DECODE.Hq}, "
+                               f"Hkv={DECODE.Hkv}, d={DECODE.d}, k={DECODE.topk}"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["hsa", "reference"], default="hsa")
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    import torch.distributed as dist
+
+    if world > 1:
+        import torch
+
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    r = run_gpu(args, rank, world, local_rank)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        log("timing the CPU oracle baseline")
+        cpu = cpu_baseline()
+    if rank == 0:
+        line = {"metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": r["ms_step"], "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_obj(),
+                "roofline": r["roofline"], "cpu_baseline": cpu, "e2e": r["e2e"], "gpu_launches": r["launches"],
+                "clocks": r["clocks"], "kernels": r["kernels"], "decode": r["decode"],
+                "wall_ms_per_step": r["wall_ms_step"]}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,187 @@
+/*
+ * hsa.h — C ABI of the Hierarchical Sparse Attention (HSA) hot path on GB300
+ * (sm_103a). HSA: arXiv 2504.16795, "Hardware-aligned Hierarchical Sparse
+ * Attention for Efficient Long-term Memory Access".
+ *
+ * The operator (one GQA group g of query heads [g*G, (g+1)*G) sharing KV head g):
+ *   K̄_i      = (1/S) sum_{s<S} K_{iS+s}                        chunk summaries
+ *   s_{t,i}  = c_sel * (sum_{h in g} q_{t,h}) · K̄_i,  i < floor(t/S)
+ *   I_t      = top-k of s_{t,.} (ties: lower chunk index), listed by decreasing index
+ *   w_{t,j}  = softmax_j(s_{t,I_j})                              chunk weights
+ *   O_{t,h}  = sum_j w_{t,j} softmax(c_att q_{t,h} K_{I_j}^T) V_{I_j}
+ * and its gradients into q, K, V (through w also into the scores, K̄ and K).
+ *
+ * Conventions for every call
+ *   Layout   Row-major, head dimension contiguous:
+ *              q, O, dO, dq    [B, L, Hq, d]
+ *              K, V, dK, dV    [B, L, Hkv, d]
+ *              K̄ (kbar32/16)   [B, L/S, Hkv, d]   (complete chunks only)
+ *              idx, s_sel, w   [B, L, Hkv, topk]
+ *            Query head h belongs to group h / (Hq/Hkv).
+ *   Types    q, K, V, O, dO, kbar16: bf16 (passed as void*); scores, weights,
+ *            kbar32 and every gradient: fp32; indices: int32.
+ *   Memory   Every pointer is device memory owned by the caller, 16-byte
+ *            aligned. The library never allocates or frees memory and keeps
+ *            no state between calls; scratch comes from the caller's
+ *            workspace (size from hsa_workspace_size).
+ *   Streams  All work is enqueued on `stream`; nothing synchronises the host.
+ *   Errors   Arguments are validated before any launch: a bad argument returns
+ *            HSA_ERR_INVALID_ARG, a shape outside the supported set
+ *            HSA_ERR_UNSUPPORTED, a short workspace HSA_ERR_WORKSPACE, and
+ *            nothing is launched in these cases. A failed launch returns
+ *            HSA_ERR_CUDA. Empty problems (B, L or Bq zero) return HSA_OK and
+ *            launch nothing.
+ *   Support  d in {64, 128}; S = 64; Hq a multiple of Hkv with
+ *            G = Hq/Hkv in {1, 2, 4, 8, 16}; 1 <= topk <= 32;
+ *            B * L * Hkv * topk < 2^31.
+ *   Causality Token t (0-indexed) sees the completed chunks before its own
+ *            chunk (i < t/S); a trailing partial chunk is never selectable.
+ *            Fewer visible chunks than topk: all are selected and the rest of
+ *            the row is padded with idx = -1, s_sel = -inf, w = 0. No visible
+ *            chunk: O = 0 and no gradient.
+ */
+#ifndef HSA_H
+#define HSA_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    HSA_OK = 0,
+    HSA_ERR_INVALID_ARG = 1,
+    HSA_ERR_UNSUPPORTED = 2,
+    HSA_ERR_WORKSPACE = 3,
+    HSA_ERR_CUDA = 4
+} hsa_status_t;
+
+typedef struct {
+    int B, L, Hq, Hkv, d, S, topk;
+    float scale_sel;  /* c_sel; <= 0 selects 1/sqrt((Hq/Hkv) * d) */
+    float scale_attn; /* c_att; <= 0 selects 1/sqrt(d) */
+} hsa_shape_t;
+
+typedef struct {
+    int Bq, Hq, Hkv, d, S, topk;
+    long long n_chunks; /* complete chunks in the memory: the memory holds n_chunks * S tokens */
+    float scale_sel;    /* <= 0 selects 1/sqrt((Hq/Hkv) * d) */
+    float scale_attn;   /* <= 0 selects 1/sqrt(d) */
+} hsa_decode_shape_t;
+
+typedef enum {
+    HSA_OP_SELECT = 1,
+    HSA_OP_INDEX = 2,
+    HSA_OP_FORWARD = 3,
+    HSA_OP_BACKWARD = 4
+} hsa_op_t;
+
+/* Human-readable name of a status code (static storage). */
+const char* hsa_status_string(hsa_status_t status);
+
+/* Library version: major * 10000 + minor * 100 + patch. */
+int hsa_version(void);
+
+/* Number of CUDA kernels this library has launched since it was loaded (a
+ * diagnostic for launch accounting; counts launches, not their completion). */
+unsigned long long hsa_kernel_launches(void);
+
+/* Workspace bytes that `op` needs for `shape` (0 when it needs none). Returns
+ * 0 too for an invalid shape; the call itself then reports the error. */
+size_t hsa_workspace_size(int op, const hsa_shape_t* shape);
+
+/* Workspace bytes of hsa_decode for `shape`. */
+size_t hsa_decode_workspace_size(const hsa_decode_shape_t* shape);
+
+/*
+ * Chunk mean pool (§3.1 "Chunk Selection": K̄_i is the mean-pooled chunk
+ * representation; Appendix A, Eq. 3: q·K̄_c equals the mean of the chunk's
+ * token logits).
+ *   K      [B, L, Hkv, d] bf16, input.
+ *   kbar32 [B, L/S, Hkv, d] fp32, output: fp32 sum in token order, divided by S.
+ *   kbar16 [B, L/S, Hkv, d] bf16, output (may be NULL): round-to-nearest-even of kbar32.
+ * Rows of a trailing partial chunk are not read.
+ */
+hsa_status_t hsa_chunk_pool(const hsa_shape_t* shape, const void* K, float* kbar32, void* kbar16,
+                            cudaStream_t stream);
+
+/*
+ * Top-k chunk selection per token and GQA group (§3.1 "Chunk Selection": the
+ * score q̂·K̂/sqrt(d_g) over visible chunks and I = {i : rank(s_i) < k}; §3.1.1
+ * "Chunk Weights": I' lists the chosen chunks by decreasing index).
+ *   q      [B, L, Hq, d] bf16, input.
+ *   kbar32 [B, L/S, Hkv, d] fp32, input (from hsa_chunk_pool).
+ *   idx    [B, L, Hkv, topk] int32, output: chosen chunks, decreasing index, -1 padded.
+ *   s_sel  [B, L, Hkv, topk] fp32, output: their scores, -inf padded.
+ * Scores are fp32: q̂ = fp32 sum of the group's heads in head order,
+ * dot = fused multiply-add chain over d in order, s = dot * c_sel. The score
+ * matrix is never written to memory. ws may be NULL when the workspace size
+ * is 0.
+ */
+hsa_status_t hsa_select_topk(const hsa_shape_t* shape, const void* q, const float* kbar32, int32_t* idx,
+                             float* s_sel, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/*
+ * Inverse selection index (replaces the mask M and rank R of §3.1.2, used by
+ * Algorithm 3): for every (b, g, chunk i) the list of selection slots that
+ * chose it, as a CSR over keys key = (b * Hkv + g) * (L/S) + i:
+ *   offsets [B*Hkv*(L/S) + 1] int32, output: entries of key k are
+ *           entries[offsets[k] .. offsets[k+1]).
+ *   entries [B*L*Hkv*topk] int32, output (capacity): the flat slot index
+ *           p = ((b*L + t)*Hkv + g)*topk + j of idx, in increasing p (so in
+ *           increasing token order) within each key.
+ * Deterministic (a stable radix sort); needs workspace HSA_OP_INDEX.
+ */
+hsa_status_t hsa_build_index(const hsa_shape_t* shape, const int32_t* idx, int32_t* offsets, int32_t* entries,
+                             void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/*
+ * Hierarchical attention forward (§3.1.1 "Hierarchical Attention", Algorithm
+ * 1; chunk weights by softmax over the selected scores, the "w/o s.b."
+ * variant of §4.1).
+ *   q [B,L,Hq,d], K, V [B,L,Hkv,d] bf16; idx, s_sel from hsa_select_topk;
+ *   offsets, entries from hsa_build_index (same idx).
+ *   O [B,L,Hq,d] bf16, output.  w [B,L,Hkv,topk] fp32, output (0 at padded slots).
+ * Needs workspace HSA_OP_FORWARD. Chunk-major: each (b, g, chunk) tile of K
+ * and V is read once and shared by every query head that selected it.
+ */
+hsa_status_t hsa_forward(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
+                         const int32_t* idx, const float* s_sel, const int32_t* offsets, const int32_t* entries,
+                         void* O, float* w, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/*
+ * Backward (Algorithm 2: dq and the chunk-weight gradient; Algorithm 3: dK,
+ * dV per chunk; Appendix A: the chunk weights carry gradient into the
+ * selection scores, hence into q, K̄ and, through the mean pool, K).
+ *   Inputs as in hsa_forward plus kbar32, the forward's w and O, and dO [B,L,Hq,d] bf16.
+ *   dq [B,L,Hq,d], dK, dV [B,L,Hkv,d] fp32, outputs (fully written).
+ * Deterministic: every dK/dV row is owned by one thread block that walks its
+ * chunk's entries in index order; no floating-point atomics.
+ * Needs workspace HSA_OP_BACKWARD.
+ */
+hsa_status_t hsa_backward(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
+                          const float* kbar32, const int32_t* idx, const float* w, const void* O, const void* dO,
+                          const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,
+                          void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/*
+ * Decode against a resident memory (§3.2 "Inference": only the chunk
+ * summaries are scanned on every step, then the k selected chunks are
+ * fetched). One query token per batch row; all n_chunks chunks are visible.
+ *   q      [Bq, Hq, d] bf16.
+ *   K_mem, V_mem [n_chunks*S, Hkv, d] bf16 (the memory).
+ *   kbar32 [n_chunks, Hkv, d] fp32 (hsa_chunk_pool of K_mem with B = 1).
+ *   O [Bq, Hq, d] bf16, idx, s_sel, w [Bq, Hkv, topk], outputs.
+ * Needs workspace hsa_decode_workspace_size.
+ */
+hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const void* K_mem, const void* V_mem,
+                        const float* kbar32, void* O, int32_t* idx, float* s_sel, float* w, void* ws,
+                        size_t ws_bytes, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* HSA_H */

@@ -41,10 +41,10 @@ def lib():
         vp, ci, cd = ctypes.c_void_p, ctypes.c_int, ctypes.c_double
         i64 = ctypes.c_int64
         L.hsa_oracle_pool.argtypes = [vp, ci, ci, ci, ci, ci, ci, vp]
-        L.hsa_oracle_select.argtypes = [vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, ci, vp, vp, vp]
-        L.hsa_oracle_forward.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, vp, vp]
+        L.hsa_oracle_select.argtypes = [vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, ci, vp, vp, vp, vp]
+        L.hsa_oracle_forward.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, vp, vp, vp]
         L.hsa_oracle_backward.argtypes = [vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, cd,
-                                          vp, vp, vp, vp, vp]
+                                          vp, vp, vp, vp, vp, vp]
         L.hsa_oracle_decode_select.argtypes = [vp, vp, i64, ci, ci, ci, ci, ci, cd, ci, vp, vp, vp]
         L.hsa_oracle_decode_attend.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, cd, vp, vp]
         for f in (L.hsa_oracle_pool, L.hsa_oracle_select, L.hsa_oracle_forward, L.hsa_oracle_backward,
@@ -72,6 +72,14 @@ def _p(x):
     return ctypes.c_void_p(x.ctypes.data) if x is not None else None
 
 
+def _mask(token_mask, B, L):
+    if token_mask is None:
+        return None
+    m = np.ascontiguousarray(token_mask, dtype=np.uint8)
+    assert m.shape == (B, L)
+    return m
+
+
 def pool(K, S, f32=False):
     """K [B, L, Hkv, d] -> K̄ [B, L//S, Hkv, d]."""
     K = _f64(K)
@@ -81,23 +89,26 @@ def pool(K, S, f32=False):
     return kbar
 
 
-def select(q, kbar, S, topk, scale_sel=None, f32=False):
-    """q [B, L, Hq, d], K̄ [B, L//S, Hkv, d] -> idx [B,L,Hkv,k] int32, s_sel, gap [B,L,Hkv]."""
+def select(q, kbar, S, topk, scale_sel=None, f32=False, token_mask=None):
+    """q [B, L, Hq, d], K̄ [B, L//S, Hkv, d] -> idx [B,L,Hkv,k] int32, s_sel, gap [B,L,Hkv].
+
+    token_mask [B, L] (optional): rows outside it are left as idx = -1, s_sel = 0, gap = 0."""
     q, kbar = _f64(q), _f64(kbar)
     B, L, Hq, d = q.shape
     Hkv = kbar.shape[2]
     if scale_sel is None:
         scale_sel = default_scales(Hq // Hkv, d)[0]
-    idx = np.zeros((B, L, Hkv, topk), dtype=np.int32)
+    idx = np.full((B, L, Hkv, topk), -1, dtype=np.int32)
     s_sel = np.zeros((B, L, Hkv, topk))
     gap = np.zeros((B, L, Hkv))
-    lib().hsa_oracle_select(_p(q), _p(kbar), B, L, Hq, Hkv, d, S, topk, float(scale_sel), int(f32), _p(idx),
+    m = _mask(token_mask, B, L)
+    lib().hsa_oracle_select(_p(q), _p(kbar), B, L, Hq, Hkv, d, S, topk, float(scale_sel), int(f32), _p(m), _p(idx),
                             _p(s_sel), _p(gap))
     return idx, s_sel, gap
 
 
-def forward(q, K, V, idx, s_sel, S, scale_attn=None):
-    """-> O [B, L, Hq, d], w [B, L, Hkv, k]."""
+def forward(q, K, V, idx, s_sel, S, scale_attn=None, token_mask=None):
+    """-> O [B, L, Hq, d], w [B, L, Hkv, k] (rows outside token_mask stay 0)."""
     q, K, V, s_sel = _f64(q), _f64(K), _f64(V), _f64(s_sel)
     idx = np.ascontiguousarray(idx, dtype=np.int32)
     B, L, Hq, d = q.shape
@@ -107,13 +118,14 @@ def forward(q, K, V, idx, s_sel, S, scale_attn=None):
         scale_attn = default_scales(Hq // Hkv, d)[1]
     O = np.zeros_like(q)
     w = np.zeros((B, L, Hkv, topk))
+    m = _mask(token_mask, B, L)
     lib().hsa_oracle_forward(_p(q), _p(K), _p(V), _p(idx), _p(s_sel), B, L, Hq, Hkv, d, S, topk, float(scale_attn),
-                             _p(O), _p(w))
+                             _p(m), _p(O), _p(w))
     return O, w
 
 
-def backward(q, K, V, kbar, idx, s_sel, dO, S, scale_sel=None, scale_attn=None):
-    """-> dict(dq, dK, dV, dkbar, ds)."""
+def backward(q, K, V, kbar, idx, s_sel, dO, S, scale_sel=None, scale_attn=None, token_mask=None):
+    """-> dict(dq, dK, dV, dkbar, ds); with token_mask only those tokens contribute."""
     q, K, V, kbar, s_sel, dO = map(_f64, (q, K, V, kbar, s_sel, dO))
     idx = np.ascontiguousarray(idx, dtype=np.int32)
     B, L, Hq, d = q.shape
@@ -125,8 +137,9 @@ def backward(q, K, V, kbar, idx, s_sel, dO, S, scale_sel=None, scale_attn=None):
     dq, dK, dV = np.zeros_like(q), np.zeros_like(K), np.zeros_like(V)
     dkbar = np.zeros_like(kbar)
     ds = np.zeros((B, L, Hkv, topk))
+    m = _mask(token_mask, B, L)
     lib().hsa_oracle_backward(_p(q), _p(K), _p(V), _p(kbar), _p(idx), _p(s_sel), _p(dO), B, L, Hq, Hkv, d, S, topk,
-                              float(scale_sel), float(scale_attn), _p(dq), _p(dK), _p(dV), _p(dkbar), _p(ds))
+                              float(scale_sel), float(scale_attn), _p(m), _p(dq), _p(dK), _p(dV), _p(dkbar), _p(ds))
     return dict(dq=dq, dK=dK, dV=dV, dkbar=dkbar, ds=ds)
 
 

@@ -156,9 +156,11 @@ static void group_query(const double* q_row, int G, int g, int d, int f32, doubl
 /* ------------------------------------------------------------------ chunk selection
  * q [B, L, Hq, d], kbar [B, L/S, Hkv, d] -> idx [B, L, Hkv, topk] int32,
  * s_sel [B, L, Hkv, topk]; gap (optional) [B, L, Hkv] = k-th minus (k+1)-th score.
+ * token_mask (optional, [B, L]): only rows whose mask byte is nonzero are computed.
  */
 void hsa_oracle_select(const double* q, const double* kbar, int B, int L, int Hq, int Hkv, int d, int S,
-                       int topk, double scale_sel, int f32, int32_t* idx, double* s_sel, double* gap) {
+                       int topk, double scale_sel, int f32, const uint8_t* token_mask, int32_t* idx, double* s_sel,
+                       double* gap) {
     const int Nc = L / S, G = Hq / Hkv;
 #pragma omp parallel
     {
@@ -167,6 +169,7 @@ void hsa_oracle_select(const double* q, const double* kbar, int B, int L, int Hq
 #pragma omp for collapse(2) schedule(dynamic, 16)
         for (int b = 0; b < B; ++b)
             for (int t = 0; t < L; ++t) {
+                if (token_mask && !token_mask[(int64_t)b * L + t]) continue;
                 const int64_t nvis = (t / S) < Nc ? (t / S) : Nc;
                 const double* q_row = q + at4(b, t, 0, 0, L, Hq, d);
                 for (int g = 0; g < Hkv; ++g) {
@@ -220,10 +223,11 @@ static void chunk_attention(const double* qh, const double* Kc, const double* Vc
 
 /* ------------------------------------------------------------------ forward
  * O [B, L, Hq, d] = sum_j w_j Attn(q_t, K_{I_j}, V_{I_j}); w [B, L, Hkv, topk].
+ * token_mask (optional, [B, L]): only those tokens are computed.
  */
 void hsa_oracle_forward(const double* q, const double* K, const double* V, const int32_t* idx,
                         const double* s_sel, int B, int L, int Hq, int Hkv, int d, int S, int topk,
-                        double scale_attn, double* O, double* w) {
+                        double scale_attn, const uint8_t* token_mask, double* O, double* w) {
     const int G = Hq / Hkv;
 #pragma omp parallel
     {
@@ -233,6 +237,7 @@ void hsa_oracle_forward(const double* q, const double* K, const double* V, const
         for (int b = 0; b < B; ++b)
             for (int t = 0; t < L; ++t)
                 for (int g = 0; g < Hkv; ++g) {
+                    if (token_mask && !token_mask[(int64_t)b * L + t]) continue;
                     const int64_t o = at4(b, t, g, 0, L, Hkv, topk);
                     const int keff = count_selected(idx + o, topk);
                     chunk_weights(s_sel + o, keff, topk, w + o);
@@ -269,11 +274,15 @@ void hsa_oracle_forward(const double* q, const double* K, const double* V, const
  *   ds_j     = w_j (dw_j - sum_j' w_j' dw_j')        (softmax over the selected scores)
  *   dq_h    += c_sel sum_j ds_j K̄_{I_j} (every head of the group) ; dK̄_{I_j} += c_sel ds_j q̂
  *   dK_{iS+s} += dK̄_i / S                             (mean pool)
+ * token_mask (optional, [B, L]): only those tokens are processed, so dq rows
+ * of other tokens stay 0 and dK, dV, dK̄ collect the masked tokens'
+ * contributions only (exact for a chunk whose selecting tokens are all in
+ * the mask).
  */
 void hsa_oracle_backward(const double* q, const double* K, const double* V, const double* kbar,
                          const int32_t* idx, const double* s_sel, const double* dO, int B, int L, int Hq,
-                         int Hkv, int d, int S, int topk, double scale_sel, double scale_attn, double* dq,
-                         double* dK, double* dV, double* dkbar, double* ds) {
+                         int Hkv, int d, int S, int topk, double scale_sel, double scale_attn,
+                         const uint8_t* token_mask, double* dq, double* dK, double* dV, double* dkbar, double* ds) {
     const int G = Hq / Hkv, Nc = L / S;
 #pragma omp parallel for collapse(2) schedule(dynamic, 1)
     for (int b = 0; b < B; ++b)
@@ -292,6 +301,7 @@ void hsa_oracle_backward(const double* q, const double* K, const double* V, cons
                     dV[at4(b, t, g, e, L, Hkv, d)] = 0.0;
                 }
             for (int t = 0; t < L; ++t) {
+                if (token_mask && !token_mask[(int64_t)b * L + t]) continue;
                 const int64_t o = at4(b, t, g, 0, L, Hkv, topk);
                 const int32_t* I = idx + o;
                 const int keff = count_selected(I, topk);

@@ -1,0 +1,247 @@
+// C ABI of the HSA hot path: argument validation, workspace sizing and
+// dispatch to the kernels. Nothing here allocates device memory; every check
+// runs before the first launch.
+#include <atomic>
+#include <cmath>
+#include <cstdint>
+
+#include "common.cuh"
+
+namespace hsa {
+static std::atomic<unsigned long long> g_launches{0};
+void note_launches(unsigned long long n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+}  // namespace hsa
+
+namespace {
+
+using hsa::Dims;
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+bool pow2_group(int G) { return G == 1 || G == 2 || G == 4 || G == 8 || G == 16; }
+
+// Validates a prefill shape; fills Dims on success.
+hsa_status_t resolve(const hsa_shape_t* s, Dims* out) {
+  if (s == nullptr) return HSA_ERR_INVALID_ARG;
+  if (s->B < 0 || s->L < 0 || s->Hq <= 0 || s->Hkv <= 0 || s->d <= 0 || s->S <= 0 || s->topk <= 0)
+    return HSA_ERR_INVALID_ARG;
+  if (s->Hq % s->Hkv != 0) return HSA_ERR_INVALID_ARG;
+  if (std::isnan(s->scale_sel) || std::isnan(s->scale_attn) || std::isinf(s->scale_sel) ||
+      std::isinf(s->scale_attn))
+    return HSA_ERR_INVALID_ARG;
+  const int G = s->Hq / s->Hkv;
+  if (!pow2_group(G)) return HSA_ERR_UNSUPPORTED;
+  if (s->d != 64 && s->d != 128) return HSA_ERR_UNSUPPORTED;
+  if (s->S != hsa::kChunk) return HSA_ERR_UNSUPPORTED;
+  if (s->topk > 32) return HSA_ERR_UNSUPPORTED;
+  const long long slots = (long long)s->B * s->L * s->Hkv * s->topk;
+  if (slots >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
+  const long long rows = (long long)s->B * s->L * s->Hq;
+  if (rows >= (1LL << 40)) return HSA_ERR_UNSUPPORTED;
+  Dims D;
+  D.B = s->B;
+  D.L = s->L;
+  D.Hq = s->Hq;
+  D.Hkv = s->Hkv;
+  D.d = s->d;
+  D.S = s->S;
+  D.topk = s->topk;
+  D.G = G;
+  D.Nc = s->L / s->S;
+  D.scale_sel = s->scale_sel > 0.f ? s->scale_sel : (float)(1.0 / std::sqrt((double)G * s->d));
+  D.scale_attn = s->scale_attn > 0.f ? s->scale_attn : (float)(1.0 / std::sqrt((double)s->d));
+  *out = D;
+  return HSA_OK;
+}
+
+bool empty(const Dims& D) { return D.B == 0 || D.L == 0; }
+
+hsa_status_t cuda_status(cudaError_t e) { return e == cudaSuccess ? HSA_OK : HSA_ERR_CUDA; }
+
+#define HSA_REQUIRE_PTR(p)                          \
+  do {                                              \
+    if ((p) == nullptr || !aligned16(p)) return HSA_ERR_INVALID_ARG; \
+  } while (0)
+
+}  // namespace
+
+extern "C" {
+
+const char* hsa_status_string(hsa_status_t status) {
+  switch (status) {
+    case HSA_OK: return "HSA_OK";
+    case HSA_ERR_INVALID_ARG: return "HSA_ERR_INVALID_ARG: null, misaligned or inconsistent argument";
+    case HSA_ERR_UNSUPPORTED: return "HSA_ERR_UNSUPPORTED: shape outside the supported set";
+    case HSA_ERR_WORKSPACE: return "HSA_ERR_WORKSPACE: workspace missing or too small";
+    case HSA_ERR_CUDA: return "HSA_ERR_CUDA: a kernel launch failed";
+  }
+  return "HSA_ERR_UNKNOWN";
+}
+
+int hsa_version(void) { return 100; }
+
+unsigned long long hsa_kernel_launches(void) { return hsa::g_launches.load(std::memory_order_relaxed); }
+
+size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {
+  Dims D;
+  if (resolve(shape, &D) != HSA_OK) return 0;
+  if (empty(D)) return 0;
+  switch (op) {
+    case HSA_OP_SELECT: return 0;
+    case HSA_OP_INDEX: return hsa::index_workspace(D);
+    case HSA_OP_FORWARD: return hsa::forward_workspace(D);
+    case HSA_OP_BACKWARD: return hsa::backward_workspace(D);
+  }
+  return 0;
+}
+
+hsa_status_t hsa_chunk_pool(const hsa_shape_t* shape, const void* K, float* kbar32, void* kbar16,
+                            cudaStream_t stream) {
+  Dims D;
+  hsa_status_t st = resolve(shape, &D);
+  if (st != HSA_OK) return st;
+  if (empty(D) || D.Nc == 0) return HSA_OK;
+  HSA_REQUIRE_PTR(K);
+  HSA_REQUIRE_PTR(kbar32);
+  if (kbar16 != nullptr && !aligned16(kbar16)) return HSA_ERR_INVALID_ARG;
+  return cuda_status(hsa::launch_pool(D, K, kbar32, kbar16, stream));
+}
+
+hsa_status_t hsa_select_topk(const hsa_shape_t* shape, const void* q, const float* kbar32, int32_t* idx,
+                             float* s_sel, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  Dims D;
+  hsa_status_t st = resolve(shape, &D);
+  if (st != HSA_OK) return st;
+  if (empty(D)) return HSA_OK;
+  HSA_REQUIRE_PTR(q);
+  HSA_REQUIRE_PTR(idx);
+  HSA_REQUIRE_PTR(s_sel);
+  if (D.Nc > 0) HSA_REQUIRE_PTR(kbar32);
+  (void)ws;
+  (void)ws_bytes;
+  return cuda_status(hsa::launch_select(D, q, kbar32, idx, s_sel, stream));
+}
+
+hsa_status_t hsa_build_index(const hsa_shape_t* shape, const int32_t* idx, int32_t* offsets, int32_t* entries,
+                             void* ws, size_t ws_bytes, cudaStream_t stream) {
+  Dims D;
+  hsa_status_t st = resolve(shape, &D);
+  if (st != HSA_OK) return st;
+  HSA_REQUIRE_PTR(offsets);
+  if (empty(D)) return HSA_OK;
+  HSA_REQUIRE_PTR(idx);
+  HSA_REQUIRE_PTR(entries);
+  const size_t need = hsa::index_workspace(D);
+  if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
+  return cuda_status(hsa::launch_index(D, idx, offsets, entries, ws, stream));
+}
+
+hsa_status_t hsa_forward(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
+                         const int32_t* idx, const float* s_sel, const int32_t* offsets, const int32_t* entries,
+                         void* O, float* w, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  Dims D;
+  hsa_status_t st = resolve(shape, &D);
+  if (st != HSA_OK) return st;
+  if (empty(D)) return HSA_OK;
+  HSA_REQUIRE_PTR(q);
+  HSA_REQUIRE_PTR(K);
+  HSA_REQUIRE_PTR(V);
+  HSA_REQUIRE_PTR(idx);
+  HSA_REQUIRE_PTR(s_sel);
+  HSA_REQUIRE_PTR(offsets);
+  HSA_REQUIRE_PTR(entries);
+  HSA_REQUIRE_PTR(O);
+  HSA_REQUIRE_PTR(w);
+  const size_t need = hsa::forward_workspace(D);
+  if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
+  return cuda_status(hsa::launch_forward(D, q, K, V, idx, s_sel, offsets, entries, O, w, ws, stream));
+}
+
+hsa_status_t hsa_backward(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
+                          const float* kbar32, const int32_t* idx, const float* w, const void* O, const void* dO,
+                          const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,
+                          void* ws, size_t ws_bytes, cudaStream_t stream) {
+  Dims D;
+  hsa_status_t st = resolve(shape, &D);
+  if (st != HSA_OK) return st;
+  if (empty(D)) return HSA_OK;
+  HSA_REQUIRE_PTR(q);
+  HSA_REQUIRE_PTR(K);
+  HSA_REQUIRE_PTR(V);
+  if (D.Nc > 0) HSA_REQUIRE_PTR(kbar32);
+  HSA_REQUIRE_PTR(idx);
+  HSA_REQUIRE_PTR(w);
+  HSA_REQUIRE_PTR(O);
+  HSA_REQUIRE_PTR(dO);
+  HSA_REQUIRE_PTR(offsets);
+  HSA_REQUIRE_PTR(entries);
+  HSA_REQUIRE_PTR(dq);
+  HSA_REQUIRE_PTR(dK);
+  HSA_REQUIRE_PTR(dV);
+  const size_t need = hsa::backward_workspace(D);
+  if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
+  return cuda_status(
+      hsa::launch_backward(D, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq, dK, dV, ws, stream));
+}
+
+namespace {
+hsa_status_t resolve_decode(const hsa_decode_shape_t* s, hsa::DecodeDims* out) {
+  if (s == nullptr) return HSA_ERR_INVALID_ARG;
+  if (s->Bq < 0 || s->Hq <= 0 || s->Hkv <= 0 || s->d <= 0 || s->S <= 0 || s->topk <= 0 || s->n_chunks < 0)
+    return HSA_ERR_INVALID_ARG;
+  if (s->Hq % s->Hkv != 0) return HSA_ERR_INVALID_ARG;
+  if (std::isnan(s->scale_sel) || std::isnan(s->scale_attn) || std::isinf(s->scale_sel) ||
+      std::isinf(s->scale_attn))
+    return HSA_ERR_INVALID_ARG;
+  const int G = s->Hq / s->Hkv;
+  if (!pow2_group(G)) return HSA_ERR_UNSUPPORTED;
+  if (s->d != 64 && s->d != 128) return HSA_ERR_UNSUPPORTED;
+  if (s->S != hsa::kChunk) return HSA_ERR_UNSUPPORTED;
+  if (s->topk > 32) return HSA_ERR_UNSUPPORTED;
+  if (s->n_chunks >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
+  if ((long long)s->Bq * s->Hkv * s->topk >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
+  hsa::DecodeDims D;
+  D.Bq = s->Bq;
+  D.Hq = s->Hq;
+  D.Hkv = s->Hkv;
+  D.d = s->d;
+  D.S = s->S;
+  D.topk = s->topk;
+  D.G = G;
+  D.Nc = s->n_chunks;
+  D.scale_sel = s->scale_sel > 0.f ? s->scale_sel : (float)(1.0 / std::sqrt((double)G * s->d));
+  D.scale_attn = s->scale_attn > 0.f ? s->scale_attn : (float)(1.0 / std::sqrt((double)s->d));
+  *out = D;
+  return HSA_OK;
+}
+}  // namespace
+
+size_t hsa_decode_workspace_size(const hsa_decode_shape_t* shape) {
+  hsa::DecodeDims D;
+  if (resolve_decode(shape, &D) != HSA_OK || D.Bq == 0) return 0;
+  return hsa::decode_workspace(D);
+}
+
+hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const void* K_mem, const void* V_mem,
+                        const float* kbar32, void* O, int32_t* idx, float* s_sel, float* w, void* ws,
+                        size_t ws_bytes, cudaStream_t stream) {
+  hsa::DecodeDims D;
+  hsa_status_t st = resolve_decode(shape, &D);
+  if (st != HSA_OK) return st;
+  if (D.Bq == 0) return HSA_OK;
+  HSA_REQUIRE_PTR(q);
+  HSA_REQUIRE_PTR(O);
+  HSA_REQUIRE_PTR(idx);
+  HSA_REQUIRE_PTR(s_sel);
+  HSA_REQUIRE_PTR(w);
+  if (D.Nc > 0) {
+    HSA_REQUIRE_PTR(K_mem);
+    HSA_REQUIRE_PTR(V_mem);
+    HSA_REQUIRE_PTR(kbar32);
+  }
+  const size_t need = hsa::decode_workspace(D);
+  if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+  return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, ws, stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,191 @@
+// Internal helpers shared by the HSA CUDA kernels (sm_103a).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "hsa.h"
+
+namespace hsa {
+
+constexpr int kChunk = 64;  // S: the only chunk size the kernels are built for
+constexpr int kWarp = 32;
+
+// Resolved shape shared by host launchers.
+struct Dims {
+  int B, L, Hq, Hkv, d, S, topk, G, Nc;
+  float scale_sel, scale_attn;
+  long long slots() const { return (long long)B * L * Hkv * topk; }
+  long long keys() const { return (long long)B * Hkv * Nc; }
+};
+
+// ------------------------------------------------------------------ bf16
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+__device__ __forceinline__ float bf16_bits_to_f32(uint16_t v) { return __uint_as_float(((uint32_t)v) << 16); }
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+__device__ __forceinline__ uint16_t f32_to_bf16_bits(float x) {
+  __nv_bfloat16 h = __float2bfloat16_rn(x);
+  return *reinterpret_cast<uint16_t*>(&h);
+}
+
+// ------------------------------------------------------------------ ranking keys
+// A 64-bit key whose unsigned order is the rank order of the paper's top-k:
+// larger score first, equal scores by lower chunk index. 0 never beats a real key.
+__device__ __forceinline__ uint32_t order_bits(float s) {
+  uint32_t u = __float_as_uint(s);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float order_bits_to_float(uint32_t o) {
+  uint32_t u = (o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o;
+  return __uint_as_float(u);
+}
+__device__ __forceinline__ unsigned long long rank_key(float s, uint32_t chunk) {
+  return ((unsigned long long)order_bits(s) << 32) | (unsigned long long)(0xFFFFFFFFu - chunk);
+}
+__device__ __forceinline__ uint32_t key_chunk(unsigned long long k) {
+  return 0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFull);
+}
+__device__ __forceinline__ float key_score(unsigned long long k) { return order_bits_to_float((uint32_t)(k >> 32)); }
+
+// A warp holds a running top-k list, lane l keeping the key of rank l (l < k,
+// descending). Insert x (already known to beat the current k-th key).
+__device__ __forceinline__ void warp_topk_insert(unsigned long long& mine, unsigned long long x, int k, int lane) {
+  unsigned above = __ballot_sync(0xFFFFFFFFu, lane < k && mine > x);
+  int pos = __popc(above);
+  unsigned long long up = __shfl_up_sync(0xFFFFFFFFu, mine, 1);
+  if (lane < k) {
+    if (lane == pos) mine = x;
+    else if (lane > pos) mine = up;
+  }
+}
+
+// Offer one candidate per lane to the running list; threshold = current k-th key.
+__device__ __forceinline__ void warp_topk_offer(unsigned long long& mine, unsigned long long cand, int k, int lane) {
+  unsigned long long thr = __shfl_sync(0xFFFFFFFFu, mine, k - 1);
+  unsigned m = __ballot_sync(0xFFFFFFFFu, cand > thr);
+  while (m) {
+    int src = __ffs(m) - 1;
+    unsigned long long x = __shfl_sync(0xFFFFFFFFu, cand, src);
+    warp_topk_insert(mine, x, k, lane);
+    thr = __shfl_sync(0xFFFFFFFFu, mine, k - 1);
+    m &= ~(1u << src);
+    m &= __ballot_sync(0xFFFFFFFFu, cand > thr);
+  }
+}
+
+// Write a finished list (ranks 0..k-1, valid where key != 0) as idx/s_sel
+// ordered by decreasing chunk index, padding with -1 / -inf.
+__device__ __forceinline__ int warp_emit_selection(unsigned long long mine, int k, int lane, int32_t* idx_out,
+                                                   float* s_out) {
+  bool valid = lane < k && mine != 0ull;
+  unsigned vm = __ballot_sync(0xFFFFFFFFu, valid);
+  int keff = __popc(vm);  // valid entries occupy lanes 0..keff-1
+  uint32_t c = valid ? key_chunk(mine) : 0u;
+  int rank = 0;
+  for (int l = 0; l < keff; ++l) {
+    uint32_t other = __shfl_sync(0xFFFFFFFFu, c, l);
+    rank += (other > c) ? 1 : 0;
+  }
+  if (valid) {
+    idx_out[rank] = (int32_t)c;
+    s_out[rank] = key_score(mine);
+  } else if (lane < k) {
+    idx_out[lane] = -1;
+    s_out[lane] = -__int_as_float(0x7f800000);
+  }
+  return keff;
+}
+
+// ------------------------------------------------------------------ async copies / tensor-core fragments
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+// D = A(16x16, row) * B(16x8, col) + D, bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Byte offset of element (row, col) in a shared tile of bf16 rows of `cols`
+// elements, with the 16-byte chunks of each row XOR-swizzled by (row & 7) so
+// that ldmatrix reads of 8 consecutive rows hit distinct banks.
+template <int COLS>
+__device__ __forceinline__ uint32_t swz(int row, int col) {
+  return (uint32_t)(row * (COLS * 2) + ((((col >> 3) ^ (row & 7))) << 4) + ((col & 7) << 1));
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+  return v;
+}
+
+// ------------------------------------------------------------------ host helpers
+// Number of kernels this library has launched since it was loaded.
+void note_launches(unsigned long long n);
+
+inline int grid_cap(long long blocks, long long cap = 152LL * 64) {
+  if (blocks < 1) return 1;
+  return (int)(blocks < cap ? blocks : cap);
+}
+
+}  // namespace hsa
+
+// Launchers implemented in the kernel translation units; all return cudaError_t.
+namespace hsa {
+cudaError_t launch_pool(const Dims& D, const void* K, float* kbar32, void* kbar16, cudaStream_t st);
+cudaError_t launch_select(const Dims& D, const void* q, const float* kbar32, int32_t* idx, float* s_sel,
+                          cudaStream_t st);
+size_t index_workspace(const Dims& D);
+cudaError_t launch_index(const Dims& D, const int32_t* idx, int32_t* offsets, int32_t* entries, void* ws,
+                         cudaStream_t st);
+size_t forward_workspace(const Dims& D);
+cudaError_t launch_forward(const Dims& D, const void* q, const void* K, const void* V, const int32_t* idx,
+                           const float* s_sel, const int32_t* offsets, const int32_t* entries, void* O, float* w,
+                           void* ws, cudaStream_t st);
+size_t backward_workspace(const Dims& D);
+cudaError_t launch_backward(const Dims& D, const void* q, const void* K, const void* V, const float* kbar32,
+                            const int32_t* idx, const float* w, const void* O, const void* dO,
+                            const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,
+                            void* ws, cudaStream_t st);
+struct DecodeDims {
+  int Bq, Hq, Hkv, d, S, topk, G;
+  long long Nc;
+  float scale_sel, scale_attn;
+};
+size_t decode_workspace(const DecodeDims& D);
+cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
+                          void* O, int32_t* idx, float* s_sel, float* w, void* ws, cudaStream_t st);
+}  // namespace hsa

@@ -1,0 +1,262 @@
+// Inverse selection index: for every (b, g, chunk) the selection slots that
+// chose it. This replaces the dense mask M and rank R of the paper's backward
+// (§3.1.2, Algorithm 3 scans every token for every chunk) with a CSR built by
+// a stable LSD radix sort of the slots by key (b*Hkv + g)*Nc + chunk, so each
+// key's list comes out in increasing slot (token) order, deterministically.
+//
+//   pass p (8-bit digit p):   per-tile digit histogram -> exclusive scan over
+//                             (digit, tile) -> stable scatter within each tile
+//   offsets:                  per-key counts -> exclusive scan
+// Padded slots (idx = -1) get the sentinel key B*Hkv*Nc and sort to the end.
+#include "common.cuh"
+
+namespace hsa {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kItems = 8;  // per thread
+constexpr int kTile = kThreads * kItems;
+constexpr int kScanThreads = 1024;
+constexpr int kScanItems = 4;
+constexpr int kScanTile = kScanThreads * kScanItems;
+
+struct KeyMap {
+  const int32_t* idx;
+  int L, Hkv, topk, Nc;
+  uint32_t sentinel;
+  __device__ __forceinline__ uint32_t key(long long p) const {
+    const int c = idx[p];
+    if (c < 0 || c >= Nc) return sentinel;  // padding (or an out-of-range index) is never listed
+    const long long g = (p / topk) % Hkv;
+    const long long b = p / ((long long)topk * Hkv * L);
+    return (uint32_t)((b * Hkv + g) * Nc + c);
+  }
+};
+
+// Digit histogram of one tile, written digit-major: hist[digit * n_tiles + tile].
+__global__ void __launch_bounds__(kThreads) radix_hist_kernel(KeyMap km, const uint32_t* __restrict__ keys_in,
+                                                              long long n, int shift, uint32_t* __restrict__ hist,
+                                                              int n_tiles) {
+  __shared__ uint32_t h[256];
+  h[threadIdx.x] = 0;
+  __syncthreads();
+  const long long base = (long long)blockIdx.x * kTile;
+#pragma unroll
+  for (int r = 0; r < kItems; ++r) {
+    const long long p = base + r * kThreads + threadIdx.x;
+    if (p < n) {
+      const uint32_t k = keys_in ? keys_in[p] : km.key(p);
+      atomicAdd(&h[(k >> shift) & 255u], 1u);
+    }
+  }
+  __syncthreads();
+  hist[(long long)threadIdx.x * n_tiles + blockIdx.x] = h[threadIdx.x];
+}
+
+// Stable scatter: items are visited in their input order (round r covers
+// items base + r*256 .. base + r*256 + 255 in thread order); the rank of an
+// item among equal digits is (items of that digit in earlier rounds) +
+// (in earlier warps of this round) + (in earlier lanes of this warp).
+__global__ void __launch_bounds__(kThreads) radix_scatter_kernel(KeyMap km, const uint32_t* __restrict__ keys_in,
+                                                                 const int32_t* __restrict__ vals_in, long long n,
+                                                                 int shift, const uint32_t* __restrict__ base_off,
+                                                                 int n_tiles, uint32_t* __restrict__ keys_out,
+                                                                 int32_t* __restrict__ vals_out) {
+  __shared__ uint32_t run[256];
+  __shared__ uint32_t cnt[kThreads / 32][256];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  run[tid] = base_off[(long long)tid * n_tiles + blockIdx.x];
+  const long long base = (long long)blockIdx.x * kTile;
+  for (int r = 0; r < kItems; ++r) {
+#pragma unroll
+    for (int w = 0; w < kThreads / 32; ++w) cnt[w][tid] = 0;
+    __syncthreads();
+    const long long p = base + r * kThreads + tid;
+    const bool valid = p < n;
+    uint32_t k = 0;
+    int32_t v = 0;
+    if (valid) {
+      k = keys_in ? keys_in[p] : km.key(p);
+      v = vals_in ? vals_in[p] : (int32_t)p;
+    }
+    const uint32_t dig = valid ? ((k >> shift) & 255u) : 256u;
+    const unsigned peers = __match_any_sync(0xFFFFFFFFu, dig);
+    const int before = __popc(peers & ((1u << lane) - 1u));
+    const int leader = 31 - __clz(peers);
+    if (valid && lane == leader) cnt[warp][dig] = __popc(peers);
+    __syncthreads();
+    if (valid) {
+      uint32_t pos = run[dig] + before;
+      for (int w = 0; w < warp; ++w) pos += cnt[w][dig];
+      vals_out[pos] = v;
+      if (keys_out) keys_out[pos] = k;
+    }
+    __syncthreads();
+    uint32_t add = 0;
+#pragma unroll
+    for (int w = 0; w < kThreads / 32; ++w) add += cnt[w][tid];
+    run[tid] += add;
+    __syncthreads();
+  }
+}
+
+__global__ void count_keys_kernel(KeyMap km, long long n, uint32_t* __restrict__ counts) {
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long p = (long long)blockIdx.x * blockDim.x + threadIdx.x; p < n; p += stride) {
+    const uint32_t k = km.key(p);
+    if (k != km.sentinel) atomicAdd(&counts[k], 1u);
+  }
+}
+
+// ---- exclusive scan of uint32 (in place), up to kScanTile^2 elements
+__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* warp_sums, uint32_t& total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sums[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    uint32_t s = lane < (int)(blockDim.x / 32) ? warp_sums[lane] : 0u;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      uint32_t y = __shfl_up_sync(0xFFFFFFFFu, s, o);
+      if (lane >= o) s += y;
+    }
+    warp_sums[lane] = s;  // inclusive over warps
+  }
+  __syncthreads();
+  total = warp_sums[blockDim.x / 32 - 1];
+  const uint32_t warp_base = warp > 0 ? warp_sums[warp - 1] : 0u;
+  __syncthreads();
+  return warp_base + x - v;
+}
+
+__global__ void __launch_bounds__(kScanThreads) scan_tiles_kernel(uint32_t* __restrict__ a, long long n,
+                                                                  uint32_t* __restrict__ tile_sums) {
+  __shared__ uint32_t ws[32];
+  const long long base = (long long)blockIdx.x * kScanTile + (long long)threadIdx.x * kScanItems;
+  uint32_t v[kScanItems], s = 0;
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i) {
+    v[i] = base + i < n ? a[base + i] : 0u;
+    s += v[i];
+  }
+  uint32_t total;
+  uint32_t ex = block_exclusive_scan(s, ws, total);
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i) {
+    if (base + i < n) a[base + i] = ex;
+    ex += v[i];
+  }
+  if (threadIdx.x == 0 && tile_sums) tile_sums[blockIdx.x] = total;
+}
+
+__global__ void __launch_bounds__(kScanThreads) add_tile_base_kernel(uint32_t* __restrict__ a, long long n,
+                                                                     const uint32_t* __restrict__ tile_base) {
+  const long long base = (long long)blockIdx.x * kScanTile + (long long)threadIdx.x * kScanItems;
+  const uint32_t add = tile_base[blockIdx.x];
+#pragma unroll
+  for (int i = 0; i < kScanItems; ++i)
+    if (base + i < n) a[base + i] += add;
+}
+
+// Exclusive scan of a[0..n); writes the grand total to a[n] when with_total.
+cudaError_t exclusive_scan(uint32_t* a, long long n, uint32_t* tile_sums, cudaStream_t st) {
+  const long long tiles = (n + kScanTile - 1) / kScanTile;
+  if (tiles <= 1) {
+    scan_tiles_kernel<<<1, kScanThreads, 0, st>>>(a, n, nullptr);
+    note_launches(1);
+    return cudaGetLastError();
+  }
+  if (tiles > kScanTile) return cudaErrorInvalidValue;
+  scan_tiles_kernel<<<(unsigned)tiles, kScanThreads, 0, st>>>(a, n, tile_sums);
+  note_launches(1);
+  scan_tiles_kernel<<<1, kScanThreads, 0, st>>>(tile_sums, tiles, nullptr);
+  note_launches(1);
+  add_tile_base_kernel<<<(unsigned)tiles, kScanThreads, 0, st>>>(a, n, tile_sums);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+struct IndexLayout {
+  long long n, n_tiles, hist_len, keys;
+  int passes;
+  size_t off_keys_a, off_keys_b, off_vals_a, off_vals_b, off_hist, off_sums, total;
+};
+
+inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+IndexLayout layout(const Dims& D) {
+  IndexLayout lo{};
+  lo.n = D.slots();
+  lo.keys = D.keys();
+  lo.n_tiles = (lo.n + kTile - 1) / kTile;
+  lo.hist_len = 256 * lo.n_tiles;
+  int bits = 1;
+  while ((1ull << bits) <= (unsigned long long)lo.keys) ++bits;  // sentinel = keys must fit
+  lo.passes = (bits + 7) / 8;
+  size_t o = 0;
+  lo.off_keys_a = o;
+  o = align256(o + sizeof(uint32_t) * (size_t)lo.n);
+  lo.off_keys_b = o;
+  o = align256(o + sizeof(uint32_t) * (size_t)lo.n);
+  lo.off_vals_a = o;
+  o = align256(o + sizeof(int32_t) * (size_t)lo.n);
+  lo.off_vals_b = o;
+  o = align256(o + sizeof(int32_t) * (size_t)lo.n);
+  lo.off_hist = o;
+  const long long scan_len = lo.hist_len > lo.keys + 1 ? lo.hist_len : lo.keys + 1;
+  o = align256(o + sizeof(uint32_t) * (size_t)scan_len);
+  lo.off_sums = o;
+  o = align256(o + sizeof(uint32_t) * (size_t)((scan_len + kScanTile - 1) / kScanTile + 1));
+  lo.total = o;
+  return lo;
+}
+
+}  // namespace
+
+size_t index_workspace(const Dims& D) { return layout(D).total; }
+
+cudaError_t launch_index(const Dims& D, const int32_t* idx, int32_t* offsets, int32_t* entries, void* ws,
+                         cudaStream_t st) {
+  const IndexLayout lo = layout(D);
+  if (lo.n == 0) return cudaSuccess;
+  if ((lo.hist_len + kScanTile - 1) / kScanTile > kScanTile) return cudaErrorInvalidValue;
+  char* w = (char*)ws;
+  uint32_t* keys_buf[2] = {(uint32_t*)(w + lo.off_keys_a), (uint32_t*)(w + lo.off_keys_b)};
+  int32_t* vals_buf[2] = {(int32_t*)(w + lo.off_vals_a), (int32_t*)(w + lo.off_vals_b)};
+  uint32_t* hist = (uint32_t*)(w + lo.off_hist);
+  uint32_t* sums = (uint32_t*)(w + lo.off_sums);
+  KeyMap km{idx, D.L, D.Hkv, D.topk, D.Nc, (uint32_t)lo.keys};
+  cudaError_t e;
+  const uint32_t* kin = nullptr;
+  const int32_t* vin = nullptr;
+  for (int pass = 0; pass < lo.passes; ++pass) {
+    const bool last = pass == lo.passes - 1;
+    uint32_t* kout = last ? nullptr : keys_buf[pass & 1];
+    int32_t* vout = last ? entries : vals_buf[pass & 1];
+    radix_hist_kernel<<<(unsigned)lo.n_tiles, kThreads, 0, st>>>(km, kin, lo.n, 8 * pass, hist, (int)lo.n_tiles);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = exclusive_scan(hist, lo.hist_len, sums, st)) != cudaSuccess) return e;
+    radix_scatter_kernel<<<(unsigned)lo.n_tiles, kThreads, 0, st>>>(km, kin, vin, lo.n, 8 * pass, hist,
+                                                                   (int)lo.n_tiles, kout, vout);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    kin = kout;
+    vin = vout;
+  }
+  // offsets: counts per key, exclusive scan over keys + 1 (last = number of valid slots)
+  uint32_t* counts = (uint32_t*)offsets;
+  if ((e = cudaMemsetAsync(counts, 0, sizeof(uint32_t) * (size_t)(lo.keys + 1), st)) != cudaSuccess) return e;
+  count_keys_kernel<<<grid_cap((lo.n + 255) / 256, 152LL * 8), 256, 0, st>>>(km, lo.n, counts);
+  note_launches(1);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  return exclusive_scan(counts, lo.keys + 1, sums, st);
+}
+
+}  // namespace hsa

@@ -135,7 +135,12 @@ def bf16_to_f32(x: np.ndarray) -> np.ndarray:
 
 
 def bf16_to_f64(x: np.ndarray) -> np.ndarray:
-    return bf16_to_f32(x).astype(np.float64)
+    """Exact widening of bf16 bit patterns to fp64."""
+    x = np.ascontiguousarray(x, dtype=np.uint16)
+    out = np.empty(x.shape, dtype=np.float64)
+    if x.size:
+        host_lib().synth_bf16_to_f64(x.ctypes.data, out.ctypes.data, x.size)
+    return out
 
 
 def f32_to_bf16(x: np.ndarray) -> np.ndarray:

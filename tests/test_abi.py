@@ -1,0 +1,134 @@
+"""The C ABI loads, exports everything include/*.h declares, and validates
+arguments before any launch (these calls never reach the GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2504_16795_gb300 as hsa
+import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA = 0, 1, 2, 3, 4
+
+
+def declared(header):
+    text = open(header).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b((?:hsa|synth_dev)_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    hsa.build()
+    return hsa.load()
+
+
+def test_library_exports_every_declared_entry_point(lib):
+    names = declared(os.path.join(ROOT, "include", "hsa.h"))
+    assert {"hsa_chunk_pool", "hsa_select_topk", "hsa_build_index", "hsa_forward", "hsa_backward",
+            "hsa_decode"} <= set(names)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_synth_device_library_exports_its_header():
+    dev = ctypes.CDLL(synth.build_device())
+    for n in declared(os.path.join(ROOT, "synth", "synth.h")):
+        assert hasattr(dev, n), n
+
+
+def test_status_strings(lib):
+    for code in (OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA):
+        assert hsa.status_string(code).startswith("HSA_")
+
+
+def shape(**kw):
+    base = dict(B=1, L=1024, Hq=8, Hkv=1, d=128, S=64, topk=8)
+    base.update(kw)
+    return hsa.Shape(**base)
+
+
+FAKE = 1 << 20  # an aligned address that is never dereferenced: every call below fails validation first
+
+
+def call_forward(lib, s, ws_bytes=None, **ptrs):
+    p = dict(q=FAKE, K=FAKE, V=FAKE, idx=FAKE, s_sel=FAKE, off=FAKE, ent=FAKE, O=FAKE, w=FAKE, ws=FAKE)
+    p.update(ptrs)
+    need = hsa.workspace_size(hsa.HSA_OP_FORWARD, s)
+    c = s.c()
+    vp = ctypes.c_void_p
+    return lib.hsa_forward(ctypes.byref(c), vp(p["q"]), vp(p["K"]), vp(p["V"]), vp(p["idx"]), vp(p["s_sel"]),
+                           vp(p["off"]), vp(p["ent"]), vp(p["O"]), vp(p["w"]), vp(p["ws"]),
+                           need if ws_bytes is None else ws_bytes, None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(d=96), UNSUPPORTED),
+    (dict(d=256), UNSUPPORTED),
+    (dict(Hq=12, Hkv=4), UNSUPPORTED),   # G = 3
+    (dict(Hq=64, Hkv=2), UNSUPPORTED),   # G = 32
+    (dict(S=32), UNSUPPORTED),
+    (dict(topk=33), UNSUPPORTED),
+    (dict(Hq=6, Hkv=4), INVALID),        # not a multiple
+    (dict(topk=0), INVALID),
+    (dict(L=-1), INVALID),
+    (dict(B=1 << 20, L=1 << 20), UNSUPPORTED),  # slot count overflows int32
+])
+def test_shape_validation(lib, kw, code):
+    assert call_forward(lib, shape(**kw), ws_bytes=0) == code
+
+
+def test_null_and_misaligned_pointers_are_rejected(lib):
+    s = shape()
+    assert call_forward(lib, s, q=0) == INVALID
+    assert call_forward(lib, s, K=FAKE + 8) == INVALID
+    assert call_forward(lib, s, O=FAKE + 2) == INVALID
+
+
+def test_short_workspace_is_rejected(lib):
+    s = shape()
+    need = hsa.workspace_size(hsa.HSA_OP_FORWARD, s)
+    assert need > 0
+    assert call_forward(lib, s, ws_bytes=need - 1) == WORKSPACE
+    assert call_forward(lib, s, ws=0) == WORKSPACE
+
+
+def test_empty_problems_succeed_without_launching(lib):
+    assert call_forward(lib, shape(B=0), q=0, K=0, V=0) == OK
+    assert call_forward(lib, shape(L=0), q=0, K=0, V=0) == OK
+    d = hsa.DecodeShape(Bq=0, Hq=8, Hkv=1, d=128, n_chunks=10)
+    c = d.c()
+    vp = ctypes.c_void_p
+    assert lib.hsa_decode(ctypes.byref(c), *[vp(0)] * 9, 0, None) == OK
+
+
+def test_decode_validation(lib):
+    vp = ctypes.c_void_p
+    for kw, code in [(dict(d=80), UNSUPPORTED), (dict(n_chunks=-1), INVALID), (dict(topk=40), UNSUPPORTED)]:
+        base = dict(Bq=4, Hq=8, Hkv=1, d=128, n_chunks=100)
+        base.update(kw)
+        c = hsa.DecodeShape(**base).c()
+        assert lib.hsa_decode(ctypes.byref(c), *[vp(FAKE)] * 9, 1 << 30, None) == code
+    c = hsa.DecodeShape(Bq=4, Hq=8, Hkv=1, d=128, n_chunks=100).c()
+    assert lib.hsa_decode(ctypes.byref(c), *[vp(FAKE)] * 9, 16, None) == WORKSPACE
+
+
+def test_workspace_sizes_scale_with_the_problem(lib):
+    s = shape(B=2, L=32768, Hq=32, Hkv=4)
+    slots = 2 * 32768 * 4 * 8
+    assert hsa.workspace_size(hsa.HSA_OP_SELECT, s) == 0
+    assert hsa.workspace_size(hsa.HSA_OP_FORWARD, s) == slots * 8 * 128 * 2
+    assert hsa.workspace_size(hsa.HSA_OP_BACKWARD, s) >= slots * 8 * 128 * 4
+    assert hsa.workspace_size(hsa.HSA_OP_INDEX, s) >= slots * 16
+    assert hsa.workspace_size(hsa.HSA_OP_FORWARD, shape(d=96)) == 0
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    import paper_2504_16795_gb300.binding as b
+    monkeypatch.setattr(b, "_lib", None)
+    monkeypatch.setattr(b._build, "LIB", str(tmp_path / "absent.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        b.load()

@@ -39,6 +39,15 @@ UNIT = "tokens/s"
 PREFILL = synth.WORKLOADS[3]
 DECODE = synth.WORKLOADS[5]
 
+
+def select_workload(number, batch):
+    """The timed prefill workload (default: the long-context one); smaller ones serve profiling."""
+    global PREFILL
+    w = synth.WORKLOADS[number]
+    if w.decode or not w.backward:
+        raise SystemExit(f"workload {number} is not a fwd+bwd prefill workload")
+    PREFILL = w.with_(B=batch) if batch else w
+
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of the dominant
 # kernel from one ncu capture, keyed by the source file it was compiled from
 # and that file's sha256 at capture time (reported as null once the source
@@ -109,7 +118,7 @@ def bound_of(flops, nbytes, pk):
 # ----------------------------------------------------------------------------- clocks
 
 class ClockSampler:
-    """nvidia-smi samples (200 ms) while the timed region runs."""
+    """nvidia-smi samples (every 100 ms) while the timed region runs."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -126,7 +135,7 @@ class ClockSampler:
         try:
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
                                          stdout=self.f, stderr=subprocess.DEVNULL)
         except OSError:
             self.proc = None
@@ -464,13 +473,16 @@ def config_obj():
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=40)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["hsa", "reference"], default="hsa")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", type=int, default=3, help="prefill workload number (3 is the headline)")
+    ap.add_argument("--batch", type=int, default=0, help="override the workload's batch (profiling)")
     args = ap.parse_args()
+    select_workload(args.workload, args.batch)
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

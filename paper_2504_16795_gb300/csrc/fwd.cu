@@ -211,12 +211,17 @@ __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict_
   const int GD8 = G * (D / 8);
   const uint4* src = reinterpret_cast<const uint4*>(Opart) + p0 * GD8;
   uint4* dst = reinterpret_cast<uint4*>(O) + row * GD8;  // heads of group g are contiguous in O
-  for (int ch = lane; ch < GD8; ch += 32) {
+  // every lane runs every iteration (the weight broadcast needs the full warp);
+  // lanes past the row's last 16-byte chunk only skip the memory accesses
+  for (int base = 0; base < GD8; base += 32) {
+    const int ch = base + lane;
+    const bool active = ch < GD8;
     float acc[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i] = 0.f;
     for (int j = 0; j < keff; ++j) {
       const float wb = __shfl_sync(0xFFFFFFFFu, wj, j);
+      if (!active) continue;
       const uint4 v = src[(long long)j * GD8 + ch];
       acc[0] += wb * bf16_lo(v.x);
       acc[1] += wb * bf16_hi(v.x);
@@ -227,6 +232,7 @@ __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict_
       acc[6] += wb * bf16_lo(v.w);
       acc[7] += wb * bf16_hi(v.w);
     }
+    if (!active) continue;
     uint4 out;
     out.x = pack_bf16x2(acc[0], acc[1]);
     out.y = pack_bf16x2(acc[2], acc[3]);

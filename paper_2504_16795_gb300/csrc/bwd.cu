@@ -13,12 +13,17 @@
 //   dK_I  += c_att da^T q_h,  dV_I += w_j P^T dO_h  (Algorithm 3)
 //   dK̄_I  += c_sel ds_j q̂_t ;  dK_{I,s} += dK̄_I / S  (mean pool)
 //
+// The mean-pool term reaches every row s of the chunk equally, and q̂_t is
+// the sum of the slot's G query rows, so adding c_sel ds_j / S to every
+// element of the slot's rows of the dS tile that feeds dK = dS^T Q produces
+// dK̄_I / S inside the same tensor-core product.
+//
 // Chunk-major and deterministic: one block per (b, g, chunk) owns that
 // chunk's dK/dV rows, walks the chunk's slots (from the inverse index) in
 // increasing token order 128 query rows at a time and accumulates dK, dV and
 // dK̄ on chip; no floating-point atomics anywhere. Each slot's dq
-// contribution goes to a workspace row and a second kernel sums the k slots
-// of each token in slot order.
+// contribution goes to a bf16 workspace row and a second kernel sums the k
+// slots of each token in slot order (fp32).
 #include "common.cuh"
 
 namespace hsa {
@@ -34,9 +39,8 @@ struct BwdSmem {
   uint16_t Q[2][kRows * D];
   uint16_t dO[2][kRows * D];
   uint16_t P[kRows * kChunk];   // w * P, bf16
-  uint16_t dS[kRows * kChunk];  // c_att * w * P∘(dP' - D), bf16
+  uint16_t dS[kRows * kChunk];  // c_att * w * P∘(dP' - D) + c_sel * ds / S, bf16
   float kbar[D];
-  float ds[kRows];
   float wslot[2][kRows];
   float delta[2][kRows];
   int pslot[2][kRows];
@@ -52,7 +56,7 @@ struct BwdArgs {
   const float* delta;  // [B, L, Hkv]
   const int32_t* offsets;
   const int32_t* entries;
-  float* dqpart;  // [slots, G, D]
+  uint16_t* dqpart;  // [slots, G, D] bf16
   float* dK;
   float* dV;
   int L, Hq, Hkv, G, log2G, topk, Nc;
@@ -82,7 +86,6 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
 #pragma unroll
   for (int i = 0; i < NH / 8; ++i) dv[i][0] = dv[i][1] = dv[i][2] = dv[i][3] = dk[i][0] = dk[i][1] = dk[i][2] =
       dk[i][3] = 0.f;
-  float kbar_acc = 0.f;  // thread tid < D: sum over slots of ds * q̂[tid]
 
   if (cnt > 0) {
     for (int u = tid; u < kChunk * D8; u += kThreads) {
@@ -220,8 +223,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
     const float w0 = sm.wslot[buf][sl0], w1 = sm.wslot[buf][sl1];
     const float ds0 = w0 * (dw0 - sm.delta[buf][sl0]);
     const float ds1 = w1 * (dw1 - sm.delta[buf][sl1]);
-    if ((lane & 3) == 0 && (R0 & (a.G - 1)) == 0) sm.ds[sl0] = ds0;
-    if ((lane & 3) == 0 && (R1 & (a.G - 1)) == 0) sm.ds[sl1] = ds1;
+    const float pool0 = a.scale_sel * ds0 * (1.f / kChunk), pool1 = a.scale_sel * ds1 * (1.f / kChunk);
     // da (scaled by c_att for the products) and w P, to fragments and shared tiles
     const float ca0 = a.scale_attn * w0, ca1 = a.scale_attn * w1;
     uint32_t dsf[4][4];
@@ -239,9 +241,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
         *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(sm.P) + swz<kChunk>(R0, 8 * nt + cc)) = p0;
         *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(sm.P) + swz<kChunk>(R1, 8 * nt + cc)) = p1;
         *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(sm.dS) + swz<kChunk>(R0, 8 * nt + cc)) =
-            dsf[kk][2 * h];
+            pack_bf16x2(g00 + pool0, g01 + pool0);
         *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(sm.dS) + swz<kChunk>(R1, 8 * nt + cc)) =
-            dsf[kk][2 * h + 1];
+            pack_bf16x2(g10 + pool1, g11 + pool1);
       }
     }
     // dsf[kk] is already in A-fragment order {row0 keys 0-7, row1 keys 0-7, row0 keys 8-15, row1 keys 8-15}
@@ -249,8 +251,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
     const int e0 = it * epi + sl0, e1 = it * epi + sl1;
     const int p0 = e0 < cnt ? sm.pslot[buf][sl0] : -1;
     const int p1 = e1 < cnt ? sm.pslot[buf][sl1] : -1;
-    float* dq0 = p0 >= 0 ? a.dqpart + ((long long)p0 * a.G + (R0 & (a.G - 1))) * D : nullptr;
-    float* dq1 = p1 >= 0 ? a.dqpart + ((long long)p1 * a.G + (R1 & (a.G - 1))) * D : nullptr;
+    uint16_t* dq0 = p0 >= 0 ? a.dqpart + ((long long)p0 * a.G + (R0 & (a.G - 1))) * D : nullptr;
+    uint16_t* dq1 = p1 >= 0 ? a.dqpart + ((long long)p1 * a.G + (R1 & (a.G - 1))) * D : nullptr;
     const float cs0 = a.scale_sel * ds0, cs1 = a.scale_sel * ds1;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
@@ -273,11 +275,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
       for (int nt = 0; nt < D / 16; ++nt) {
         const int col = half * (D / 2) + 8 * nt + cc;
         if (dq0)
-          *reinterpret_cast<float2*>(dq0 + col) =
-              make_float2(acc[nt][0] + cs0 * sm.kbar[col], acc[nt][1] + cs0 * sm.kbar[col + 1]);
+          *reinterpret_cast<uint32_t*>(dq0 + col) =
+              pack_bf16x2(acc[nt][0] + cs0 * sm.kbar[col], acc[nt][1] + cs0 * sm.kbar[col + 1]);
         if (dq1)
-          *reinterpret_cast<float2*>(dq1 + col) =
-              make_float2(acc[nt][2] + cs1 * sm.kbar[col], acc[nt][3] + cs1 * sm.kbar[col + 1]);
+          *reinterpret_cast<uint32_t*>(dq1 + col) =
+              pack_bf16x2(acc[nt][2] + cs1 * sm.kbar[col], acc[nt][3] + cs1 * sm.kbar[col + 1]);
       }
     }
     __syncthreads();  // P, dS tiles and ds complete
@@ -301,31 +303,17 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
         mma_bf16(dk[2 * np + 1], as, bq[2], bq[3]);
       }
     }
-    // dK̄ accumulation: ds_j * q̂_t, slots in order
-    if (tid < D) {
-      const char* qrow = reinterpret_cast<const char*>(sm.Q[buf]);
-      const int nslot = min(epi, cnt - it * epi);
-      for (int e = 0; e < nslot; ++e) {
-        float qh = 0.f;
-        for (int hh = 0; hh < a.G; ++hh)
-          qh = qh + bf16_bits_to_f32(*reinterpret_cast<const uint16_t*>(qrow + swz<D>(e * a.G + hh, tid)));
-        kbar_acc = fmaf(sm.ds[e], qh, kbar_acc);
-      }
-    }
     __syncthreads();  // buffers of this step free for the prefetch two steps ahead
   }
 
-  // epilogue: dK = dK_att + c_sel * dK̄ / S (every row of the chunk), dV
-  if (tid < D) sm.kbar[tid] = a.scale_sel * kbar_acc / (float)kChunk;
-  __syncthreads();
+  // epilogue: dK (attention and mean-pool terms) and dV of every row of the chunk
 #pragma unroll
   for (int nt = 0; nt < NH / 8; ++nt) {
     const int col = dc0 + 8 * nt + cc;
-    const float k0 = sm.kbar[col], k1 = sm.kbar[col + 1];
     const long long ra = (row0 + (long long)(sr0 + rr) * a.Hkv) * D + col;
     const long long rb = (row0 + (long long)(sr0 + rr + 8) * a.Hkv) * D + col;
-    *reinterpret_cast<float2*>(a.dK + ra) = make_float2(dk[nt][0] + k0, dk[nt][1] + k1);
-    *reinterpret_cast<float2*>(a.dK + rb) = make_float2(dk[nt][2] + k0, dk[nt][3] + k1);
+    *reinterpret_cast<float2*>(a.dK + ra) = make_float2(dk[nt][0], dk[nt][1]);
+    *reinterpret_cast<float2*>(a.dK + rb) = make_float2(dk[nt][2], dk[nt][3]);
     *reinterpret_cast<float2*>(a.dV + ra) = make_float2(dv[nt][0], dv[nt][1]);
     *reinterpret_cast<float2*>(a.dV + rb) = make_float2(dv[nt][2], dv[nt][3]);
   }
@@ -355,7 +343,7 @@ __global__ void __launch_bounds__(256) bwd_delta_kernel(const uint16_t* __restri
 // dq_t = sum_j dq'_{t,j} in slot order (one warp per (b, t, g)).
 template <int D>
 __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __restrict__ idx,
-                                                           const float* __restrict__ dqpart, float* __restrict__ dq,
+                                                           const uint16_t* __restrict__ dqpart, float* __restrict__ dq,
                                                            long long n_rows, int G, int topk, int Nc) {
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
@@ -367,19 +355,26 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
     valid = c >= 0 && c < Nc;
   }
   const int keff = __popc(__ballot_sync(0xFFFFFFFFu, valid));
-  const int GD4 = G * (D / 4);
-  const float4* src = reinterpret_cast<const float4*>(dqpart) + p0 * GD4;
-  float4* dst = reinterpret_cast<float4*>(dq) + row * GD4;
-  for (int ch = lane; ch < GD4; ch += 32) {
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  const int GD8 = G * (D / 8);
+  const uint4* src = reinterpret_cast<const uint4*>(dqpart) + p0 * GD8;
+  float4* dst = reinterpret_cast<float4*>(dq) + row * GD8 * 2;
+  for (int ch = lane; ch < GD8; ch += 32) {
+    float acc[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i] = 0.f;
     for (int j = 0; j < keff; ++j) {
-      const float4 v = src[(long long)j * GD4 + ch];
-      acc.x += v.x;
-      acc.y += v.y;
-      acc.z += v.z;
-      acc.w += v.w;
+      const uint4 v = src[(long long)j * GD8 + ch];
+      acc[0] += bf16_lo(v.x);
+      acc[1] += bf16_hi(v.x);
+      acc[2] += bf16_lo(v.y);
+      acc[3] += bf16_hi(v.y);
+      acc[4] += bf16_lo(v.z);
+      acc[5] += bf16_hi(v.z);
+      acc[6] += bf16_lo(v.w);
+      acc[7] += bf16_hi(v.w);
     }
-    dst[ch] = acc;
+    dst[2 * ch] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    dst[2 * ch + 1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
   }
 }
 
@@ -404,8 +399,8 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
                 const float* w, const void* O, const void* dO, const int32_t* offsets, const int32_t* entries,
                 float* dq, float* dK, float* dV, void* ws, cudaStream_t st) {
   const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
-  float* dqpart = (float*)ws;
-  float* delta = (float*)((char*)ws + align256((size_t)Dm.slots() * Dm.G * D * sizeof(float)));
+  uint16_t* dqpart = (uint16_t*)ws;
+  float* delta = (float*)((char*)ws + align256((size_t)Dm.slots() * Dm.G * D * sizeof(uint16_t)));
   cudaError_t e;
   bwd_delta_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>((const uint16_t*)O, (const uint16_t*)dO, delta,
                                                                   rows, Dm.G);
@@ -461,7 +456,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
 }  // namespace
 
 size_t backward_workspace(const Dims& D) {
-  return align256((size_t)D.slots() * D.G * D.d * sizeof(float)) +
+  return align256((size_t)D.slots() * D.G * D.d * sizeof(uint16_t)) +
          align256((size_t)D.B * D.L * D.Hkv * sizeof(float));
 }
 

@@ -6,7 +6,8 @@
 //
 //   pass p (8-bit digit p):   per-tile digit histogram -> exclusive scan over
 //                             (digit, tile) -> stable scatter within each tile
-//   offsets:                  per-key counts -> exclusive scan
+//   offsets:                  from the sorted keys: offsets[k] = first position
+//                             whose key is >= k (one pass, no atomics)
 // Padded slots (idx = -1) get the sentinel key B*Hkv*Nc and sort to the end.
 #include "common.cuh"
 
@@ -100,11 +101,17 @@ __global__ void __launch_bounds__(kThreads) radix_scatter_kernel(KeyMap km, cons
   }
 }
 
-__global__ void count_keys_kernel(KeyMap km, long long n, uint32_t* __restrict__ counts) {
+// offsets[k] = first position of the sorted key array with key >= k, for
+// k = 0..n_keys (the sentinel key n_keys sorts last). Position i writes the
+// keys in (key[i-1], key[i]]; position n closes the range up to n_keys.
+__global__ void offsets_from_sorted_kernel(const uint32_t* __restrict__ sorted, long long n, long long n_keys,
+                                           int32_t* __restrict__ offsets) {
   const long long stride = (long long)gridDim.x * blockDim.x;
-  for (long long p = (long long)blockIdx.x * blockDim.x + threadIdx.x; p < n; p += stride) {
-    const uint32_t k = km.key(p);
-    if (k != km.sentinel) atomicAdd(&counts[k], 1u);
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i <= n; i += stride) {
+    const long long cur = i < n ? (long long)sorted[i] : n_keys;
+    const long long prev = i > 0 ? (long long)sorted[i - 1] : -1;
+    const long long hi = cur < n_keys ? cur : n_keys;
+    for (long long k = prev + 1; k <= hi; ++k) offsets[k] = (int32_t)i;
   }
 }
 
@@ -164,7 +171,7 @@ __global__ void __launch_bounds__(kScanThreads) add_tile_base_kernel(uint32_t* _
     if (base + i < n) a[base + i] += add;
 }
 
-// Exclusive scan of a[0..n); writes the grand total to a[n] when with_total.
+// Exclusive scan of a[0..n) in place (tile_sums: scratch for the tile totals).
 cudaError_t exclusive_scan(uint32_t* a, long long n, uint32_t* tile_sums, cudaStream_t st) {
   const long long tiles = (n + kScanTile - 1) / kScanTile;
   if (tiles <= 1) {
@@ -209,7 +216,7 @@ IndexLayout layout(const Dims& D) {
   lo.off_vals_b = o;
   o = align256(o + sizeof(int32_t) * (size_t)lo.n);
   lo.off_hist = o;
-  const long long scan_len = lo.hist_len > lo.keys + 1 ? lo.hist_len : lo.keys + 1;
+  const long long scan_len = lo.hist_len;
   o = align256(o + sizeof(uint32_t) * (size_t)scan_len);
   lo.off_sums = o;
   o = align256(o + sizeof(uint32_t) * (size_t)((scan_len + kScanTile - 1) / kScanTile + 1));
@@ -237,7 +244,7 @@ cudaError_t launch_index(const Dims& D, const int32_t* idx, int32_t* offsets, in
   const int32_t* vin = nullptr;
   for (int pass = 0; pass < lo.passes; ++pass) {
     const bool last = pass == lo.passes - 1;
-    uint32_t* kout = last ? nullptr : keys_buf[pass & 1];
+    uint32_t* kout = keys_buf[pass & 1];
     int32_t* vout = last ? entries : vals_buf[pass & 1];
     radix_hist_kernel<<<(unsigned)lo.n_tiles, kThreads, 0, st>>>(km, kin, lo.n, 8 * pass, hist, (int)lo.n_tiles);
     note_launches(1);
@@ -250,13 +257,10 @@ cudaError_t launch_index(const Dims& D, const int32_t* idx, int32_t* offsets, in
     kin = kout;
     vin = vout;
   }
-  // offsets: counts per key, exclusive scan over keys + 1 (last = number of valid slots)
-  uint32_t* counts = (uint32_t*)offsets;
-  if ((e = cudaMemsetAsync(counts, 0, sizeof(uint32_t) * (size_t)(lo.keys + 1), st)) != cudaSuccess) return e;
-  count_keys_kernel<<<grid_cap((lo.n + 255) / 256, 152LL * 8), 256, 0, st>>>(km, lo.n, counts);
+  // offsets from the sorted keys of the last pass
+  offsets_from_sorted_kernel<<<grid_cap((lo.n + 256) / 256, 152LL * 8), 256, 0, st>>>(kin, lo.n, lo.keys, offsets);
   note_launches(1);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  return exclusive_scan(counts, lo.keys + 1, sums, st);
+  return cudaGetLastError();
 }
 
 }  // namespace hsa

@@ -56,7 +56,8 @@ typedef enum {
     HSA_ERR_INVALID_ARG = 1,
     HSA_ERR_UNSUPPORTED = 2,
     HSA_ERR_WORKSPACE = 3,
-    HSA_ERR_CUDA = 4
+    HSA_ERR_CUDA = 4,
+    HSA_ERR_TIMEOUT = 5
 } hsa_status_t;
 
 typedef struct {
@@ -88,6 +89,15 @@ int hsa_version(void);
 /* Number of CUDA kernels this library has launched since it was loaded (a
  * diagnostic for launch accounting; counts launches, not their completion). */
 unsigned long long hsa_kernel_launches(void);
+
+/* Device-side health check. Pipelined kernels give up on any internal wait
+ * that lasts longer than 2 s (instead of hanging the GPU) and record it in a
+ * device status word; this call waits for the device to finish its work,
+ * reads and clears that word and returns HSA_ERR_TIMEOUT if a wait gave up
+ * since the previous check (the results of that launch are then invalid),
+ * HSA_ERR_CUDA if the device reports an error, HSA_OK otherwise.
+ * Synchronising: not for use inside a timed region. */
+hsa_status_t hsa_device_check(void);
 
 /* Workspace bytes that `op` needs for `shape` (0 when it needs none). Returns
  * 0 too for an invalid shape; the call itself then reports the error. */

@@ -19,6 +19,7 @@ from .binding import (  # noqa: F401
     chunk_pool,
     decode,
     decode_workspace_size,
+    device_check,
     forward,
     hsa_backward_path,
     hsa_forward_path,

@@ -102,6 +102,8 @@ def load():
     L.hsa_version.restype = i
     L.hsa_kernel_launches.restype = ctypes.c_ulonglong
     L.hsa_kernel_launches.argtypes = []
+    L.hsa_device_check.restype = i
+    L.hsa_device_check.argtypes = []
     L.hsa_workspace_size.restype = sz
     L.hsa_workspace_size.argtypes = [i, sp]
     L.hsa_decode_workspace_size.restype = sz
@@ -122,6 +124,11 @@ def load():
 def kernel_launches() -> int:
     """Kernels launched by libhsa.so since it was loaded."""
     return int(load().hsa_kernel_launches())
+
+
+def device_check() -> None:
+    """Synchronise and raise if a device-side wait gave up since the last check."""
+    _check(load().hsa_device_check(), "hsa_device_check")
 
 
 def status_string(status: int) -> str:

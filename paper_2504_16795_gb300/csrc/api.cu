@@ -74,6 +74,7 @@ const char* hsa_status_string(hsa_status_t status) {
     case HSA_ERR_UNSUPPORTED: return "HSA_ERR_UNSUPPORTED: shape outside the supported set";
     case HSA_ERR_WORKSPACE: return "HSA_ERR_WORKSPACE: workspace missing or too small";
     case HSA_ERR_CUDA: return "HSA_ERR_CUDA: a kernel launch failed";
+    case HSA_ERR_TIMEOUT: return "HSA_ERR_TIMEOUT: a device-side wait gave up (results invalid)";
   }
   return "HSA_ERR_UNKNOWN";
 }
@@ -81,6 +82,13 @@ const char* hsa_status_string(hsa_status_t status) {
 int hsa_version(void) { return 100; }
 
 unsigned long long hsa_kernel_launches(void) { return hsa::g_launches.load(std::memory_order_relaxed); }
+
+hsa_status_t hsa_device_check(void) {
+  if (cudaDeviceSynchronize() != cudaSuccess) return HSA_ERR_CUDA;
+  const unsigned s = hsa::forward_take_status();
+  if (s == ~0u) return HSA_ERR_CUDA;
+  return s ? HSA_ERR_TIMEOUT : HSA_OK;
+}
 
 size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {
   Dims D;

@@ -172,6 +172,7 @@ size_t index_workspace(const Dims& D);
 cudaError_t launch_index(const Dims& D, const int32_t* idx, int32_t* offsets, int32_t* entries, void* ws,
                          cudaStream_t st);
 size_t forward_workspace(const Dims& D);
+unsigned forward_take_status();
 cudaError_t launch_forward(const Dims& D, const void* q, const void* K, const void* V, const int32_t* idx,
                            const float* s_sel, const int32_t* offsets, const int32_t* entries, void* O, float* w,
                            void* ws, cudaStream_t st);

@@ -11,19 +11,37 @@
 // rescaling. The normalised per-slot result O' (bf16) goes to a workspace
 // and a second kernel forms O_t = sum_j w_j O'_{t,j} with the chunk weights
 // w = softmax_j(s_sel) (the "w/o s.b." variant of §4.1), slots in order j.
-#include "common.cuh"
+#include "tc.cuh"
 
 namespace hsa {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kRows = 128;  // query rows per step (8 warps x 16)
+constexpr int kRows = 128;     // query rows per step (tensor-core M)
+constexpr int kQStages = 3;    // gathered query tiles in flight
+constexpr int kThreads = 288;  // 4 softmax/epilogue warps, 4 loader warps, 1 MMA warp
+constexpr int kTmemCols = 512;
+
+__device__ unsigned g_fwd_status;
 
 template <int D>
 struct FwdSmem {
-  uint16_t K[kChunk * D];
-  uint16_t V[kChunk * D];
-  uint16_t Q[2][kRows * D];
+  uint16_t Q[kQStages][kRows * D];  // gathered query rows, K-major SW128
+  uint16_t K[kChunk * D];           // chunk keys [s][d]
+  uint16_t Vt[D * kChunk];          // chunk values transposed [d][s]
+  uint16_t P[2][kRows * kChunk];    // normalised probabilities (bf16)
+  uint64_t bar[16];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+enum {
+  BAR_Q_FULL = 0,   // 3: tile landed (128 loader arrivals)
+  BAR_Q_EMPTY = 3,  // 3: S MMA of the tile finished (commit)
+  BAR_S_FULL = 6,   // 2: S accumulator ready (commit)
+  BAR_S_EMPTY = 8,  // 2: S read by the softmax warps (128 arrivals)
+  BAR_P_FULL = 10,  // 2: P tile written (128 arrivals)
+  BAR_O_FULL = 12,  // 2: O accumulator ready (commit)
+  BAR_O_EMPTY = 14  // 2: O read by the epilogue (128 arrivals)
 };
 
 struct FwdArgs {
@@ -38,9 +56,9 @@ struct FwdArgs {
 };
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 2) fwd_chunk_kernel(FwdArgs a) {
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>(smem_raw);
+__global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int key = blockIdx.x;
@@ -52,135 +70,193 @@ __global__ void __launch_bounds__(kThreads, 2) fwd_chunk_kernel(FwdArgs a) {
   const int epi = kRows >> a.log2G;  // slots per step
   const int niter = (cnt + epi - 1) / epi;
   const int slot_div = a.Hkv * a.topk;
+  auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
+  volatile int* abort_flag = &sm.abort_flag;
 
-  {  // chunk K, V tiles
-    const long long row0 = ((long long)b * a.L + (long long)c * kChunk) * a.Hkv + g;
-    for (int u = tid; u < kChunk * D8; u += kThreads) {
-      const int r = u / D8, ch = u % D8;
-      const long long src = (row0 + (long long)r * a.Hkv) * D + ch * 8;
-      cp_async16(smem_u32(sm.K) + swz<D>(r, ch * 8), a.K + src);
-      cp_async16(smem_u32(sm.V) + swz<D>(r, ch * 8), a.V + src);
+  if (tid == 0) {
+    for (int i = 0; i < 3; ++i) {
+      tc::mbar_init(bar(BAR_Q_FULL + i), 128);
+      tc::mbar_init(bar(BAR_Q_EMPTY + i), 1);
     }
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(bar(BAR_S_FULL + i), 1);
+      tc::mbar_init(bar(BAR_S_EMPTY + i), 128);
+      tc::mbar_init(bar(BAR_P_FULL + i), 128);
+      tc::mbar_init(bar(BAR_O_FULL + i), 1);
+      tc::mbar_init(bar(BAR_O_EMPTY + i), 128);
+    }
+    sm.abort_flag = 0;
+    tc::fence_mbar_init();
   }
-  auto load_q = [&](int it, int buf) {
-    const uint32_t base = smem_u32(sm.Q[buf]);
-    for (int u = tid; u < kRows * D8; u += kThreads) {
-      const int r = u / D8, ch = u % D8;
-      const int e = it * epi + (r >> a.log2G);
-      const uint32_t dst = base + swz<D>(r, ch * 8);
-      if (e < cnt) {
-        const int p = a.entries[off + e];
-        const int t = (p / slot_div) % a.L;
-        const long long src = (((long long)b * a.L + t) * a.Hq + (long long)g * a.G + (r & (a.G - 1))) * D + ch * 8;
-        cp_async16(dst, a.q + src);
-      } else {
-        asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(dst), "r"(0));
+  if (warp == 8) tc::tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+  if (warp >= 4 && warp < 8) {  // chunk K (K-major rows s) and V^T (rows d), once per block
+    const int lt = tid - 128;
+    const long long row0 = ((long long)b * a.L + (long long)c * kChunk) * a.Hkv + g;
+    for (int u = lt; u < kChunk * D8; u += 128) {
+      const int srow = u / D8, ch = u % D8;
+      const long long src = (row0 + (long long)srow * a.Hkv) * D + ch * 8;
+      cp_async16(smem_u32(sm.K) + tc::sw128_offset(kChunk, srow, ch * 8), a.K + src);
+      const uint4 v = __ldg(reinterpret_cast<const uint4*>(a.V + src));
+      const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const uint16_t h = (uint16_t)(i & 1 ? (w4[i >> 1] >> 16) : (w4[i >> 1] & 0xFFFFu));
+        *reinterpret_cast<uint16_t*>(reinterpret_cast<char*>(sm.Vt) + tc::sw128_offset(D, ch * 8 + i, srow)) = h;
       }
     }
-  };
-  load_q(0, 0);
-  cp_async_commit();
-
-  const uint32_t kb = smem_u32(sm.K), vb = smem_u32(sm.V);
-  for (int it = 0; it < niter; ++it) {
-    const int buf = it & 1;
-    if (it + 1 < niter) load_q(it + 1, buf ^ 1);
     cp_async_commit();
-    cp_async_wait<1>();
-    __syncthreads();
-    const uint32_t qb = smem_u32(sm.Q[buf]);
-    const int r0 = warp * 16;
+    cp_async_wait<0>();
+    tc::fence_proxy_async_smem();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = sm.tmem_base;
 
-    // S = Q K^T : 16 rows x 64 keys per warp
-    float s[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.f;
-#pragma unroll
-    for (int kd = 0; kd < D / 16; ++kd) {
-      uint32_t af[4];
-      ldsm_x4(af, qb + swz<D>(r0 + (lane & 7) + 8 * ((lane >> 3) & 1), 16 * kd + 8 * (lane >> 4)));
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        uint32_t bf[4];
-        ldsm_x4(bf, kb + swz<D>(16 * np + (lane & 7) + 8 * (lane >> 4), 16 * kd + 8 * ((lane >> 3) & 1)));
-        mma_bf16(s[2 * np], af, bf[0], bf[1]);
-        mma_bf16(s[2 * np + 1], af, bf[2], bf[3]);
+  if (warp >= 4 && warp < 8) {
+    // ---------------------------------------------------------------- loaders
+    const int lt = tid - 128;
+    for (int i = 0; i < niter; ++i) {
+      const int st = i % kQStages;
+      tc::mbar_wait(bar(BAR_Q_EMPTY + st), ((i / kQStages) & 1) ^ 1, abort_flag, &g_fwd_status);
+      const uint32_t base = smem_u32(sm.Q[st]);
+      for (int u = lt; u < kRows * D8; u += 128) {
+        const int r = u / D8, ch = u % D8;
+        const int e = i * epi + (r >> a.log2G);
+        const uint32_t dst = base + tc::sw128_offset(kRows, r, ch * 8);
+        if (e < cnt) {
+          const int p = a.entries[off + e];
+          const int t = (p / slot_div) % a.L;
+          const long long src =
+              (((long long)b * a.L + t) * a.Hq + (long long)g * a.G + (r & (a.G - 1))) * D + ch * 8;
+          cp_async16(dst, a.q + src);
+        } else {
+          asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(dst), "r"(0));
+        }
+      }
+      cp_async_commit();
+      if (i >= 1) {
+        cp_async_wait<1>();
+        tc::fence_proxy_async_smem();
+        tc::mbar_arrive(bar(BAR_Q_FULL + (i - 1) % kQStages));
       }
     }
-    // softmax over the chunk's 64 keys (rows lane/4 and lane/4 + 8)
-    float m0 = -INFINITY, m1 = -INFINITY;
+    cp_async_wait<0>();
+    tc::fence_proxy_async_smem();
+    tc::mbar_arrive(bar(BAR_Q_FULL + (niter - 1) % kQStages));
+  } else if (warp == 8) {
+    // ---------------------------------------------------------------- MMA issue (one thread)
+    if (lane == 0) {
+      constexpr uint32_t idS = tc::idesc_bf16(kRows, kChunk);
+      constexpr uint32_t idO = tc::idesc_bf16(kRows, D);
+      const uint32_t kbase = smem_u32(sm.K), vbase = smem_u32(sm.Vt);
+      auto issue_S = [&](int i) {
+        const int st = i % kQStages, sb = i & 1;
+        tc::mbar_wait(bar(BAR_Q_FULL + st), (i / kQStages) & 1, abort_flag, &g_fwd_status);
+        tc::mbar_wait(bar(BAR_S_EMPTY + sb), ((i >> 1) & 1) ^ 1, abort_flag, &g_fwd_status);
+        tc::fence_after_sync();
+        const uint32_t qbase = smem_u32(sm.Q[st]);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      s[i][0] *= a.scale_log2;
-      s[i][1] *= a.scale_log2;
-      s[i][2] *= a.scale_log2;
-      s[i][3] *= a.scale_log2;
-      m0 = fmaxf(m0, fmaxf(s[i][0], s[i][1]));
-      m1 = fmaxf(m1, fmaxf(s[i][2], s[i][3]));
-    }
-    m0 = fmaxf(m0, __shfl_xor_sync(0xFFFFFFFFu, m0, 1));
-    m0 = fmaxf(m0, __shfl_xor_sync(0xFFFFFFFFu, m0, 2));
-    m1 = fmaxf(m1, __shfl_xor_sync(0xFFFFFFFFu, m1, 1));
-    m1 = fmaxf(m1, __shfl_xor_sync(0xFFFFFFFFu, m1, 2));
-    float z0 = 0.f, z1 = 0.f;
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t blk = kk >> 2, w = kk & 3;
+          tc::mma_bf16_ss(tmem + sb * kChunk, tc::sdesc_sw128(qbase + blk * kRows * 128 + w * 32),
+                          tc::sdesc_sw128(kbase + blk * kChunk * 128 + w * 32), idS, kk > 0);
+        }
+        tc::mma_commit(bar(BAR_S_FULL + sb));
+        tc::mma_commit(bar(BAR_Q_EMPTY + st));
+      };
+      auto issue_O = [&](int i) {
+        const int pb = i & 1;
+        tc::mbar_wait(bar(BAR_P_FULL + pb), (i >> 1) & 1, abort_flag, &g_fwd_status);
+        tc::mbar_wait(bar(BAR_O_EMPTY + pb), ((i >> 1) & 1) ^ 1, abort_flag, &g_fwd_status);
+        tc::fence_after_sync();
+        const uint32_t pbase = smem_u32(sm.P[pb]);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      s[i][0] = exp2f(s[i][0] - m0);
-      s[i][1] = exp2f(s[i][1] - m0);
-      s[i][2] = exp2f(s[i][2] - m1);
-      s[i][3] = exp2f(s[i][3] - m1);
-      z0 += s[i][0] + s[i][1];
-      z1 += s[i][2] + s[i][3];
-    }
-    z0 += __shfl_xor_sync(0xFFFFFFFFu, z0, 1);
-    z0 += __shfl_xor_sync(0xFFFFFFFFu, z0, 2);
-    z1 += __shfl_xor_sync(0xFFFFFFFFu, z1, 1);
-    z1 += __shfl_xor_sync(0xFFFFFFFFu, z1, 2);
-    const float i0 = 1.f / z0, i1 = 1.f / z1;
-    uint32_t pf[4][4];
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      pf[kk][0] = pack_bf16x2(s[2 * kk][0] * i0, s[2 * kk][1] * i0);
-      pf[kk][1] = pack_bf16x2(s[2 * kk][2] * i1, s[2 * kk][3] * i1);
-      pf[kk][2] = pack_bf16x2(s[2 * kk + 1][0] * i0, s[2 * kk + 1][1] * i0);
-      pf[kk][3] = pack_bf16x2(s[2 * kk + 1][2] * i1, s[2 * kk + 1][3] * i1);
-    }
-    // O' = P V : 16 rows x D
-    float o[D / 8][4];
-#pragma unroll
-    for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-#pragma unroll
-      for (int np = 0; np < D / 16; ++np) {
-        uint32_t bf[4];
-        ldsm_x4_t(bf, vb + swz<D>(16 * kk + (lane & 7) + 8 * ((lane >> 3) & 1), 16 * np + 8 * (lane >> 4)));
-        mma_bf16(o[2 * np], pf[kk], bf[0], bf[1]);
-        mma_bf16(o[2 * np + 1], pf[kk], bf[2], bf[3]);
+        for (int kk = 0; kk < kChunk / 16; ++kk)
+          tc::mma_bf16_ss(tmem + 2 * kChunk + pb * D, tc::sdesc_sw128(pbase + kk * 32),
+                          tc::sdesc_sw128(vbase + kk * 32), idO, kk > 0);
+        tc::mma_commit(bar(BAR_O_FULL + pb));
+      };
+      for (int i = 0; i < niter; ++i) {
+        issue_S(i);
+        if (i >= 1) issue_O(i - 1);
       }
-    }
-    // stage the warp's 16 rows (bf16) over its own, now dead, query rows
-    uint16_t* stage = sm.Q[buf];
-    const int rr = lane >> 2, cc = 2 * (lane & 3);
-#pragma unroll
-    for (int nt = 0; nt < D / 8; ++nt) {
-      *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(stage) + swz<D>(r0 + rr, 8 * nt + cc)) =
-          pack_bf16x2(o[nt][0], o[nt][1]);
-      *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(stage) + swz<D>(r0 + rr + 8, 8 * nt + cc)) =
-          pack_bf16x2(o[nt][2], o[nt][3]);
+      issue_O(niter - 1);
     }
     __syncwarp();
-    for (int u = lane; u < 16 * D8; u += 32) {
-      const int r = u / D8, ch = u % D8;
-      const int R = r0 + r;
-      const int e = it * epi + (R >> a.log2G);
-      if (e < cnt) {
-        const int p = a.entries[off + e];
-        const uint4 v = *reinterpret_cast<const uint4*>(reinterpret_cast<const char*>(stage) + swz<D>(R, ch * 8));
-        *reinterpret_cast<uint4*>(a.Opart + ((long long)p * a.G + (R & (a.G - 1))) * D + ch * 8) = v;
+  } else {
+    // ---------------------------------------------------------------- softmax + epilogue (thread = row)
+    const int r = tid;
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    auto epilogue = [&](int j) {
+      const int ob = j & 1;
+      tc::mbar_wait(bar(BAR_O_FULL + ob), (j >> 1) & 1, abort_flag, &g_fwd_status);
+      tc::fence_after_sync();
+      const int e = j * epi + (r >> a.log2G);
+      const bool valid = e < cnt;
+      uint16_t* dst = nullptr;
+      if (valid) dst = a.Opart + ((long long)a.entries[off + e] * a.G + (r & (a.G - 1))) * D;
+#pragma unroll
+      for (int h = 0; h < D / 32; ++h) {
+        float o[32];
+        tc::tmem_ld32(tmem + lane_base + 2 * kChunk + ob * D + h * 32, o);
+        tc::tmem_wait_ld();
+        if (valid) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + h * 32);
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4)
+            d4[q4] = make_uint4(pack_bf16x2(o[8 * q4], o[8 * q4 + 1]), pack_bf16x2(o[8 * q4 + 2], o[8 * q4 + 3]),
+                                pack_bf16x2(o[8 * q4 + 4], o[8 * q4 + 5]),
+                                pack_bf16x2(o[8 * q4 + 6], o[8 * q4 + 7]));
+        }
       }
+      tc::fence_before_sync();
+      tc::mbar_arrive(bar(BAR_O_EMPTY + ob));
+    };
+    for (int i = 0; i < niter; ++i) {
+      const int sb = i & 1;
+      tc::mbar_wait(bar(BAR_S_FULL + sb), (i >> 1) & 1, abort_flag, &g_fwd_status);
+      tc::fence_after_sync();
+      float x[64];
+      tc::tmem_ld32(tmem + lane_base + sb * kChunk, *reinterpret_cast<float(*)[32]>(&x[0]));
+      tc::tmem_ld32(tmem + lane_base + sb * kChunk + 32, *reinterpret_cast<float(*)[32]>(&x[32]));
+      tc::tmem_wait_ld();
+      tc::fence_before_sync();
+      tc::mbar_arrive(bar(BAR_S_EMPTY + sb));
+      float m = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < 64; ++k) {
+        x[k] *= a.scale_log2;
+        m = fmaxf(m, x[k]);
+      }
+      float z = 0.f;
+#pragma unroll
+      for (int k = 0; k < 64; ++k) {
+        x[k] = exp2f(x[k] - m);
+        z += x[k];
+      }
+      const float inv = 1.f / z;
+      const uint32_t prow = smem_u32(sm.P[sb]);
+#pragma unroll
+      for (int c16 = 0; c16 < 8; ++c16) {
+        const uint32_t dst = prow + tc::sw128_offset(kRows, r, c16 * 8);
+        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(dst),
+                     "r"(pack_bf16x2(x[8 * c16] * inv, x[8 * c16 + 1] * inv)),
+                     "r"(pack_bf16x2(x[8 * c16 + 2] * inv, x[8 * c16 + 3] * inv)),
+                     "r"(pack_bf16x2(x[8 * c16 + 4] * inv, x[8 * c16 + 5] * inv)),
+                     "r"(pack_bf16x2(x[8 * c16 + 6] * inv, x[8 * c16 + 7] * inv)));
+      }
+      tc::fence_proxy_async_smem();
+      tc::mbar_arrive(bar(BAR_P_FULL + sb));
+      if (i >= 1) epilogue(i - 1);
     }
-    __syncthreads();
+    epilogue(niter - 1);
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 8) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, kTmemCols);
   }
 }
 
@@ -263,7 +339,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.topk = Dm.topk;
     a.Nc = Dm.Nc;
     a.scale_log2 = Dm.scale_attn * 1.4426950408889634f;
-    const size_t smem = sizeof(FwdSmem<D>);
+    const size_t smem = sizeof(FwdSmem<D>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(fwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     fwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a);
@@ -278,6 +354,13 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
 }
 
 }  // namespace
+
+unsigned forward_take_status() {
+  unsigned v = 0, zero = 0;
+  if (cudaMemcpyFromSymbol(&v, g_fwd_status, sizeof(v)) != cudaSuccess) return ~0u;
+  cudaMemcpyToSymbol(g_fwd_status, &zero, sizeof(zero));
+  return v;
+}
 
 size_t forward_workspace(const Dims& D) { return (size_t)D.slots() * D.G * D.d * sizeof(uint16_t); }
 

@@ -11,7 +11,7 @@ import synth
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
-OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA = 0, 1, 2, 3, 4
+OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA, TIMEOUT = 0, 1, 2, 3, 4, 5
 
 
 def declared(header):
@@ -41,7 +41,7 @@ def test_synth_device_library_exports_its_header():
 
 
 def test_status_strings(lib):
-    for code in (OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA):
+    for code in (OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA, TIMEOUT):
         assert hsa.status_string(code).startswith("HSA_")
 
 

@@ -33,7 +33,7 @@
  *            launch nothing.
  *   Support  d in {64, 128}; S = 64; Hq a multiple of Hkv with
  *            G = Hq/Hkv in {1, 2, 4, 8, 16}; 1 <= topk <= 32;
- *            B * L * Hkv * topk < 2^31.
+ *            B * L * Hkv * topk < 2^31 and B * L * Hq < 2^31.
  *   Causality Token t (0-indexed) sees the completed chunks before its own
  *            chunk (i < t/S); a trailing partial chunk is never selectable.
  *            Fewer visible chunks than topk: all are selected and the rest of

@@ -36,8 +36,8 @@ hsa_status_t resolve(const hsa_shape_t* s, Dims* out) {
   if (s->topk > 32) return HSA_ERR_UNSUPPORTED;
   const long long slots = (long long)s->B * s->L * s->Hkv * s->topk;
   if (slots >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
-  const long long rows = (long long)s->B * s->L * s->Hq;
-  if (rows >= (1LL << 40)) return HSA_ERR_UNSUPPORTED;
+  const long long rows = (long long)s->B * s->L * s->Hq;  // query rows are indexed in int32
+  if (rows >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
   Dims D;
   D.B = s->B;
   D.L = s->L;

@@ -29,6 +29,7 @@ struct FwdSmem {
   uint16_t K[kChunk * D];           // chunk keys [s][d]
   uint16_t Vt[D * kChunk];          // chunk values transposed [d][s]
   uint16_t P[2][kRows * kChunk];    // normalised probabilities (bf16)
+  int slot_row[kQStages][kRows];    // first q row of each slot of a tile (-1: past the list)
   uint64_t bar[16];
   uint32_t tmem_base;
   int abort_flag;
@@ -115,21 +116,31 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
 
   if (warp >= 4 && warp < 8) {
     // ---------------------------------------------------------------- loaders
+    // Per tile: one thread per slot resolves the slot's first query row, then
+    // the 128 loader threads copy 128 rows x D columns with table lookups.
     const int lt = tid - 128;
     for (int i = 0; i < niter; ++i) {
       const int st = i % kQStages;
       tc::mbar_wait(bar(BAR_Q_EMPTY + st), ((i / kQStages) & 1) ^ 1, abort_flag, &g_fwd_status);
-      const uint32_t base = smem_u32(sm.Q[st]);
-      for (int u = lt; u < kRows * D8; u += 128) {
-        const int r = u / D8, ch = u % D8;
-        const int e = i * epi + (r >> a.log2G);
-        const uint32_t dst = base + tc::sw128_offset(kRows, r, ch * 8);
+      if (lt < epi) {
+        const int e = i * epi + lt;
+        int row = -1;
         if (e < cnt) {
           const int p = a.entries[off + e];
           const int t = (p / slot_div) % a.L;
-          const long long src =
-              (((long long)b * a.L + t) * a.Hq + (long long)g * a.G + (r & (a.G - 1))) * D + ch * 8;
-          cp_async16(dst, a.q + src);
+          row = ((b * a.L + t) * a.Hq) + g * a.G;
+        }
+        sm.slot_row[st][lt] = row;
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      const uint32_t base = smem_u32(sm.Q[st]);
+#pragma unroll 4
+      for (int u = lt; u < kRows * D8; u += 128) {
+        const int r = u / D8, ch = u % D8;
+        const int row = sm.slot_row[st][r >> a.log2G];
+        const uint32_t dst = base + tc::sw128_offset(kRows, r, ch * 8);
+        if (row >= 0) {
+          cp_async16(dst, a.q + ((long long)(row + (r & (a.G - 1)))) * D + ch * 8);
         } else {
           asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(dst), "r"(0));
         }
@@ -188,14 +199,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
     // ---------------------------------------------------------------- softmax + epilogue (thread = row)
     const int r = tid;
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-    auto epilogue = [&](int j) {
+    auto epilogue = [&](int j, int pj) {
       const int ob = j & 1;
       tc::mbar_wait(bar(BAR_O_FULL + ob), (j >> 1) & 1, abort_flag, &g_fwd_status);
       tc::fence_after_sync();
-      const int e = j * epi + (r >> a.log2G);
-      const bool valid = e < cnt;
+      const bool valid = pj >= 0;
       uint16_t* dst = nullptr;
-      if (valid) dst = a.Opart + ((long long)a.entries[off + e] * a.G + (r & (a.G - 1))) * D;
+      if (valid) dst = a.Opart + ((long long)pj * a.G + (r & (a.G - 1))) * D;
 #pragma unroll
       for (int h = 0; h < D / 32; ++h) {
         float o[32];
@@ -213,8 +223,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_O_EMPTY + ob));
     };
+    int p_prev = -1;
     for (int i = 0; i < niter; ++i) {
       const int sb = i & 1;
+      const int e_i = i * epi + (r >> a.log2G);
+      const int p_i = e_i < cnt ? a.entries[off + e_i] : -1;  // used by this step's epilogue
       tc::mbar_wait(bar(BAR_S_FULL + sb), (i >> 1) & 1, abort_flag, &g_fwd_status);
       tc::fence_after_sync();
       float x[64];
@@ -248,9 +261,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
       }
       tc::fence_proxy_async_smem();
       tc::mbar_arrive(bar(BAR_P_FULL + sb));
-      if (i >= 1) epilogue(i - 1);
+      if (i >= 1) epilogue(i - 1, p_prev);
+      p_prev = p_i;
     }
-    epilogue(niter - 1);
+    epilogue(niter - 1, p_prev);
   }
   tc::fence_before_sync();
   __syncthreads();

@@ -85,9 +85,9 @@ unsigned long long hsa_kernel_launches(void) { return hsa::g_launches.load(std::
 
 hsa_status_t hsa_device_check(void) {
   if (cudaDeviceSynchronize() != cudaSuccess) return HSA_ERR_CUDA;
-  const unsigned s = hsa::forward_take_status();
-  if (s == ~0u) return HSA_ERR_CUDA;
-  return s ? HSA_ERR_TIMEOUT : HSA_OK;
+  const unsigned s1 = hsa::forward_take_status(), s2 = hsa::backward_take_status();
+  if (s1 == ~0u || s2 == ~0u) return HSA_ERR_CUDA;
+  return (s1 | s2) ? HSA_ERR_TIMEOUT : HSA_OK;
 }
 
 size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {

@@ -20,30 +20,58 @@
 //
 // Chunk-major and deterministic: one block per (b, g, chunk) owns that
 // chunk's dK/dV rows, walks the chunk's slots (from the inverse index) in
-// increasing token order 128 query rows at a time and accumulates dK, dV and
-// dK̄ on chip; no floating-point atomics anywhere. Each slot's dq
+// increasing token order 128 query rows at a time and accumulates dK^T and
+// dV^T in tensor memory; no floating-point atomics anywhere. Each slot's dq
 // contribution goes to a bf16 workspace row and a second kernel sums the k
 // slots of each token in slot order (fp32).
-#include "common.cuh"
+//
+// Per 128-row step on the 5th-generation tensor core (one issuing thread):
+//   S = Q K^T, dP' = dO V^T            (M = 128 rows, N = 64, K = d)
+//   dq' = dSq K                        (K read as an MN-major operand)
+//   dV^T += dO^T (wP), dK^T += Q^T dSk (M = d, N = 64, K = 128 rows; the
+//                                       row-major tiles read MN-major)
+// Warps 0-3 (one thread per row) turn S, dP' into P, dSq, dSk and store dq';
+// warps 4-7 gather the Q and dO rows of the next tiles.
+#include "tc.cuh"
 
 namespace hsa {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kRows = 128;
+constexpr int kRows = 128;     // query rows per step (tensor-core M)
+constexpr int kThreads = 288;  // 4 softmax/epilogue warps, 4 loader warps, 1 MMA warp
+constexpr int kTmemCols = 512;
+
+__device__ unsigned g_bwd_status;
 
 template <int D>
 struct BwdSmem {
-  uint16_t K[kChunk * D];
-  uint16_t V[kChunk * D];
-  uint16_t Q[2][kRows * D];
-  uint16_t dO[2][kRows * D];
-  uint16_t P[kRows * kChunk];   // w * P, bf16
-  uint16_t dS[kRows * kChunk];  // c_att * w * P∘(dP' - D) + c_sel * ds / S, bf16
+  uint16_t Q[2][kRows * D];       // gathered query rows (K-major SW128)
+  uint16_t dO[2][kRows * D];      // gathered output gradients
+  uint16_t K[kChunk * D];         // chunk keys [s][d]
+  uint16_t V[kChunk * D];         // chunk values [s][d]
+  uint16_t P[kRows * kChunk];     // w * P
+  uint16_t dSq[kRows * kChunk];   // c_att * w * P∘(dP' - D)            (feeds dq)
+  uint16_t dSk[kRows * kChunk];   // dSq + c_sel * ds / S               (feeds dK: attention + mean pool)
   float kbar[D];
-  float wslot[2][kRows];
-  float delta[2][kRows];
-  int pslot[2][kRows];
+  int slot_row[2][kRows];         // first q row of each slot (-1: past the list)
+  int slot_p[2][kRows];
+  float slot_w[2][kRows];
+  float slot_delta[2][kRows];
+  uint64_t bar[16];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+enum {
+  BAR_QD_FULL = 0,   // 2: Q and dO tiles landed (128 loader arrivals)
+  BAR_QD_EMPTY = 2,  // 2: every MMA reading the tiles finished (commit)
+  BAR_S_FULL = 4,    // 2: S and dP' ready (commit)
+  BAR_S_EMPTY = 6,   // 2: S and dP' read (128 arrivals)
+  BAR_P_FULL = 8,    // P, dSq, dSk written (128 arrivals)
+  BAR_P_EMPTY = 9,   // P, dSq, dSk consumed (commit)
+  BAR_DQ_FULL = 10,  // dq accumulator ready (commit)
+  BAR_DQ_EMPTY = 11, // dq read (128 arrivals)
+  BAR_ACC_DONE = 12  // last dK^T / dV^T update finished (commit)
 };
 
 struct BwdArgs {
@@ -63,259 +91,315 @@ struct BwdArgs {
   float scale_log2, scale_attn, scale_sel;
 };
 
+// TMEM columns
+template <int D>
+struct Cols {
+  static constexpr uint32_t S = 0;            // 2 x 64
+  static constexpr uint32_t dP = 128;         // 2 x 64
+  static constexpr uint32_t dq = 256;         // D
+  static constexpr uint32_t dVt = 256 + D;    // 64 (rows = head dim)
+  static constexpr uint32_t dKt = 320 + D;    // 64
+};
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw);
+  extern __shared__ unsigned char smem_raw[];
+  BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
-  constexpr int NH = D / 2;  // head-dim columns owned per warp for dK/dV
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int key = blockIdx.x;
   const int c = key % a.Nc, bg = key / a.Nc;
   const int b = bg / a.Hkv, g = bg % a.Hkv;
   const int off = a.offsets[key];
   const int cnt = a.offsets[key + 1] - off;
+  const long long row0 = ((long long)b * a.L + (long long)c * kChunk) * a.Hkv + g;
+  if (cnt <= 0) {  // a chunk nobody selected: no gradient
+    for (int u = tid; u < kChunk * D; u += kThreads) {
+      const long long o = (row0 + (long long)(u / D) * a.Hkv) * D + (u % D);
+      a.dK[o] = 0.f;
+      a.dV[o] = 0.f;
+    }
+    return;
+  }
   const int epi = kRows >> a.log2G;
   const int niter = (cnt + epi - 1) / epi;
   const int slot_div = a.Hkv * a.topk;
-  const long long row0 = ((long long)b * a.L + (long long)c * kChunk) * a.Hkv + g;
+  auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
+  volatile int* abort_flag = &sm.abort_flag;
+  unsigned* status = &g_bwd_status;
 
-  // warp-owned dK/dV sub-tile: chunk rows sr0..sr0+15, head dims dc0..dc0+NH-1
-  const int sr0 = 16 * (warp & 3), dc0 = NH * (warp >> 2);
-  float dv[NH / 8][4], dk[NH / 8][4];
-#pragma unroll
-  for (int i = 0; i < NH / 8; ++i) dv[i][0] = dv[i][1] = dv[i][2] = dv[i][3] = dk[i][0] = dk[i][1] = dk[i][2] =
-      dk[i][3] = 0.f;
-
-  if (cnt > 0) {
-    for (int u = tid; u < kChunk * D8; u += kThreads) {
-      const int r = u / D8, ch = u % D8;
-      const long long src = (row0 + (long long)r * a.Hkv) * D + ch * 8;
-      cp_async16(smem_u32(sm.K) + swz<D>(r, ch * 8), a.K + src);
-      cp_async16(smem_u32(sm.V) + swz<D>(r, ch * 8), a.V + src);
+  if (tid == 0) {
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(bar(BAR_QD_FULL + i), 128);
+      tc::mbar_init(bar(BAR_QD_EMPTY + i), 1);
+      tc::mbar_init(bar(BAR_S_FULL + i), 1);
+      tc::mbar_init(bar(BAR_S_EMPTY + i), 128);
     }
-    for (int u = tid; u < D; u += kThreads) sm.kbar[u] = a.kbar32[(((long long)b * a.Nc + c) * a.Hkv + g) * D + u];
+    tc::mbar_init(bar(BAR_P_FULL), 128);
+    tc::mbar_init(bar(BAR_P_EMPTY), 1);
+    tc::mbar_init(bar(BAR_DQ_FULL), 1);
+    tc::mbar_init(bar(BAR_DQ_EMPTY), 128);
+    tc::mbar_init(bar(BAR_ACC_DONE), 1);
+    sm.abort_flag = 0;
+    tc::fence_mbar_init();
   }
-  auto load_tile = [&](int it, int buf) {
-    const uint32_t qbase = smem_u32(sm.Q[buf]), obase = smem_u32(sm.dO[buf]);
-    for (int u = tid; u < kRows * D8; u += kThreads) {
-      const int r = u / D8, ch = u % D8;
-      const int e = it * epi + (r >> a.log2G);
-      const uint32_t o = swz<D>(r, ch * 8);
-      if (e < cnt) {
-        const int p = a.entries[off + e];
-        const int t = (p / slot_div) % a.L;
-        const long long src = (((long long)b * a.L + t) * a.Hq + (long long)g * a.G + (r & (a.G - 1))) * D + ch * 8;
-        cp_async16(qbase + o, a.q + src);
-        cp_async16(obase + o, a.dO + src);
-      } else {
-        asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(qbase + o), "r"(0));
-        asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(obase + o), "r"(0));
-      }
+  if (warp == 8) tc::tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+  if (warp >= 4 && warp < 8) {  // chunk K, V (rows s) and K̄, once per block
+    const int lt = tid - 128;
+    for (int u = lt; u < kChunk * D8; u += 128) {
+      const int srow = u / D8, ch = u % D8;
+      const long long src = (row0 + (long long)srow * a.Hkv) * D + ch * 8;
+      cp_async16(smem_u32(sm.K) + tc::sw128_offset(kChunk, srow, ch * 8), a.K + src);
+      cp_async16(smem_u32(sm.V) + tc::sw128_offset(kChunk, srow, ch * 8), a.V + src);
     }
-    if (tid < epi) {
-      const int e = it * epi + tid;
-      if (e < cnt) {
-        const int p = a.entries[off + e];
-        const int t = (p / slot_div) % a.L;
-        sm.pslot[buf][tid] = p;
-        sm.wslot[buf][tid] = a.w[p];
-        sm.delta[buf][tid] = a.delta[((long long)b * a.L + t) * a.Hkv + g];
-      } else {
-        sm.pslot[buf][tid] = -1;
-        sm.wslot[buf][tid] = 0.f;
-        sm.delta[buf][tid] = 0.f;
-      }
-    }
-  };
-  if (niter > 0) load_tile(0, 0);
-  cp_async_commit();
-
-  const uint32_t kb = smem_u32(sm.K), vb = smem_u32(sm.V);
-  const uint32_t pb = smem_u32(sm.P), db = smem_u32(sm.dS);
-  const int rr = lane >> 2, cc = 2 * (lane & 3);
-  for (int it = 0; it < niter; ++it) {
-    const int buf = it & 1;
-    if (it + 1 < niter) load_tile(it + 1, buf ^ 1);
+    for (int u = lt; u < D; u += 128) sm.kbar[u] = a.kbar32[(((long long)b * a.Nc + c) * a.Hkv + g) * D + u];
     cp_async_commit();
-    cp_async_wait<1>();
-    __syncthreads();
-    const uint32_t qb = smem_u32(sm.Q[buf]), ob = smem_u32(sm.dO[buf]);
-    const int r0 = warp * 16;
+    cp_async_wait<0>();
+    tc::fence_proxy_async_smem();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = sm.tmem_base;
 
-    // S = Q K^T and dP' = dO V^T (16 rows x 64 keys per warp)
-    float s[8][4], dp[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) s[i][j] = dp[i][j] = 0.f;
-#pragma unroll
-    for (int kd = 0; kd < D / 16; ++kd) {
-      uint32_t aq[4], ad[4];
-      const int ar = r0 + (lane & 7) + 8 * ((lane >> 3) & 1), ac = 16 * kd + 8 * (lane >> 4);
-      ldsm_x4(aq, qb + swz<D>(ar, ac));
-      ldsm_x4(ad, ob + swz<D>(ar, ac));
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        uint32_t bk[4], bv[4];
-        const int br = 16 * np + (lane & 7) + 8 * (lane >> 4), bc = 16 * kd + 8 * ((lane >> 3) & 1);
-        ldsm_x4(bk, kb + swz<D>(br, bc));
-        ldsm_x4(bv, vb + swz<D>(br, bc));
-        mma_bf16(s[2 * np], aq, bk[0], bk[1]);
-        mma_bf16(s[2 * np + 1], aq, bk[2], bk[3]);
-        mma_bf16(dp[2 * np], ad, bv[0], bv[1]);
-        mma_bf16(dp[2 * np + 1], ad, bv[2], bv[3]);
+  if (warp >= 4 && warp < 8) {
+    // ---------------------------------------------------------------- loaders
+    const int lt = tid - 128;
+    for (int i = 0; i < niter; ++i) {
+      const int st = i & 1;
+      // publish tile i-1 before waiting for tile i's stage: that stage is freed
+      // by the second half of step i-2, which the MMA thread issues only after
+      // the first half of step i-1 (which needs tile i-1)
+      if (i >= 1) {
+        cp_async_wait<0>();
+        tc::fence_proxy_async_smem();
+        tc::mbar_arrive(bar(BAR_QD_FULL + ((i - 1) & 1)));
       }
-    }
-    // P = softmax(c_att S) per row
-    float m0 = -INFINITY, m1 = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-#pragma unroll
-      for (int j = 0; j < 4; ++j) s[i][j] *= a.scale_log2;
-      m0 = fmaxf(m0, fmaxf(s[i][0], s[i][1]));
-      m1 = fmaxf(m1, fmaxf(s[i][2], s[i][3]));
-    }
-    m0 = fmaxf(m0, __shfl_xor_sync(0xFFFFFFFFu, m0, 1));
-    m0 = fmaxf(m0, __shfl_xor_sync(0xFFFFFFFFu, m0, 2));
-    m1 = fmaxf(m1, __shfl_xor_sync(0xFFFFFFFFu, m1, 1));
-    m1 = fmaxf(m1, __shfl_xor_sync(0xFFFFFFFFu, m1, 2));
-    float z0 = 0.f, z1 = 0.f;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      s[i][0] = exp2f(s[i][0] - m0);
-      s[i][1] = exp2f(s[i][1] - m0);
-      s[i][2] = exp2f(s[i][2] - m1);
-      s[i][3] = exp2f(s[i][3] - m1);
-      z0 += s[i][0] + s[i][1];
-      z1 += s[i][2] + s[i][3];
-    }
-    z0 += __shfl_xor_sync(0xFFFFFFFFu, z0, 1);
-    z0 += __shfl_xor_sync(0xFFFFFFFFu, z0, 2);
-    z1 += __shfl_xor_sync(0xFFFFFFFFu, z1, 1);
-    z1 += __shfl_xor_sync(0xFFFFFFFFu, z1, 2);
-    const float i0 = 1.f / z0, i1 = 1.f / z1;
-    float D0 = 0.f, D1 = 0.f;  // D_h = sum_s P_s dP'_s
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      s[i][0] *= i0;
-      s[i][1] *= i0;
-      s[i][2] *= i1;
-      s[i][3] *= i1;
-      D0 += s[i][0] * dp[i][0] + s[i][1] * dp[i][1];
-      D1 += s[i][2] * dp[i][2] + s[i][3] * dp[i][3];
-    }
-    D0 += __shfl_xor_sync(0xFFFFFFFFu, D0, 1);
-    D0 += __shfl_xor_sync(0xFFFFFFFFu, D0, 2);
-    D1 += __shfl_xor_sync(0xFFFFFFFFu, D1, 1);
-    D1 += __shfl_xor_sync(0xFFFFFFFFu, D1, 2);
-    // dw per slot: sum of D over the G rows of the slot (rows are grouped in
-    // runs of G inside each 8-row half of the warp tile; G = 16 spans both)
-    float dw0 = D0, dw1 = D1;
-    const int gl = a.G < 8 ? a.G : 8;
-    for (int o = 4; o < 4 * gl; o <<= 1) {
-      dw0 += __shfl_xor_sync(0xFFFFFFFFu, dw0, o);
-      dw1 += __shfl_xor_sync(0xFFFFFFFFu, dw1, o);
-    }
-    if (a.G == 16) dw0 = dw1 = dw0 + dw1;
-    const int R0 = r0 + rr, R1 = R0 + 8;
-    const int sl0 = R0 >> a.log2G, sl1 = R1 >> a.log2G;
-    const float w0 = sm.wslot[buf][sl0], w1 = sm.wslot[buf][sl1];
-    const float ds0 = w0 * (dw0 - sm.delta[buf][sl0]);
-    const float ds1 = w1 * (dw1 - sm.delta[buf][sl1]);
-    const float pool0 = a.scale_sel * ds0 * (1.f / kChunk), pool1 = a.scale_sel * ds1 * (1.f / kChunk);
-    // da (scaled by c_att for the products) and w P, to fragments and shared tiles
-    const float ca0 = a.scale_attn * w0, ca1 = a.scale_attn * w1;
-    uint32_t dsf[4][4];
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int nt = 2 * kk + h;
-        const float g00 = ca0 * s[nt][0] * (dp[nt][0] - D0), g01 = ca0 * s[nt][1] * (dp[nt][1] - D0);
-        const float g10 = ca1 * s[nt][2] * (dp[nt][2] - D1), g11 = ca1 * s[nt][3] * (dp[nt][3] - D1);
-        dsf[kk][2 * h] = pack_bf16x2(g00, g01);
-        dsf[kk][2 * h + 1] = pack_bf16x2(g10, g11);
-        const uint32_t p0 = pack_bf16x2(w0 * s[nt][0], w0 * s[nt][1]);
-        const uint32_t p1 = pack_bf16x2(w1 * s[nt][2], w1 * s[nt][3]);
-        *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(sm.P) + swz<kChunk>(R0, 8 * nt + cc)) = p0;
-        *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(sm.P) + swz<kChunk>(R1, 8 * nt + cc)) = p1;
-        *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(sm.dS) + swz<kChunk>(R0, 8 * nt + cc)) =
-            pack_bf16x2(g00 + pool0, g01 + pool0);
-        *reinterpret_cast<uint32_t*>(reinterpret_cast<char*>(sm.dS) + swz<kChunk>(R1, 8 * nt + cc)) =
-            pack_bf16x2(g10 + pool1, g11 + pool1);
+      tc::mbar_wait(bar(BAR_QD_EMPTY + st), ((i >> 1) & 1) ^ 1, abort_flag, status);
+      if (lt < epi) {
+        const int e = i * epi + lt;
+        int row = -1, p = -1;
+        float wv = 0.f, dl = 0.f;
+        if (e < cnt) {
+          p = a.entries[off + e];
+          const int t = (p / slot_div) % a.L;
+          row = ((b * a.L + t) * a.Hq) + g * a.G;
+          wv = a.w[p];
+          dl = a.delta[((long long)b * a.L + t) * a.Hkv + g];
+        }
+        sm.slot_row[st][lt] = row;
+        sm.slot_p[st][lt] = p;
+        sm.slot_w[st][lt] = wv;
+        sm.slot_delta[st][lt] = dl;
       }
-    }
-    // dsf[kk] is already in A-fragment order {row0 keys 0-7, row1 keys 0-7, row0 keys 8-15, row1 keys 8-15}
-    // dq rows: (c_att w da-part) K + c_sel ds K̄, written per slot
-    const int e0 = it * epi + sl0, e1 = it * epi + sl1;
-    const int p0 = e0 < cnt ? sm.pslot[buf][sl0] : -1;
-    const int p1 = e1 < cnt ? sm.pslot[buf][sl1] : -1;
-    uint16_t* dq0 = p0 >= 0 ? a.dqpart + ((long long)p0 * a.G + (R0 & (a.G - 1))) * D : nullptr;
-    uint16_t* dq1 = p1 >= 0 ? a.dqpart + ((long long)p1 * a.G + (R1 & (a.G - 1))) * D : nullptr;
-    const float cs0 = a.scale_sel * ds0, cs1 = a.scale_sel * ds1;
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      float acc[D / 16][4];
-#pragma unroll
-      for (int i = 0; i < D / 16; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-        const uint32_t af[4] = {dsf[kk][0], dsf[kk][1], dsf[kk][2], dsf[kk][3]};
-#pragma unroll
-        for (int np = 0; np < D / 32; ++np) {
-          uint32_t bf[4];
-          const int col = half * (D / 2) + 16 * np;
-          ldsm_x4_t(bf, kb + swz<D>(16 * kk + (lane & 7) + 8 * ((lane >> 3) & 1), col + 8 * (lane >> 4)));
-          mma_bf16(acc[2 * np], af, bf[0], bf[1]);
-          mma_bf16(acc[2 * np + 1], af, bf[2], bf[3]);
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
+#pragma unroll 4
+      for (int u = lt; u < kRows * D8; u += 128) {
+        const int r = u / D8, ch = u % D8;
+        const int row = sm.slot_row[st][r >> a.log2G];
+        const uint32_t o = tc::sw128_offset(kRows, r, ch * 8);
+        if (row >= 0) {
+          const long long src = ((long long)(row + (r & (a.G - 1)))) * D + ch * 8;
+          cp_async16(qb + o, a.q + src);
+          cp_async16(ob + o, a.dO + src);
+        } else {
+          asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(qb + o), "r"(0));
+          asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(ob + o), "r"(0));
         }
       }
+      cp_async_commit();
+    }
+    cp_async_wait<0>();
+    tc::fence_proxy_async_smem();
+    tc::mbar_arrive(bar(BAR_QD_FULL + ((niter - 1) & 1)));
+  } else if (warp == 8) {
+    // ---------------------------------------------------------------- MMA issue (one thread)
+    if (lane == 0) {
+      constexpr uint32_t idSP = tc::idesc_bf16(kRows, kChunk);                // S, dP': Q K^T, dO V^T
+      constexpr uint32_t idDQ = tc::idesc_bf16(kRows, D, false, true);        // dq = dSq K   (K as MN-major B)
+      constexpr uint32_t idKV = tc::idesc_bf16(kRows, kChunk, true, true);    // dV^T, dK^T  (both MN-major)
+      // head-dim operands of M = 128: the second 64-block sits one tile block
+      // further; with D = 64 it repeats the first (rows 64..127 are unused)
+      constexpr uint32_t kMnQ = D == 128 ? (uint32_t)kRows * 128 : 0u;
+      constexpr uint32_t kMnK = (uint32_t)kChunk * 128;
+      const uint32_t kbase = smem_u32(sm.K), vbase = smem_u32(sm.V);
+      const uint32_t pbase = smem_u32(sm.P), dsq = smem_u32(sm.dSq), dsk = smem_u32(sm.dSk);
+      auto issue_SdP = [&](int i) {
+        const int st = i & 1, sb = i & 1;
+        tc::mbar_wait(bar(BAR_QD_FULL + st), (i >> 1) & 1, abort_flag, status);
+        tc::mbar_wait(bar(BAR_S_EMPTY + sb), ((i >> 1) & 1) ^ 1, abort_flag, status);
+        tc::fence_after_sync();
+        const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
 #pragma unroll
-      for (int nt = 0; nt < D / 16; ++nt) {
-        const int col = half * (D / 2) + 8 * nt + cc;
-        if (dq0)
-          *reinterpret_cast<uint32_t*>(dq0 + col) =
-              pack_bf16x2(acc[nt][0] + cs0 * sm.kbar[col], acc[nt][1] + cs0 * sm.kbar[col + 1]);
-        if (dq1)
-          *reinterpret_cast<uint32_t*>(dq1 + col) =
-              pack_bf16x2(acc[nt][2] + cs1 * sm.kbar[col], acc[nt][3] + cs1 * sm.kbar[col + 1]);
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t blk = kk >> 2, wq = kk & 3;
+          const uint32_t ao = blk * kRows * 128 + wq * 32, bo = blk * kChunk * 128 + wq * 32;
+          tc::mma_bf16_ss(tmem + Cols<D>::S + sb * kChunk, tc::sdesc_sw128(qb + ao), tc::sdesc_sw128(kbase + bo),
+                          idSP, kk > 0);
+          tc::mma_bf16_ss(tmem + Cols<D>::dP + sb * kChunk, tc::sdesc_sw128(ob + ao), tc::sdesc_sw128(vbase + bo),
+                          idSP, kk > 0);
+        }
+        tc::mma_commit(bar(BAR_S_FULL + sb));
+      };
+      auto issue_rest = [&](int i) {
+        const int st = i & 1;
+        tc::mbar_wait(bar(BAR_P_FULL), i & 1, abort_flag, status);
+        tc::mbar_wait(bar(BAR_DQ_EMPTY), (i & 1) ^ 1, abort_flag, status);
+        tc::fence_after_sync();
+        // dq' = dSq K : M = 128 rows, N = D, K = 64 chunk rows
+#pragma unroll
+        for (int kk = 0; kk < kChunk / 16; ++kk)
+          tc::mma_bf16_ss(tmem + Cols<D>::dq, tc::sdesc_sw128(dsq + kk * 32),
+                          tc::sdesc_sw128_mn(kbase + kk * 2048, kMnK), idDQ, kk > 0);
+        tc::mma_commit(bar(BAR_DQ_FULL));
+        // dV^T += dO^T (wP), dK^T += Q^T dSk : M = head dim, N = 64, K = 128 rows
+        const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
+#pragma unroll
+        for (int kk = 0; kk < kRows / 16; ++kk) {
+          const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
+          tc::mma_bf16_ss(tmem + Cols<D>::dVt, tc::sdesc_sw128_mn(ob + kk * 2048, kMnQ),
+                          tc::sdesc_sw128_mn(pbase + kk * 2048, 0), idKV, acc);
+          tc::mma_bf16_ss(tmem + Cols<D>::dKt, tc::sdesc_sw128_mn(qb + kk * 2048, kMnQ),
+                          tc::sdesc_sw128_mn(dsk + kk * 2048, 0), idKV, acc);
+        }
+        tc::mma_commit(bar(BAR_QD_EMPTY + st));
+        tc::mma_commit(bar(BAR_P_EMPTY));
+      };
+      for (int i = 0; i < niter; ++i) {
+        issue_SdP(i);
+        if (i >= 1) issue_rest(i - 1);
+      }
+      issue_rest(niter - 1);
+      tc::mma_commit(bar(BAR_ACC_DONE));
+    }
+    __syncwarp();
+  } else {
+    // ---------------------------------------------------------------- softmax / gradient rows (thread = row)
+    const int r = tid;
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    const float inv_S = 1.f / (float)kChunk;
+    auto dq_epilogue = [&](int j, int pj, float dsj) {
+      tc::mbar_wait(bar(BAR_DQ_FULL), j & 1, abort_flag, status);
+      tc::fence_after_sync();
+      uint16_t* dst = pj >= 0 ? a.dqpart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
+      const float cs = a.scale_sel * dsj;
+#pragma unroll
+      for (int h = 0; h < D / 32; ++h) {
+        float v[32];
+        tc::tmem_ld32(tmem + lane_base + Cols<D>::dq + h * 32, v);
+        tc::tmem_wait_ld();
+        if (dst) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + h * 32);
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            float o[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) o[k] = v[8 * q4 + k] + cs * sm.kbar[h * 32 + 8 * q4 + k];
+            d4[q4] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
+                                pack_bf16x2(o[6], o[7]));
+          }
+        }
+      }
+      tc::fence_before_sync();
+      tc::mbar_arrive(bar(BAR_DQ_EMPTY));
+    };
+    int p_prev = -1;
+    float ds_prev = 0.f;
+    for (int i = 0; i < niter; ++i) {
+      const int sb = i & 1, st = i & 1;
+      tc::mbar_wait(bar(BAR_S_FULL + sb), (i >> 1) & 1, abort_flag, status);
+      tc::fence_after_sync();
+      float x[64], y[64];
+      tc::tmem_ld32(tmem + lane_base + Cols<D>::S + sb * kChunk, *reinterpret_cast<float(*)[32]>(&x[0]));
+      tc::tmem_ld32(tmem + lane_base + Cols<D>::S + sb * kChunk + 32, *reinterpret_cast<float(*)[32]>(&x[32]));
+      tc::tmem_ld32(tmem + lane_base + Cols<D>::dP + sb * kChunk, *reinterpret_cast<float(*)[32]>(&y[0]));
+      tc::tmem_ld32(tmem + lane_base + Cols<D>::dP + sb * kChunk + 32, *reinterpret_cast<float(*)[32]>(&y[32]));
+      tc::tmem_wait_ld();
+      tc::fence_before_sync();
+      tc::mbar_arrive(bar(BAR_S_EMPTY + sb));
+      // the loaders' slot tables of this tile (released with BAR_QD_FULL, whose
+      // phase cannot advance before this thread has produced the step's P)
+      tc::mbar_wait(bar(BAR_QD_FULL + st), (i >> 1) & 1, abort_flag, status);
+      const int slot = r >> a.log2G;
+      const float wv = sm.slot_w[st][slot], dl = sm.slot_delta[st][slot];
+      const int pv = sm.slot_p[st][slot];
+      float m = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < 64; ++k) {
+        x[k] *= a.scale_log2;
+        m = fmaxf(m, x[k]);
+      }
+      float z = 0.f;
+#pragma unroll
+      for (int k = 0; k < 64; ++k) {
+        x[k] = exp2f(x[k] - m);
+        z += x[k];
+      }
+      const float inv = 1.f / z;
+      float Drow = 0.f;
+#pragma unroll
+      for (int k = 0; k < 64; ++k) {
+        x[k] *= inv;
+        Drow += x[k] * y[k];
+      }
+      float dw = Drow;  // sum over the G rows of the slot (consecutive lanes)
+      for (int o = 1; o < a.G; o <<= 1) dw += __shfl_xor_sync(0xFFFFFFFFu, dw, o);
+      const float dsv = wv * (dw - dl);
+      const float ca = a.scale_attn * wv, pool = a.scale_sel * dsv * inv_S;
+      tc::mbar_wait(bar(BAR_P_EMPTY), (i & 1) ^ 1, abort_flag, status);
+      const uint32_t prow = smem_u32(sm.P), qrow = smem_u32(sm.dSq), krow = smem_u32(sm.dSk);
+#pragma unroll
+      for (int c16 = 0; c16 < 8; ++c16) {
+        const uint32_t o = tc::sw128_offset(kRows, r, c16 * 8);
+        uint32_t pp[4], gq[4], gk[4];
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const int k0 = 8 * c16 + 2 * h;
+          const float g0 = ca * x[k0] * (y[k0] - Drow), g1 = ca * x[k0 + 1] * (y[k0 + 1] - Drow);
+          pp[h] = pack_bf16x2(wv * x[k0], wv * x[k0 + 1]);
+          gq[h] = pack_bf16x2(g0, g1);
+          gk[h] = pack_bf16x2(g0 + pool, g1 + pool);
+        }
+        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(prow + o), "r"(pp[0]), "r"(pp[1]), "r"(pp[2]),
+                     "r"(pp[3]));
+        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(qrow + o), "r"(gq[0]), "r"(gq[1]), "r"(gq[2]),
+                     "r"(gq[3]));
+        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(krow + o), "r"(gk[0]), "r"(gk[1]), "r"(gk[2]),
+                     "r"(gk[3]));
+      }
+      tc::fence_proxy_async_smem();
+      tc::mbar_arrive(bar(BAR_P_FULL));
+      if (i >= 1) dq_epilogue(i - 1, p_prev, ds_prev);
+      p_prev = pv;
+      ds_prev = dsv;
+    }
+    dq_epilogue(niter - 1, p_prev, ds_prev);
+    // dK, dV of the chunk: TMEM lane = head dim, column = chunk row
+    tc::mbar_wait(bar(BAR_ACC_DONE), 0, abort_flag, status);
+    tc::fence_after_sync();
+    if (warp * 32 < D) {
+      const int dcol = r;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        float dv[32], dk[32];
+        tc::tmem_ld32(tmem + lane_base + Cols<D>::dVt + h * 32, dv);
+        tc::tmem_ld32(tmem + lane_base + Cols<D>::dKt + h * 32, dk);
+        tc::tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          const long long o = (row0 + (long long)(h * 32 + k) * a.Hkv) * D + dcol;
+          a.dV[o] = dv[k];
+          a.dK[o] = dk[k];
+        }
       }
     }
-    __syncthreads();  // P, dS tiles and ds complete
-
-    // dV += (wP)^T dO,  dK += (c_att w da)^T Q  over the 128 rows of this step
-#pragma unroll
-    for (int kr = 0; kr < kRows / 16; ++kr) {
-      uint32_t ap[4], as[4];
-      const int ar = 16 * kr + (lane & 7) + 8 * (lane >> 4), ac = sr0 + 8 * ((lane >> 3) & 1);
-      ldsm_x4_t(ap, pb + swz<kChunk>(ar, ac));
-      ldsm_x4_t(as, db + swz<kChunk>(ar, ac));
-#pragma unroll
-      for (int np = 0; np < NH / 16; ++np) {
-        uint32_t bo[4], bq[4];
-        const int br = 16 * kr + (lane & 7) + 8 * ((lane >> 3) & 1), bcol = dc0 + 16 * np + 8 * (lane >> 4);
-        ldsm_x4_t(bo, ob + swz<D>(br, bcol));
-        ldsm_x4_t(bq, qb + swz<D>(br, bcol));
-        mma_bf16(dv[2 * np], ap, bo[0], bo[1]);
-        mma_bf16(dv[2 * np + 1], ap, bo[2], bo[3]);
-        mma_bf16(dk[2 * np], as, bq[0], bq[1]);
-        mma_bf16(dk[2 * np + 1], as, bq[2], bq[3]);
-      }
-    }
-    __syncthreads();  // buffers of this step free for the prefetch two steps ahead
   }
-
-  // epilogue: dK (attention and mean-pool terms) and dV of every row of the chunk
-#pragma unroll
-  for (int nt = 0; nt < NH / 8; ++nt) {
-    const int col = dc0 + 8 * nt + cc;
-    const long long ra = (row0 + (long long)(sr0 + rr) * a.Hkv) * D + col;
-    const long long rb = (row0 + (long long)(sr0 + rr + 8) * a.Hkv) * D + col;
-    *reinterpret_cast<float2*>(a.dK + ra) = make_float2(dk[nt][0], dk[nt][1]);
-    *reinterpret_cast<float2*>(a.dK + rb) = make_float2(dk[nt][2], dk[nt][3]);
-    *reinterpret_cast<float2*>(a.dV + ra) = make_float2(dv[nt][0], dv[nt][1]);
-    *reinterpret_cast<float2*>(a.dV + rb) = make_float2(dv[nt][2], dv[nt][3]);
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 8) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, kTmemCols);
   }
 }
 
@@ -431,7 +515,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.scale_log2 = Dm.scale_attn * 1.4426950408889634f;
     a.scale_attn = Dm.scale_attn;
     a.scale_sel = Dm.scale_sel;
-    const size_t smem = sizeof(BwdSmem<D>);
+    const size_t smem = sizeof(BwdSmem<D>) + 1024;
     if ((e = cudaFuncSetAttribute(bwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
         cudaSuccess)
       return e;
@@ -454,6 +538,13 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
 }
 
 }  // namespace
+
+unsigned backward_take_status() {
+  unsigned v = 0, zero = 0;
+  if (cudaMemcpyFromSymbol(&v, g_bwd_status, sizeof(v)) != cudaSuccess) return ~0u;
+  cudaMemcpyToSymbol(g_bwd_status, &zero, sizeof(zero));
+  return v;
+}
 
 size_t backward_workspace(const Dims& D) {
   return align256((size_t)D.slots() * D.G * D.d * sizeof(uint16_t)) +

@@ -177,6 +177,7 @@ cudaError_t launch_forward(const Dims& D, const void* q, const void* K, const vo
                            const float* s_sel, const int32_t* offsets, const int32_t* entries, void* O, float* w,
                            void* ws, cudaStream_t st);
 size_t backward_workspace(const Dims& D);
+unsigned backward_take_status();
 cudaError_t launch_backward(const Dims& D, const void* q, const void* K, const void* V, const float* kbar32,
                             const int32_t* idx, const float* w, const void* O, const void* dO,
                             const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,

@@ -105,11 +105,13 @@ __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.
 
 // ------------------------------------------------------------------ MMA
 // Instruction descriptor of kind::f16 with bf16 A and B, fp32 accumulator,
-// both operands K-major, shape M x N.
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+// shape M x N; a_mn / b_mn select the MN-major (instead of K-major) operand.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn = false, bool b_mn = false) {
   return (1u << 4)                      // accumulator format: f32
          | (1u << 7)                    // A format: bf16
          | (1u << 10)                   // B format: bf16
+         | ((a_mn ? 1u : 0u) << 15)     // A major-ness
+         | ((b_mn ? 1u : 0u) << 16)     // B major-ness
          | ((uint32_t)(N >> 3) << 17)   // N / 8
          | ((uint32_t)(M >> 4) << 24);  // M / 16
 }
@@ -123,6 +125,19 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t addr) {
          | ((uint64_t)(1024 >> 4) << 32)     // stride byte offset: next 8-row atom
          | ((uint64_t)1 << 46)               // descriptor version
          | ((uint64_t)2 << 61);              // 128-byte swizzle
+}
+
+// MN-major, 128-byte swizzle: each 128-byte row holds 64 consecutive M (or N)
+// elements of one K index; 8 K-rows form a 1024-byte atom (stride 1024 along
+// K) and the next 64 M/N elements start `mn_block_bytes` further on. A
+// K-major tile [k-row][64 columns] read this way is its own transpose, so
+// the same shared tile serves both operand orientations.
+__device__ __forceinline__ uint64_t sdesc_sw128_mn(uint32_t addr, uint32_t mn_block_bytes) {
+  return (uint64_t)((addr & 0x3FFFFu) >> 4)                     // start address
+         | ((uint64_t)((mn_block_bytes >> 4) & 0x3FFFu) << 16)  // leading byte offset: next 64 M/N elements
+         | ((uint64_t)(1024 >> 4) << 32)                        // stride byte offset: next 8 K-rows
+         | ((uint64_t)1 << 46)                                  // descriptor version
+         | ((uint64_t)2 << 61);                                 // 128-byte swizzle
 }
 
 // D[tmem] (+)= A[smem] * B[smem]^T over one K=16 slice; issued by one thread.

@@ -32,6 +32,8 @@
 //                                       row-major tiles read MN-major)
 // Warps 0-3 (one thread per row) turn S, dP' into P, dSq, dSk and store dq';
 // warps 4-7 gather the Q and dO rows of the next tiles.
+#include <cstring>
+
 #include "tc.cuh"
 
 namespace hsa {
@@ -88,6 +90,8 @@ struct BwdArgs {
   float* dK;
   float* dV;
   int L, Hq, Hkv, G, log2G, topk, Nc;
+  int n_rows;   // B * L * Hq (a row index past it reads zeros)
+  int use_tma;  // G >= 8: each slot's G rows arrive as one swizzled TMA box
   float scale_log2, scale_attn, scale_sel;
 };
 
@@ -102,7 +106,8 @@ struct Cols {
 };
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
+__global__ void __launch_bounds__(kThreads, 1)
+    bwd_chunk_kernel(BwdArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_do) {
   extern __shared__ unsigned char smem_raw[];
   BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
@@ -130,7 +135,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
 
   if (tid == 0) {
     for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(bar(BAR_QD_FULL + i), 128);
+      tc::mbar_init(bar(BAR_QD_FULL + i), a.use_tma ? 1 : 128);
       tc::mbar_init(bar(BAR_QD_EMPTY + i), 1);
       tc::mbar_init(bar(BAR_S_FULL + i), 1);
       tc::mbar_init(bar(BAR_S_EMPTY + i), 128);
@@ -170,7 +175,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
       // publish tile i-1 before waiting for tile i's stage: that stage is freed
       // by the second half of step i-2, which the MMA thread issues only after
       // the first half of step i-1 (which needs tile i-1)
-      if (i >= 1) {
+      if (i >= 1 && !a.use_tma) {
         cp_async_wait<0>();
         tc::fence_proxy_async_smem();
         tc::mbar_arrive(bar(BAR_QD_FULL + ((i - 1) & 1)));
@@ -192,8 +197,25 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
         sm.slot_w[st][lt] = wv;
         sm.slot_delta[st][lt] = dl;
       }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
       const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
+      if (a.use_tma) {
+        // every slot thread issues its own boxes; after the loader barrier one
+        // arrival carries the byte count and publishes the slot tables
+        if (lt < epi) {
+          const int row = sm.slot_row[st][lt];
+          const int y = row >= 0 ? row : a.n_rows;  // past the list: zeros
+#pragma unroll
+          for (int kb = 0; kb < D / 64; ++kb) {
+            const uint32_t o = kb * kRows * 128 + lt * a.G * 128;
+            tc::tma_load_2d(qb + o, &tmap_q, kb * 64, y, bar(BAR_QD_FULL + st));
+            tc::tma_load_2d(ob + o, &tmap_do, kb * 64, y, bar(BAR_QD_FULL + st));
+          }
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (lt == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), 2 * kRows * D * 2);
+        continue;
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
 #pragma unroll 4
       for (int u = lt; u < kRows * D8; u += 128) {
         const int r = u / D8, ch = u % D8;
@@ -210,9 +232,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_chunk_kernel(BwdArgs a) {
       }
       cp_async_commit();
     }
-    cp_async_wait<0>();
-    tc::fence_proxy_async_smem();
-    tc::mbar_arrive(bar(BAR_QD_FULL + ((niter - 1) & 1)));
+    if (!a.use_tma) {
+      cp_async_wait<0>();
+      tc::fence_proxy_async_smem();
+      tc::mbar_arrive(bar(BAR_QD_FULL + ((niter - 1) & 1)));
+    }
   } else if (warp == 8) {
     // ---------------------------------------------------------------- MMA issue (one thread)
     if (lane == 0) {
@@ -519,7 +543,15 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     if ((e = cudaFuncSetAttribute(bwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
         cudaSuccess)
       return e;
-    bwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a);
+    CUtensorMap tq, tdo;
+    memset(&tq, 0, sizeof(tq));
+    memset(&tdo, 0, sizeof(tdo));
+    a.n_rows = Dm.B * Dm.L * Dm.Hq;
+    a.use_tma = Dm.G >= 8 ? 1 : 0;
+    if (a.use_tma && (!tc::make_rows_tmap(&tq, q, (unsigned long long)a.n_rows, D, Dm.G) ||
+                      !tc::make_rows_tmap(&tdo, dO, (unsigned long long)a.n_rows, D, Dm.G)))
+      return cudaErrorNotSupported;
+    bwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq, tdo);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

@@ -11,6 +11,8 @@
 // rescaling. The normalised per-slot result O' (bf16) goes to a workspace
 // and a second kernel forms O_t = sum_j w_j O'_{t,j} with the chunk weights
 // w = softmax_j(s_sel) (the "w/o s.b." variant of §4.1), slots in order j.
+#include <cstring>
+
 #include "tc.cuh"
 
 namespace hsa {
@@ -53,11 +55,13 @@ struct FwdArgs {
   const int32_t* entries;
   uint16_t* Opart;  // [slots, G, D]
   int L, Hq, Hkv, G, log2G, topk, Nc;
+  int n_rows;   // B * L * Hq (query rows; a row index past it reads zeros)
+  int use_tma;  // G >= 8: each slot's G rows arrive as one swizzled TMA box
   float scale_log2;  // c_att * log2(e)
 };
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const __grid_constant__ CUtensorMap tmap_q) {
   extern __shared__ unsigned char smem_raw[];
   FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
@@ -76,7 +80,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
 
   if (tid == 0) {
     for (int i = 0; i < 3; ++i) {
-      tc::mbar_init(bar(BAR_Q_FULL + i), 128);
+      tc::mbar_init(bar(BAR_Q_FULL + i), a.use_tma ? 1 : 128);
       tc::mbar_init(bar(BAR_Q_EMPTY + i), 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -122,18 +126,30 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
     for (int i = 0; i < niter; ++i) {
       const int st = i % kQStages;
       tc::mbar_wait(bar(BAR_Q_EMPTY + st), ((i / kQStages) & 1) ^ 1, abort_flag, &g_fwd_status);
+      int row = -1;
       if (lt < epi) {
         const int e = i * epi + lt;
-        int row = -1;
         if (e < cnt) {
           const int p = a.entries[off + e];
           const int t = (p / slot_div) % a.L;
           row = ((b * a.L + t) * a.Hq) + g * a.G;
         }
-        sm.slot_row[st][lt] = row;
       }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
       const uint32_t base = smem_u32(sm.Q[st]);
+      if (a.use_tma) {
+        // every slot thread issues its own boxes; the single expected arrival
+        // carries the byte count (completions may land before it)
+        if (lt < epi) {
+          const int y = row >= 0 ? row : a.n_rows;  // past the list: zeros
+#pragma unroll
+          for (int kb = 0; kb < D / 64; ++kb)
+            tc::tma_load_2d(base + kb * kRows * 128 + lt * a.G * 128, &tmap_q, kb * 64, y, bar(BAR_Q_FULL + st));
+        }
+        if (lt == 0) tc::mbar_arrive_expect_tx(bar(BAR_Q_FULL + st), kRows * D * 2);
+        continue;
+      }
+      if (lt < epi) sm.slot_row[st][lt] = row;
+      asm volatile("bar.sync 1, 128;" ::: "memory");
 #pragma unroll 4
       for (int u = lt; u < kRows * D8; u += 128) {
         const int r = u / D8, ch = u % D8;
@@ -152,9 +168,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a) {
         tc::mbar_arrive(bar(BAR_Q_FULL + (i - 1) % kQStages));
       }
     }
-    cp_async_wait<0>();
-    tc::fence_proxy_async_smem();
-    tc::mbar_arrive(bar(BAR_Q_FULL + (niter - 1) % kQStages));
+    if (!a.use_tma) {
+      cp_async_wait<0>();
+      tc::fence_proxy_async_smem();
+      tc::mbar_arrive(bar(BAR_Q_FULL + (niter - 1) % kQStages));
+    }
   } else if (warp == 8) {
     // ---------------------------------------------------------------- MMA issue (one thread)
     if (lane == 0) {
@@ -356,7 +374,12 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     const size_t smem = sizeof(FwdSmem<D>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(fwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    fwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a);
+    CUtensorMap tq;
+    memset(&tq, 0, sizeof(tq));
+    a.n_rows = Dm.B * Dm.L * Dm.Hq;
+    a.use_tma = Dm.G >= 8 ? 1 : 0;
+    if (a.use_tma && !tc::make_rows_tmap(&tq, q, (unsigned long long)a.n_rows, D, Dm.G)) return cudaErrorNotSupported;
+    fwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

@@ -30,8 +30,9 @@
 //   dq' = dSq K                        (K read as an MN-major operand)
 //   dV^T += dO^T (wP), dK^T += Q^T dSk (M = d, N = 64, K = 128 rows; the
 //                                       row-major tiles read MN-major)
-// Warps 0-3 (one thread per row) turn S, dP' into P, dSq, dSk and store dq';
-// warps 4-7 gather the Q and dO rows of the next tiles.
+// Warps 0-3 (one thread per row) turn S, dP' into P, dSq, dSk; warps 4-7
+// store dq' (plus the selection term) and finally dK, dV; warp 8 gathers the
+// Q and dO rows of the next tiles; one thread of warp 9 issues the MMAs.
 #include <cstring>
 
 #include "tc.cuh"
@@ -40,7 +41,7 @@ namespace hsa {
 namespace {
 
 constexpr int kRows = 128;     // query rows per step (tensor-core M)
-constexpr int kThreads = 288;  // 4 softmax/epilogue warps, 4 loader warps, 1 MMA warp
+constexpr int kThreads = 320;  // warps 0-3 softmax/gradients, 4-7 epilogue, 8 loader, 9 MMA
 constexpr int kTmemCols = 512;
 
 __device__ unsigned g_bwd_status;
@@ -59,13 +60,15 @@ struct BwdSmem {
   int slot_p[2][kRows];
   float slot_w[2][kRows];
   float slot_delta[2][kRows];
+  float row_ds[2][kRows];         // softmax -> epilogue: ds of the row's slot
+  int row_p[2][kRows];            // softmax -> epilogue: the row's slot id (-1: none)
   uint64_t bar[16];
   uint32_t tmem_base;
   int abort_flag;
 };
 
 enum {
-  BAR_QD_FULL = 0,   // 2: Q and dO tiles landed (128 loader arrivals)
+  BAR_QD_FULL = 0,   // 2: Q and dO tiles landed
   BAR_QD_EMPTY = 2,  // 2: every MMA reading the tiles finished (commit)
   BAR_S_FULL = 4,    // 2: S and dP' ready (commit)
   BAR_S_EMPTY = 6,   // 2: S and dP' read (128 arrivals)
@@ -73,7 +76,8 @@ enum {
   BAR_P_EMPTY = 9,   // P, dSq, dSk consumed (commit)
   BAR_DQ_FULL = 10,  // dq accumulator ready (commit)
   BAR_DQ_EMPTY = 11, // dq read (128 arrivals)
-  BAR_ACC_DONE = 12  // last dK^T / dV^T update finished (commit)
+  BAR_ACC_DONE = 12, // last dK^T / dV^T update finished (commit)
+  BAR_DS_FULL = 13   // 2: row_ds / row_p of a step written (128 arrivals)
 };
 
 struct BwdArgs {
@@ -135,10 +139,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (tid == 0) {
     for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(bar(BAR_QD_FULL + i), a.use_tma ? 1 : 128);
+      tc::mbar_init(bar(BAR_QD_FULL + i), a.use_tma ? 1 : 32);
       tc::mbar_init(bar(BAR_QD_EMPTY + i), 1);
       tc::mbar_init(bar(BAR_S_FULL + i), 1);
       tc::mbar_init(bar(BAR_S_EMPTY + i), 128);
+      tc::mbar_init(bar(BAR_DS_FULL + i), 128);
     }
     tc::mbar_init(bar(BAR_P_FULL), 128);
     tc::mbar_init(bar(BAR_P_EMPTY), 1);
@@ -148,16 +153,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm.abort_flag = 0;
     tc::fence_mbar_init();
   }
-  if (warp == 8) tc::tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
-  if (warp >= 4 && warp < 8) {  // chunk K, V (rows s) and K̄, once per block
-    const int lt = tid - 128;
-    for (int u = lt; u < kChunk * D8; u += 128) {
+  if (warp == 9) tc::tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+  if (warp < 8) {  // chunk K, V (rows s) and K̄, once per block
+    for (int u = tid; u < kChunk * D8; u += 256) {
       const int srow = u / D8, ch = u % D8;
       const long long src = (row0 + (long long)srow * a.Hkv) * D + ch * 8;
       cp_async16(smem_u32(sm.K) + tc::sw128_offset(kChunk, srow, ch * 8), a.K + src);
       cp_async16(smem_u32(sm.V) + tc::sw128_offset(kChunk, srow, ch * 8), a.V + src);
     }
-    for (int u = lt; u < D; u += 128) sm.kbar[u] = a.kbar32[(((long long)b * a.Nc + c) * a.Hkv + g) * D + u];
+    for (int u = tid; u < D; u += 256) sm.kbar[u] = a.kbar32[(((long long)b * a.Nc + c) * a.Hkv + g) * D + u];
     cp_async_commit();
     cp_async_wait<0>();
     tc::fence_proxy_async_smem();
@@ -167,57 +171,84 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::fence_after_sync();
   const uint32_t tmem = sm.tmem_base;
 
-  if (warp >= 4 && warp < 8) {
-    // ---------------------------------------------------------------- loaders
-    const int lt = tid - 128;
+  if (warp == 8) {
+    // ---------------------------------------------------------------- loader warp
+    // The slot data of tile i+1 (entries -> token -> weight, Δ) is fetched
+    // before waiting for tile i's stage, so its dependent global loads are off
+    // the critical path.
+    int n_row = -1, n_p = -1;
+    float n_w = 0.f, n_dl = 0.f;
+    auto fetch = [&](int i) {
+      n_row = -1, n_p = -1, n_w = 0.f, n_dl = 0.f;
+      const int e = i * epi + lane;
+      if (lane < epi && e < cnt) {
+        n_p = a.entries[off + e];
+        const int t = (n_p / slot_div) % a.L;
+        n_row = ((b * a.L + t) * a.Hq) + g * a.G;
+        n_w = a.w[n_p];
+        n_dl = a.delta[((long long)b * a.L + t) * a.Hkv + g];
+      }
+    };
+    fetch(0);
     for (int i = 0; i < niter; ++i) {
       const int st = i & 1;
-      // publish tile i-1 before waiting for tile i's stage: that stage is freed
-      // by the second half of step i-2, which the MMA thread issues only after
-      // the first half of step i-1 (which needs tile i-1)
+      const int c_row = n_row, c_p = n_p;
+      const float c_w = n_w, c_dl = n_dl;
+      if (i + 1 < niter && epi <= 32) fetch(i + 1);
+      // cp.async path: publish tile i-1 before waiting for tile i's stage (that
+      // stage is freed by the second half of step i-2, which the MMA thread
+      // issues only after the first half of step i-1, which needs tile i-1)
       if (i >= 1 && !a.use_tma) {
         cp_async_wait<0>();
         tc::fence_proxy_async_smem();
         tc::mbar_arrive(bar(BAR_QD_FULL + ((i - 1) & 1)));
       }
       tc::mbar_wait(bar(BAR_QD_EMPTY + st), ((i >> 1) & 1) ^ 1, abort_flag, status);
-      if (lt < epi) {
-        const int e = i * epi + lt;
-        int row = -1, p = -1;
-        float wv = 0.f, dl = 0.f;
-        if (e < cnt) {
-          p = a.entries[off + e];
-          const int t = (p / slot_div) % a.L;
-          row = ((b * a.L + t) * a.Hq) + g * a.G;
-          wv = a.w[p];
-          dl = a.delta[((long long)b * a.L + t) * a.Hkv + g];
+      if (epi <= 32) {
+        if (lane < epi) {
+          sm.slot_row[st][lane] = c_row;
+          sm.slot_p[st][lane] = c_p;
+          sm.slot_w[st][lane] = c_w;
+          sm.slot_delta[st][lane] = c_dl;
         }
-        sm.slot_row[st][lt] = row;
-        sm.slot_p[st][lt] = p;
-        sm.slot_w[st][lt] = wv;
-        sm.slot_delta[st][lt] = dl;
+      } else {
+        for (int sl = lane; sl < epi; sl += 32) {
+          const int e = i * epi + sl;
+          int row = -1, p = -1;
+          float wv = 0.f, dl = 0.f;
+          if (e < cnt) {
+            p = a.entries[off + e];
+            const int t = (p / slot_div) % a.L;
+            row = ((b * a.L + t) * a.Hq) + g * a.G;
+            wv = a.w[p];
+            dl = a.delta[((long long)b * a.L + t) * a.Hkv + g];
+          }
+          sm.slot_row[st][sl] = row;
+          sm.slot_p[st][sl] = p;
+          sm.slot_w[st][sl] = wv;
+          sm.slot_delta[st][sl] = dl;
+        }
       }
       const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
       if (a.use_tma) {
-        // every slot thread issues its own boxes; after the loader barrier one
-        // arrival carries the byte count and publishes the slot tables
-        if (lt < epi) {
-          const int row = sm.slot_row[st][lt];
-          const int y = row >= 0 ? row : a.n_rows;  // past the list: zeros
+        // lane l < epi gathers slot l's G rows of q and dO (one box per 64
+        // columns); the single expected arrival carries the byte count and
+        // publishes the slot tables written above
+        if (lane < epi) {
+          const int y = c_row >= 0 ? c_row : a.n_rows;  // past the list: zeros
 #pragma unroll
           for (int kb = 0; kb < D / 64; ++kb) {
-            const uint32_t o = kb * kRows * 128 + lt * a.G * 128;
+            const uint32_t o = kb * kRows * 128 + lane * a.G * 128;
             tc::tma_load_2d(qb + o, &tmap_q, kb * 64, y, bar(BAR_QD_FULL + st));
             tc::tma_load_2d(ob + o, &tmap_do, kb * 64, y, bar(BAR_QD_FULL + st));
           }
         }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (lt == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), 2 * kRows * D * 2);
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), 2 * kRows * D * 2);
         continue;
       }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-#pragma unroll 4
-      for (int u = lt; u < kRows * D8; u += 128) {
+      __syncwarp();
+      for (int u = lane; u < kRows * D8; u += 32) {
         const int r = u / D8, ch = u % D8;
         const int row = sm.slot_row[st][r >> a.log2G];
         const uint32_t o = tc::sw128_offset(kRows, r, ch * 8);
@@ -237,7 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_proxy_async_smem();
       tc::mbar_arrive(bar(BAR_QD_FULL + ((niter - 1) & 1)));
     }
-  } else if (warp == 8) {
+  } else if (warp == 9) {
     // ---------------------------------------------------------------- MMA issue (one thread)
     if (lane == 0) {
       constexpr uint32_t idSP = tc::idesc_bf16(kRows, kChunk);                // S, dP': Q K^T, dO V^T
@@ -251,8 +282,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t pbase = smem_u32(sm.P), dsq = smem_u32(sm.dSq), dsk = smem_u32(sm.dSk);
       auto issue_SdP = [&](int i) {
         const int st = i & 1, sb = i & 1;
-        tc::mbar_wait(bar(BAR_QD_FULL + st), (i >> 1) & 1, abort_flag, status);
-        tc::mbar_wait(bar(BAR_S_EMPTY + sb), ((i >> 1) & 1) ^ 1, abort_flag, status);
         tc::fence_after_sync();
         const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
 #pragma unroll
@@ -268,8 +297,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       auto issue_rest = [&](int i) {
         const int st = i & 1;
-        tc::mbar_wait(bar(BAR_P_FULL), i & 1, abort_flag, status);
-        tc::mbar_wait(bar(BAR_DQ_EMPTY), (i & 1) ^ 1, abort_flag, status);
         tc::fence_after_sync();
         // dq' = dSq K : M = 128 rows, N = D, K = 64 chunk rows
 #pragma unroll
@@ -290,46 +317,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::mma_commit(bar(BAR_QD_EMPTY + st));
         tc::mma_commit(bar(BAR_P_EMPTY));
       };
-      for (int i = 0; i < niter; ++i) {
-        issue_SdP(i);
-        if (i >= 1) issue_rest(i - 1);
+      // Event loop: issue whichever is ready — S/dP' of step nS (tile landed,
+      // accumulator buffer read) or the second half of step nR (P tiles written,
+      // dq accumulator read). Neither barrier can run a phase past the one
+      // polled before the corresponding issue, so parity polling is exact.
+      int nS = 0, nR = 0;
+      unsigned long long t0 = tc::globaltimer();
+      while (nR < niter) {
+        bool progressed = false;
+        if (nS < niter && nS < nR + 2 && tc::mbar_try_wait(bar(BAR_QD_FULL + (nS & 1)), (nS >> 1) & 1) &&
+            tc::mbar_try_wait(bar(BAR_S_EMPTY + (nS & 1)), ((nS >> 1) & 1) ^ 1)) {
+          issue_SdP(nS++);
+          progressed = true;
+        }
+        if (nR < nS && tc::mbar_try_wait(bar(BAR_P_FULL), nR & 1) &&
+            tc::mbar_try_wait(bar(BAR_DQ_EMPTY), (nR & 1) ^ 1)) {
+          issue_rest(nR++);
+          progressed = true;
+        }
+        if (progressed) {
+          t0 = tc::globaltimer();
+        } else if (!tc::within_limit(t0, abort_flag, status)) {
+          break;
+        }
       }
-      issue_rest(niter - 1);
       tc::mma_commit(bar(BAR_ACC_DONE));
     }
     __syncwarp();
-  } else {
+  } else if (warp < 4) {
     // ---------------------------------------------------------------- softmax / gradient rows (thread = row)
     const int r = tid;
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     const float inv_S = 1.f / (float)kChunk;
-    auto dq_epilogue = [&](int j, int pj, float dsj) {
-      tc::mbar_wait(bar(BAR_DQ_FULL), j & 1, abort_flag, status);
-      tc::fence_after_sync();
-      uint16_t* dst = pj >= 0 ? a.dqpart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
-      const float cs = a.scale_sel * dsj;
-#pragma unroll
-      for (int h = 0; h < D / 32; ++h) {
-        float v[32];
-        tc::tmem_ld32(tmem + lane_base + Cols<D>::dq + h * 32, v);
-        tc::tmem_wait_ld();
-        if (dst) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + h * 32);
-#pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4) {
-            float o[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) o[k] = v[8 * q4 + k] + cs * sm.kbar[h * 32 + 8 * q4 + k];
-            d4[q4] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
-                                pack_bf16x2(o[6], o[7]));
-          }
-        }
-      }
-      tc::fence_before_sync();
-      tc::mbar_arrive(bar(BAR_DQ_EMPTY));
-    };
-    int p_prev = -1;
-    float ds_prev = 0.f;
     for (int i = 0; i < niter; ++i) {
       const int sb = i & 1, st = i & 1;
       tc::mbar_wait(bar(BAR_S_FULL + sb), (i >> 1) & 1, abort_flag, status);
@@ -342,34 +361,44 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::tmem_wait_ld();
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_S_EMPTY + sb));
-      // the loaders' slot tables of this tile (released with BAR_QD_FULL, whose
+      // the loader's slot tables of this tile (released with BAR_QD_FULL, whose
       // phase cannot advance before this thread has produced the step's P)
       tc::mbar_wait(bar(BAR_QD_FULL + st), (i >> 1) & 1, abort_flag, status);
       const int slot = r >> a.log2G;
       const float wv = sm.slot_w[st][slot], dl = sm.slot_delta[st][slot];
       const int pv = sm.slot_p[st][slot];
-      float m = -INFINITY;
+      float mx[8], zz[8], dd[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) mx[u] = x[u];
+#pragma unroll
+      for (int k = 8; k < 64; ++k) mx[k & 7] = fmaxf(mx[k & 7], x[k]);
+      const float m = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      const float ms = m * a.scale_log2;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) zz[u] = 0.f;
 #pragma unroll
       for (int k = 0; k < 64; ++k) {
-        x[k] *= a.scale_log2;
-        m = fmaxf(m, x[k]);
+        x[k] = exp2f(fmaf(x[k], a.scale_log2, -ms));
+        zz[k & 7] += x[k];
       }
-      float z = 0.f;
+      const float inv = 1.f / (((zz[0] + zz[1]) + (zz[2] + zz[3])) + ((zz[4] + zz[5]) + (zz[6] + zz[7])));
 #pragma unroll
-      for (int k = 0; k < 64; ++k) {
-        x[k] = exp2f(x[k] - m);
-        z += x[k];
-      }
-      const float inv = 1.f / z;
-      float Drow = 0.f;
+      for (int u = 0; u < 8; ++u) dd[u] = 0.f;
 #pragma unroll
       for (int k = 0; k < 64; ++k) {
         x[k] *= inv;
-        Drow += x[k] * y[k];
+        dd[k & 7] = fmaf(x[k], y[k], dd[k & 7]);
       }
+      const float Drow = ((dd[0] + dd[1]) + (dd[2] + dd[3])) + ((dd[4] + dd[5]) + (dd[6] + dd[7]));
       float dw = Drow;  // sum over the G rows of the slot (consecutive lanes)
       for (int o = 1; o < a.G; o <<= 1) dw += __shfl_xor_sync(0xFFFFFFFFu, dw, o);
       const float dsv = wv * (dw - dl);
+      // hand ds and the slot id to the epilogue warps (double-buffered: the
+      // buffer of step i is rewritten at step i+2, after the epilogue of step i
+      // has released the dq accumulator that step i+1's dq product waits for)
+      sm.row_ds[sb][r] = dsv;
+      sm.row_p[sb][r] = pv;
+      tc::mbar_arrive(bar(BAR_DS_FULL + sb));
       const float ca = a.scale_attn * wv, pool = a.scale_sel * dsv * inv_S;
       tc::mbar_wait(bar(BAR_P_EMPTY), (i & 1) ^ 1, abort_flag, status);
       const uint32_t prow = smem_u32(sm.P), qrow = smem_u32(sm.dSq), krow = smem_u32(sm.dSk);
@@ -394,15 +423,42 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc::fence_proxy_async_smem();
       tc::mbar_arrive(bar(BAR_P_FULL));
-      if (i >= 1) dq_epilogue(i - 1, p_prev, ds_prev);
-      p_prev = pv;
-      ds_prev = dsv;
     }
-    dq_epilogue(niter - 1, p_prev, ds_prev);
+  } else {
+    // ---------------------------------------------------------------- epilogue (thread = row, then head dim)
+    const int r = tid - 128;
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    for (int j = 0; j < niter; ++j) {
+      const int sb = j & 1;
+      tc::mbar_wait(bar(BAR_DS_FULL + sb), (j >> 1) & 1, abort_flag, status);
+      const float dsj = sm.row_ds[sb][r];
+      const int pj = sm.row_p[sb][r];
+      tc::mbar_wait(bar(BAR_DQ_FULL), j & 1, abort_flag, status);
+      tc::fence_after_sync();
+      uint16_t* dst = pj >= 0 ? a.dqpart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
+      const float cs = a.scale_sel * dsj;
+      float v[D];
+#pragma unroll
+      for (int h = 0; h < D / 32; ++h) tc::tmem_ld32(tmem + lane_base + Cols<D>::dq + h * 32, *reinterpret_cast<float(*)[32]>(&v[h * 32]));
+      tc::tmem_wait_ld();
+      tc::fence_before_sync();
+      tc::mbar_arrive(bar(BAR_DQ_EMPTY));
+      if (dst) {
+        uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+        for (int q8 = 0; q8 < D / 8; ++q8) {
+          float o[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) o[k] = v[8 * q8 + k] + cs * sm.kbar[8 * q8 + k];
+          d4[q8] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
+                              pack_bf16x2(o[6], o[7]));
+        }
+      }
+    }
     // dK, dV of the chunk: TMEM lane = head dim, column = chunk row
     tc::mbar_wait(bar(BAR_ACC_DONE), 0, abort_flag, status);
     tc::fence_after_sync();
-    if (warp * 32 < D) {
+    if ((warp & 3) * 32 < D) {
       const int dcol = r;
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
@@ -421,7 +477,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc::fence_before_sync();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == 9) {
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, kTmemCols);
   }

@@ -20,7 +20,7 @@ namespace {
 
 constexpr int kRows = 128;     // query rows per step (tensor-core M)
 constexpr int kQStages = 3;    // gathered query tiles in flight
-constexpr int kThreads = 288;  // 4 softmax/epilogue warps, 4 loader warps, 1 MMA warp
+constexpr int kThreads = 320;  // warps 0-3 softmax, 4-7 epilogue, 8 loader, 9 MMA
 constexpr int kTmemCols = 512;
 
 __device__ unsigned g_fwd_status;
@@ -31,20 +31,20 @@ struct FwdSmem {
   uint16_t K[kChunk * D];           // chunk keys [s][d]
   uint16_t Vt[D * kChunk];          // chunk values transposed [d][s]
   uint16_t P[2][kRows * kChunk];    // normalised probabilities (bf16)
-  int slot_row[kQStages][kRows];    // first q row of each slot of a tile (-1: past the list)
+  int slot_row[kQStages][kRows];    // cp.async path: first q row of each slot (-1: past the list)
   uint64_t bar[16];
   uint32_t tmem_base;
   int abort_flag;
 };
 
 enum {
-  BAR_Q_FULL = 0,   // 3: tile landed (128 loader arrivals)
+  BAR_Q_FULL = 0,   // 3: tile landed
   BAR_Q_EMPTY = 3,  // 3: S MMA of the tile finished (commit)
   BAR_S_FULL = 6,   // 2: S accumulator ready (commit)
   BAR_S_EMPTY = 8,  // 2: S read by the softmax warps (128 arrivals)
   BAR_P_FULL = 10,  // 2: P tile written (128 arrivals)
   BAR_O_FULL = 12,  // 2: O accumulator ready (commit)
-  BAR_O_EMPTY = 14  // 2: O read by the epilogue (128 arrivals)
+  BAR_O_EMPTY = 14  // 2: O read by the epilogue warps (128 arrivals)
 };
 
 struct FwdArgs {
@@ -77,10 +77,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
   const int slot_div = a.Hkv * a.topk;
   auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
   volatile int* abort_flag = &sm.abort_flag;
+  unsigned* status = &g_fwd_status;
 
   if (tid == 0) {
     for (int i = 0; i < 3; ++i) {
-      tc::mbar_init(bar(BAR_Q_FULL + i), a.use_tma ? 1 : 128);
+      tc::mbar_init(bar(BAR_Q_FULL + i), a.use_tma ? 1 : 32);
       tc::mbar_init(bar(BAR_Q_EMPTY + i), 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -93,11 +94,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
     sm.abort_flag = 0;
     tc::fence_mbar_init();
   }
-  if (warp == 8) tc::tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
-  if (warp >= 4 && warp < 8) {  // chunk K (K-major rows s) and V^T (rows d), once per block
-    const int lt = tid - 128;
+  if (warp == 9) tc::tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+  if (warp < 8) {  // chunk K (K-major rows s) and V^T (rows d), once per block
     const long long row0 = ((long long)b * a.L + (long long)c * kChunk) * a.Hkv + g;
-    for (int u = lt; u < kChunk * D8; u += 128) {
+    for (int u = tid; u < kChunk * D8; u += 256) {
       const int srow = u / D8, ch = u % D8;
       const long long src = (row0 + (long long)srow * a.Hkv) * D + ch * 8;
       cp_async16(smem_u32(sm.K) + tc::sw128_offset(kChunk, srow, ch * 8), a.K + src);
@@ -118,40 +118,50 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
   tc::fence_after_sync();
   const uint32_t tmem = sm.tmem_base;
 
-  if (warp >= 4 && warp < 8) {
-    // ---------------------------------------------------------------- loaders
-    // Per tile: one thread per slot resolves the slot's first query row, then
-    // the 128 loader threads copy 128 rows x D columns with table lookups.
-    const int lt = tid - 128;
+  if (warp == 8) {
+    // ---------------------------------------------------------------- loader warp
+    // TMA path: the next tile's slot rows are resolved before waiting for the
+    // current tile's stage, so the dependent global loads are off the critical path.
+    auto slot_y = [&](int i) {
+      const int e = i * epi + lane;
+      int y = a.n_rows;  // past the list: the box reads zeros
+      if (lane < epi && e < cnt) {
+        const int p = a.entries[off + e];
+        const int t = (p / slot_div) % a.L;
+        y = ((b * a.L + t) * a.Hq) + g * a.G;
+      }
+      return y;
+    };
+    int y_next = a.use_tma ? slot_y(0) : 0;
     for (int i = 0; i < niter; ++i) {
       const int st = i % kQStages;
-      tc::mbar_wait(bar(BAR_Q_EMPTY + st), ((i / kQStages) & 1) ^ 1, abort_flag, &g_fwd_status);
-      int row = -1;
-      if (lt < epi) {
-        const int e = i * epi + lt;
+      const int y = y_next;
+      if (a.use_tma && i + 1 < niter) y_next = slot_y(i + 1);
+      tc::mbar_wait(bar(BAR_Q_EMPTY + st), ((i / kQStages) & 1) ^ 1, abort_flag, status);
+      const uint32_t base = smem_u32(sm.Q[st]);
+      if (a.use_tma) {
+        // lane l < epi gathers slot l's G rows as one box per 64 columns; the
+        // single expected arrival carries the byte count
+        if (lane < epi) {
+#pragma unroll
+          for (int kb = 0; kb < D / 64; ++kb)
+            tc::tma_load_2d(base + kb * kRows * 128 + lane * a.G * 128, &tmap_q, kb * 64, y, bar(BAR_Q_FULL + st));
+        }
+        if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_Q_FULL + st), kRows * D * 2);
+        continue;
+      }
+      for (int sl = lane; sl < epi; sl += 32) {
+        const int e = i * epi + sl;
+        int row = -1;
         if (e < cnt) {
           const int p = a.entries[off + e];
           const int t = (p / slot_div) % a.L;
           row = ((b * a.L + t) * a.Hq) + g * a.G;
         }
+        sm.slot_row[st][sl] = row;
       }
-      const uint32_t base = smem_u32(sm.Q[st]);
-      if (a.use_tma) {
-        // every slot thread issues its own boxes; the single expected arrival
-        // carries the byte count (completions may land before it)
-        if (lt < epi) {
-          const int y = row >= 0 ? row : a.n_rows;  // past the list: zeros
-#pragma unroll
-          for (int kb = 0; kb < D / 64; ++kb)
-            tc::tma_load_2d(base + kb * kRows * 128 + lt * a.G * 128, &tmap_q, kb * 64, y, bar(BAR_Q_FULL + st));
-        }
-        if (lt == 0) tc::mbar_arrive_expect_tx(bar(BAR_Q_FULL + st), kRows * D * 2);
-        continue;
-      }
-      if (lt < epi) sm.slot_row[st][lt] = row;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-#pragma unroll 4
-      for (int u = lt; u < kRows * D8; u += 128) {
+      __syncwarp();
+      for (int u = lane; u < kRows * D8; u += 32) {
         const int r = u / D8, ch = u % D8;
         const int row = sm.slot_row[st][r >> a.log2G];
         const uint32_t dst = base + tc::sw128_offset(kRows, r, ch * 8);
@@ -173,7 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
       tc::fence_proxy_async_smem();
       tc::mbar_arrive(bar(BAR_Q_FULL + (niter - 1) % kQStages));
     }
-  } else if (warp == 8) {
+  } else if (warp == 9) {
     // ---------------------------------------------------------------- MMA issue (one thread)
     if (lane == 0) {
       constexpr uint32_t idS = tc::idesc_bf16(kRows, kChunk);
@@ -181,8 +191,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
       const uint32_t kbase = smem_u32(sm.K), vbase = smem_u32(sm.Vt);
       auto issue_S = [&](int i) {
         const int st = i % kQStages, sb = i & 1;
-        tc::mbar_wait(bar(BAR_Q_FULL + st), (i / kQStages) & 1, abort_flag, &g_fwd_status);
-        tc::mbar_wait(bar(BAR_S_EMPTY + sb), ((i >> 1) & 1) ^ 1, abort_flag, &g_fwd_status);
         tc::fence_after_sync();
         const uint32_t qbase = smem_u32(sm.Q[st]);
 #pragma unroll
@@ -196,8 +204,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
       };
       auto issue_O = [&](int i) {
         const int pb = i & 1;
-        tc::mbar_wait(bar(BAR_P_FULL + pb), (i >> 1) & 1, abort_flag, &g_fwd_status);
-        tc::mbar_wait(bar(BAR_O_EMPTY + pb), ((i >> 1) & 1) ^ 1, abort_flag, &g_fwd_status);
         tc::fence_after_sync();
         const uint32_t pbase = smem_u32(sm.P[pb]);
 #pragma unroll
@@ -206,47 +212,38 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
                           tc::sdesc_sw128(vbase + kk * 32), idO, kk > 0);
         tc::mma_commit(bar(BAR_O_FULL + pb));
       };
-      for (int i = 0; i < niter; ++i) {
-        issue_S(i);
-        if (i >= 1) issue_O(i - 1);
-      }
-      issue_O(niter - 1);
-    }
-    __syncwarp();
-  } else {
-    // ---------------------------------------------------------------- softmax + epilogue (thread = row)
-    const int r = tid;
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-    auto epilogue = [&](int j, int pj) {
-      const int ob = j & 1;
-      tc::mbar_wait(bar(BAR_O_FULL + ob), (j >> 1) & 1, abort_flag, &g_fwd_status);
-      tc::fence_after_sync();
-      const bool valid = pj >= 0;
-      uint16_t* dst = nullptr;
-      if (valid) dst = a.Opart + ((long long)pj * a.G + (r & (a.G - 1))) * D;
-#pragma unroll
-      for (int h = 0; h < D / 32; ++h) {
-        float o[32];
-        tc::tmem_ld32(tmem + lane_base + 2 * kChunk + ob * D + h * 32, o);
-        tc::tmem_wait_ld();
-        if (valid) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + h * 32);
-#pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4)
-            d4[q4] = make_uint4(pack_bf16x2(o[8 * q4], o[8 * q4 + 1]), pack_bf16x2(o[8 * q4 + 2], o[8 * q4 + 3]),
-                                pack_bf16x2(o[8 * q4 + 4], o[8 * q4 + 5]),
-                                pack_bf16x2(o[8 * q4 + 6], o[8 * q4 + 7]));
+      // Event loop: issue S of step nS (tile landed, S buffer read) or O of step
+      // nO (P written, O buffer read), whichever is ready. Neither barrier can
+      // run a phase past the polled one before the corresponding issue.
+      int nS = 0, nO = 0;
+      unsigned long long t0 = tc::globaltimer();
+      while (nO < niter) {
+        bool progressed = false;
+        if (nS < niter && nS < nO + 2 && tc::mbar_try_wait(bar(BAR_Q_FULL + nS % kQStages), (nS / kQStages) & 1) &&
+            tc::mbar_try_wait(bar(BAR_S_EMPTY + (nS & 1)), ((nS >> 1) & 1) ^ 1)) {
+          issue_S(nS++);
+          progressed = true;
+        }
+        if (nO < nS && tc::mbar_try_wait(bar(BAR_P_FULL + (nO & 1)), (nO >> 1) & 1) &&
+            tc::mbar_try_wait(bar(BAR_O_EMPTY + (nO & 1)), ((nO >> 1) & 1) ^ 1)) {
+          issue_O(nO++);
+          progressed = true;
+        }
+        if (progressed) {
+          t0 = tc::globaltimer();
+        } else if (!tc::within_limit(t0, abort_flag, status)) {
+          break;
         }
       }
-      tc::fence_before_sync();
-      tc::mbar_arrive(bar(BAR_O_EMPTY + ob));
-    };
-    int p_prev = -1;
+    }
+    __syncwarp();
+  } else if (warp < 4) {
+    // ---------------------------------------------------------------- softmax (thread = row)
+    const int r = tid;
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     for (int i = 0; i < niter; ++i) {
       const int sb = i & 1;
-      const int e_i = i * epi + (r >> a.log2G);
-      const int p_i = e_i < cnt ? a.entries[off + e_i] : -1;  // used by this step's epilogue
-      tc::mbar_wait(bar(BAR_S_FULL + sb), (i >> 1) & 1, abort_flag, &g_fwd_status);
+      tc::mbar_wait(bar(BAR_S_FULL + sb), (i >> 1) & 1, abort_flag, status);
       tc::fence_after_sync();
       float x[64];
       tc::tmem_ld32(tmem + lane_base + sb * kChunk, *reinterpret_cast<float(*)[32]>(&x[0]));
@@ -254,19 +251,21 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
       tc::tmem_wait_ld();
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_S_EMPTY + sb));
-      float m = -INFINITY;
+      float mx[8], zz[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) mx[u] = x[u];
+#pragma unroll
+      for (int k = 8; k < 64; ++k) mx[k & 7] = fmaxf(mx[k & 7], x[k]);
+      const float m = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      const float ms = m * a.scale_log2;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) zz[u] = 0.f;
 #pragma unroll
       for (int k = 0; k < 64; ++k) {
-        x[k] *= a.scale_log2;
-        m = fmaxf(m, x[k]);
+        x[k] = exp2f(fmaf(x[k], a.scale_log2, -ms));
+        zz[k & 7] += x[k];
       }
-      float z = 0.f;
-#pragma unroll
-      for (int k = 0; k < 64; ++k) {
-        x[k] = exp2f(x[k] - m);
-        z += x[k];
-      }
-      const float inv = 1.f / z;
+      const float inv = 1.f / (((zz[0] + zz[1]) + (zz[2] + zz[3])) + ((zz[4] + zz[5]) + (zz[6] + zz[7])));
       const uint32_t prow = smem_u32(sm.P[sb]);
 #pragma unroll
       for (int c16 = 0; c16 < 8; ++c16) {
@@ -279,14 +278,41 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
       }
       tc::fence_proxy_async_smem();
       tc::mbar_arrive(bar(BAR_P_FULL + sb));
-      if (i >= 1) epilogue(i - 1, p_prev);
-      p_prev = p_i;
     }
-    epilogue(niter - 1, p_prev);
+  } else {
+    // ---------------------------------------------------------------- epilogue (thread = row)
+    const int r = tid - 128;
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    int p_next = r >> a.log2G < cnt ? a.entries[off + (r >> a.log2G)] : -1;
+    for (int j = 0; j < niter; ++j) {
+      const int pj = p_next;
+      const int en = (j + 1) * epi + (r >> a.log2G);
+      p_next = en < cnt ? a.entries[off + en] : -1;  // prefetch the next step's slot
+      const int ob = j & 1;
+      tc::mbar_wait(bar(BAR_O_FULL + ob), (j >> 1) & 1, abort_flag, status);
+      tc::fence_after_sync();
+      uint16_t* dst = pj >= 0 ? a.Opart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
+#pragma unroll
+      for (int h = 0; h < D / 32; ++h) {
+        float o[32];
+        tc::tmem_ld32(tmem + lane_base + 2 * kChunk + ob * D + h * 32, o);
+        tc::tmem_wait_ld();
+        if (dst) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + h * 32);
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4)
+            d4[q4] = make_uint4(pack_bf16x2(o[8 * q4], o[8 * q4 + 1]), pack_bf16x2(o[8 * q4 + 2], o[8 * q4 + 3]),
+                                pack_bf16x2(o[8 * q4 + 4], o[8 * q4 + 5]),
+                                pack_bf16x2(o[8 * q4 + 6], o[8 * q4 + 7]));
+        }
+      }
+      tc::fence_before_sync();
+      tc::mbar_arrive(bar(BAR_O_EMPTY + ob));
+    }
   }
   tc::fence_before_sync();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == 9) {
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, kTmemCols);
   }

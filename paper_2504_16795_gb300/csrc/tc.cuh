@@ -81,6 +81,18 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// Bounded polling helper for event loops: returns false (and sets the abort
+// flag) once `t0` is older than the wait limit.
+__device__ __forceinline__ bool within_limit(unsigned long long t0, volatile int* abort_flag, unsigned* status) {
+  if (*abort_flag) return false;
+  if (globaltimer() - t0 > kWaitLimitNs) {
+    *abort_flag = 1;
+    if (status) atomicOr(status, kStatusTimeout);
+    return false;
+  }
+  return true;
+}
+
 // ------------------------------------------------------------------ proxies
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

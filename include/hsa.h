@@ -23,7 +23,9 @@
  *   Memory   Every pointer is device memory owned by the caller, 16-byte
  *            aligned. The library never allocates or frees memory and keeps
  *            no state between calls; scratch comes from the caller's
- *            workspace (size from hsa_workspace_size).
+ *            workspace (size from hsa_workspace_size). The one exception is
+ *            hsa_decode_noalloc, whose scratch is a fixed array inside the
+ *            library.
  *   Streams  All work is enqueued on `stream`; nothing synchronises the host.
  *   Errors   Arguments are validated before any launch: a bad argument returns
  *            HSA_ERR_INVALID_ARG, a shape outside the supported set
@@ -190,6 +192,33 @@ hsa_status_t hsa_backward(const hsa_shape_t* shape, const void* q, const void* K
 hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const void* K_mem, const void* V_mem,
                         const float* kbar32, void* O, int32_t* idx, float* s_sel, float* w, void* ws,
                         size_t ws_bytes, cudaStream_t stream);
+
+/* Size of the scratch array behind hsa_decode_noalloc (one per device): 8 MiB. */
+#define HSA_DECODE_NOALLOC_SCRATCH_BYTES (8u << 20)
+
+/*
+ * hsa_decode without a workspace argument: the paper has no counterpart; this
+ * is a calling convention for callers that cannot allocate device memory when
+ * they decode (a host that embeds the decoder under a device-memory budget
+ * fixed at start-up, or a serving loop that must stay out of the allocator,
+ * whose cudaMalloc/cudaFree may synchronise the device, between tokens).
+ *   Arguments, results and numerics as in hsa_decode (same kernels). The
+ *   library allocates nothing: its scratch is a fixed device array of
+ *   HSA_DECODE_NOALLOC_SCRATCH_BYTES compiled into the library, one per device.
+ *   Limit: a shape whose hsa_decode_workspace_size exceeds that size returns
+ *   HSA_ERR_WORKSPACE before any launch (the decode of 64 queries, 8 heads in
+ *   one group, d = 128, k = 8 needs about 3.4 MB at any memory length).
+ *   First call on each device: looks up the array's address on the current
+ *   device (cudaGetSymbolAddress) and caches it; make that first call before
+ *   any stream capture on that device.
+ *   Nothing in the array needs to start at zero.
+ *   Races: every call on a device uses the same array, so calls that can
+ *   overlap on one device (different streams, different host threads) corrupt
+ *   each other's results; the caller serialises them.
+ */
+hsa_status_t hsa_decode_noalloc(const hsa_decode_shape_t* shape, const void* q, const void* K_mem,
+                                const void* V_mem, const float* kbar32, void* O, int32_t* idx, float* s_sel,
+                                float* w, cudaStream_t stream);
 
 #ifdef __cplusplus
 }

@@ -18,6 +18,7 @@ from .binding import (  # noqa: F401
     build_index,
     chunk_pool,
     decode,
+    decode_noalloc,
     decode_workspace_size,
     device_check,
     forward,

@@ -114,8 +114,9 @@ def load():
     L.hsa_forward.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     L.hsa_backward.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     L.hsa_decode.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    L.hsa_decode_noalloc.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
     for f in (L.hsa_chunk_pool, L.hsa_select_topk, L.hsa_build_index, L.hsa_forward, L.hsa_backward,
-              L.hsa_decode):
+              L.hsa_decode, L.hsa_decode_noalloc):
         f.restype = i
     _lib = L
     return L
@@ -264,6 +265,22 @@ def decode(shape: DecodeShape, q, K_mem, V_mem, kbar32, O=None, idx=None, s_sel=
     s = shape.c()
     _check(load().hsa_decode(ctypes.byref(s), _ptr(q), _ptr(K_mem), _ptr(V_mem), _ptr(kbar32), _ptr(O), _ptr(idx),
                              _ptr(s_sel), _ptr(w), _ptr(wsp), nb, _stream(dev)), "hsa_decode")
+    return O, idx, s_sel, w
+
+
+def decode_noalloc(shape: DecodeShape, q, K_mem, V_mem, kbar32, O, idx, s_sel, w):
+    """hsa_decode_noalloc: decode into caller-provided outputs, scratch owned by the library.
+
+    Calls on one device share the library's scratch; callers serialise them."""
+    _need(q, "q", torch.bfloat16, (shape.Bq, shape.Hq, shape.d))
+    _need(O, "O", torch.bfloat16, (shape.Bq, shape.Hq, shape.d))
+    out = (shape.Bq, shape.Hkv, shape.topk)
+    _need(idx, "idx", torch.int32, out)
+    _need(s_sel, "s_sel", torch.float32, out)
+    _need(w, "w", torch.float32, out)
+    s = shape.c()
+    _check(load().hsa_decode_noalloc(ctypes.byref(s), _ptr(q), _ptr(K_mem), _ptr(V_mem), _ptr(kbar32), _ptr(O),
+                                     _ptr(idx), _ptr(s_sel), _ptr(w), _stream(q.device)), "hsa_decode_noalloc")
     return O, idx, s_sel, w
 
 

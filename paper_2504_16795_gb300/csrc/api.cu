@@ -253,3 +253,7 @@ hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const vo
 }
 
 }  // extern "C"
+
+hsa_status_t hsa::resolve_decode_shape(const hsa_decode_shape_t* s, hsa::DecodeDims* out) {
+  return resolve_decode(s, out);
+}

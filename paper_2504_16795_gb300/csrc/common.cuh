@@ -190,4 +190,6 @@ struct DecodeDims {
 size_t decode_workspace(const DecodeDims& D);
 cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
                           void* O, int32_t* idx, float* s_sel, float* w, void* ws, cudaStream_t st);
+// The decode shape check of hsa_decode, shared with the entry point that owns its scratch.
+hsa_status_t resolve_decode_shape(const hsa_decode_shape_t* s, DecodeDims* out);
 }  // namespace hsa

@@ -116,6 +116,23 @@ def test_decode_validation(lib):
     assert lib.hsa_decode(ctypes.byref(c), *[vp(FAKE)] * 9, 16, None) == WORKSPACE
 
 
+def test_decode_noalloc_rejects_shapes_beyond_its_scratch(lib):
+    vp = ctypes.c_void_p
+    limit = 8 << 20
+    big = hsa.DecodeShape(Bq=1024, Hq=8, Hkv=1, d=128, n_chunks=1 << 20)
+    assert hsa.decode_workspace_size(big) > limit
+    c = big.c()
+    assert lib.hsa_decode_noalloc(ctypes.byref(c), *[vp(FAKE)] * 8, None) == WORKSPACE
+    # 64 queries over a 2^26-token memory fit
+    assert hsa.decode_workspace_size(hsa.DecodeShape(Bq=64, Hq=8, Hkv=1, d=128, n_chunks=1 << 20)) <= limit
+    c = hsa.DecodeShape(Bq=0, Hq=8, Hkv=1, d=128, n_chunks=10).c()
+    assert lib.hsa_decode_noalloc(ctypes.byref(c), *[vp(0)] * 8, None) == OK
+    c = hsa.DecodeShape(Bq=4, Hq=8, Hkv=1, d=80, n_chunks=10).c()
+    assert lib.hsa_decode_noalloc(ctypes.byref(c), *[vp(FAKE)] * 8, None) == UNSUPPORTED
+    c = hsa.DecodeShape(Bq=4, Hq=8, Hkv=1, d=128, n_chunks=10).c()
+    assert lib.hsa_decode_noalloc(ctypes.byref(c), *[vp(FAKE + 8)] * 8, None) == INVALID
+
+
 def test_workspace_sizes_scale_with_the_problem(lib):
     s = shape(B=2, L=32768, Hq=32, Hkv=4)
     slots = 2 * 32768 * 4 * 8

@@ -289,6 +289,7 @@ class Workspaces:
 
     def __init__(self, shape: Shape, device):
         self.shape = shape
+        self.select = _workspace(workspace_size(HSA_OP_SELECT, shape), device, None)
         self.index = _workspace(workspace_size(HSA_OP_INDEX, shape), device, None)
         self.forward = _workspace(workspace_size(HSA_OP_FORWARD, shape), device, None)
         self.backward = _workspace(workspace_size(HSA_OP_BACKWARD, shape), device, None)
@@ -298,7 +299,7 @@ def hsa_forward_path(shape: Shape, q, K, V, wss: Optional[Workspaces] = None):
     """pool -> select -> inverse index -> attention + merge. Returns a dict of every intermediate."""
     wss = wss or Workspaces(shape, q.device)
     kbar32, kbar16 = chunk_pool(shape, K)
-    idx, s_sel = select_topk(shape, q, kbar32)
+    idx, s_sel = select_topk(shape, q, kbar32, ws=wss.select)
     offsets, entries = build_index(shape, idx, ws=wss.index)
     O, w = forward(shape, q, K, V, idx, s_sel, offsets, entries, ws=wss.forward)
     return dict(kbar32=kbar32, kbar16=kbar16, idx=idx, s_sel=s_sel, offsets=offsets, entries=entries, O=O, w=w)

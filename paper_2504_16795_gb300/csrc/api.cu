@@ -85,9 +85,10 @@ unsigned long long hsa_kernel_launches(void) { return hsa::g_launches.load(std::
 
 hsa_status_t hsa_device_check(void) {
   if (cudaDeviceSynchronize() != cudaSuccess) return HSA_ERR_CUDA;
-  const unsigned s1 = hsa::forward_take_status(), s2 = hsa::backward_take_status();
-  if (s1 == ~0u || s2 == ~0u) return HSA_ERR_CUDA;
-  return (s1 | s2) ? HSA_ERR_TIMEOUT : HSA_OK;
+  const unsigned s1 = hsa::forward_take_status(), s2 = hsa::backward_take_status(),
+                 s3 = hsa::select_take_status();
+  if (s1 == ~0u || s2 == ~0u || s3 == ~0u) return HSA_ERR_CUDA;
+  return (s1 | s2 | s3) ? HSA_ERR_TIMEOUT : HSA_OK;
 }
 
 size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {
@@ -95,7 +96,7 @@ size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {
   if (resolve(shape, &D) != HSA_OK) return 0;
   if (empty(D)) return 0;
   switch (op) {
-    case HSA_OP_SELECT: return 0;
+    case HSA_OP_SELECT: return hsa::select_tc_workspace(D);
     case HSA_OP_INDEX: return hsa::index_workspace(D);
     case HSA_OP_FORWARD: return hsa::forward_workspace(D);
     case HSA_OP_BACKWARD: return hsa::backward_workspace(D);
@@ -125,8 +126,11 @@ hsa_status_t hsa_select_topk(const hsa_shape_t* shape, const void* q, const floa
   HSA_REQUIRE_PTR(idx);
   HSA_REQUIRE_PTR(s_sel);
   if (D.Nc > 0) HSA_REQUIRE_PTR(kbar32);
-  (void)ws;
-  (void)ws_bytes;
+  if (hsa::select_tc_applies(D)) {
+    const size_t need = hsa::select_tc_workspace(D);
+    if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+    return cuda_status(hsa::launch_select_tc(D, q, kbar32, idx, s_sel, ws, stream));
+  }
   return cuda_status(hsa::launch_select(D, q, kbar32, idx, s_sel, stream));
 }
 

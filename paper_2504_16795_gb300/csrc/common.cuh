@@ -166,6 +166,12 @@ inline int grid_cap(long long blocks, long long cap = 152LL * 64) {
 // Launchers implemented in the kernel translation units; all return cudaError_t.
 namespace hsa {
 cudaError_t launch_pool(const Dims& D, const void* K, float* kbar32, void* kbar16, cudaStream_t st);
+// Tensor-core selection with exact rescoring (topk <= 16); needs select_tc_workspace bytes.
+bool select_tc_applies(const Dims& D);
+size_t select_tc_workspace(const Dims& D);
+unsigned select_take_status();
+cudaError_t launch_select_tc(const Dims& D, const void* q, const float* kbar32, int32_t* idx, float* s_sel, void* ws,
+                             cudaStream_t st);
 cudaError_t launch_select(const Dims& D, const void* q, const float* kbar32, int32_t* idx, float* s_sel,
                           cudaStream_t st);
 size_t index_workspace(const Dims& D);

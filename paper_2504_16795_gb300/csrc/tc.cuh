@@ -81,6 +81,14 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// Plain (untiled) bulk copy global -> shared, completion counted in bytes on
+// `bar`. Both addresses 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
 // Bounded polling helper for event loops: returns false (and sets the abort
 // flag) once `t0` is older than the wait limit.
 __device__ __forceinline__ bool within_limit(unsigned long long t0, volatile int* abort_flag, unsigned* status) {
@@ -197,7 +205,7 @@ __device__ __forceinline__ uint32_t sw128_offset(int rows, int row, int col) {
 // ------------------------------------------------------------------ host: tensor maps
 // A bf16 matrix of `rows` x `cols` (row pitch cols * 2 bytes) read in boxes of
 // 64 columns x box_rows rows with the 128-byte swizzle of the operand layout.
-inline bool make_rows_tmap(CUtensorMap* map, const void* base, unsigned long long rows, int cols, int box_rows) {
+inline PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
   static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
   if (encode == nullptr) {
     void* fn = nullptr;
@@ -205,14 +213,35 @@ inline bool make_rows_tmap(CUtensorMap* map, const void* base, unsigned long lon
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
             cudaSuccess ||
         q != cudaDriverEntryPointSuccess || fn == nullptr)
-      return false;
+      return nullptr;
     encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
   }
+  return encode;
+}
+
+inline bool make_rows_tmap(CUtensorMap* map, const void* base, unsigned long long rows, int cols, int box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 encode = tmap_encoder();
+  if (encode == nullptr) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
   const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
   const cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
   const cuuint32_t estr[2] = {1u, 1u};
   return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The same for an fp32 matrix: boxes of 32 columns (128 bytes) x box_rows rows.
+// In shared memory, element (r, c) of a box sits in 16-byte chunk
+// ((c / 4) ^ (r % 8)) of the box's 128-byte row r.
+inline bool make_rows_tmap_f32(CUtensorMap* map, const void* base, unsigned long long rows, int cols, int box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 encode = tmap_encoder();
+  if (encode == nullptr) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)cols * 4};
+  const cuuint32_t box[2] = {32u, (cuuint32_t)box_rows};
+  const cuuint32_t estr[2] = {1u, 1u};
+  return encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, estr,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }

@@ -94,6 +94,11 @@ def test_short_workspace_is_rejected(lib):
     assert need > 0
     assert call_forward(lib, s, ws_bytes=need - 1) == WORKSPACE
     assert call_forward(lib, s, ws=0) == WORKSPACE
+    need = hsa.workspace_size(hsa.HSA_OP_SELECT, s)
+    assert need > 0
+    c = s.c()
+    vp = ctypes.c_void_p
+    assert lib.hsa_select_topk(ctypes.byref(c), *[vp(FAKE)] * 5, need - 1, None) == WORKSPACE
 
 
 def test_empty_problems_succeed_without_launching(lib):
@@ -136,7 +141,9 @@ def test_decode_noalloc_rejects_shapes_beyond_its_scratch(lib):
 def test_workspace_sizes_scale_with_the_problem(lib):
     s = shape(B=2, L=32768, Hq=32, Hkv=4)
     slots = 2 * 32768 * 4 * 8
-    assert hsa.workspace_size(hsa.HSA_OP_SELECT, s) == 0
+    # selection on the tensor cores keeps q̂ (bf16 and fp32) per (b, g, t) row
+    assert hsa.workspace_size(hsa.HSA_OP_SELECT, s) >= 2 * 32768 * 4 * 128 * 6
+    assert hsa.workspace_size(hsa.HSA_OP_SELECT, shape(B=2, L=32768, Hq=32, Hkv=4, topk=24)) == 0
     assert hsa.workspace_size(hsa.HSA_OP_FORWARD, s) == slots * 8 * 128 * 2
     assert hsa.workspace_size(hsa.HSA_OP_BACKWARD, s) >= slots * 8 * 128 * 2
     assert hsa.workspace_size(hsa.HSA_OP_INDEX, s) >= slots * 16

@@ -17,15 +17,16 @@
 // u_i < lambda is strictly below it (with room to spare for the final
 // rounding by c_sel, so no tie can be created).
 //
-// Per block: 128 consecutive tokens of one (b, g) against tiles of 128 chunk
-// summaries. Thread r of the four scan warps owns token row r (tensor-memory
-// lane r). It keeps the k largest lower bounds in a sorted register list
-// (whose last entry is lambda) and, in a shared-memory buffer, the other
-// chunks whose upper bound reaches the current lambda (lambda only rises, so
-// a chunk dropped once stays out). A row's first 32 scores go through a
-// sorting network at once; later ones are filtered against lambda and only
-// the few that pass are inserted one by one.
-// At the end the candidates (typically k plus a few) are rescored exactly in
+// Per block: 128 consecutive tokens of one (b, g) against tiles of 64 chunk
+// summaries, in two passes over the tiles (the MMAs run twice). Thread r of
+// the four scan warps owns token row r (tensor-memory lane r).
+//   Pass 1: per group of columns, (largest bf16 score - the tile's largest
+//   eps) is at most the group's best lower bound; the k-th largest such term,
+//   lam_lo, is a lower bound of lambda (min/max only, no branches).
+//   Pass 2: every chunk whose upper bound reaches lam_lo goes to a per-row
+//   buffer (typically k plus a few); it holds every chunk whose lower bound
+//   reaches lambda, so lambda is the k-th largest lower bound in the buffer.
+// The buffer entries whose upper bound reaches lambda are rescored exactly in
 // fp32 and the top k emitted. A row whose buffer overflows is handed to an
 // exact warp-per-row pass. The L x (L/S) score matrix never leaves the chip.
 #include <algorithm>
@@ -37,47 +38,50 @@ namespace hsa {
 namespace {
 
 constexpr int kTok = 128;      // token rows per block (MMA M, tensor-memory lanes)
-constexpr int kCt = 128;       // chunk summaries per tile (MMA N)
-constexpr int kAcc = 4;        // score accumulators in tensor memory (kCt columns each)
+constexpr int kCt = 64;        // chunk summaries per tile (MMA N)
 constexpr int kThreads = 192;  // warps 0-3 scan (thread = row), 4 loader, 5 MMA
-constexpr int kTmemCols = kAcc * kCt;
 constexpr float kEpsRel = 1.f / 128.f;
 // Absolute floor of eps_i: covers products the tensor core may flush to zero
 // (operands below the normal range), far below any score it could reorder.
 constexpr float kEpsAbs = 1e-25f;
 
+// Per list size: pipeline depth, buffer capacity and blocks per SM. With
+// K_T = 8 two blocks share an SM (about 106 KB of shared memory and 128
+// tensor-memory columns each), so one block's waits overlap the other's work.
 template <int KT>
-constexpr int window_cap() { return KT <= 8 ? 32 : 48; }
+struct SelCfg {
+  static constexpr int kStages = KT <= 8 ? 2 : 4;  // chunk-summary tiles in flight
+  static constexpr int kAcc = KT <= 8 ? 2 : 4;     // score accumulators in tensor memory (kCt columns each)
+  static constexpr int kBuf = KT <= 8 ? 24 : 64;   // candidate entries per row (second pass)
+  static constexpr int kBlocksPerSm = KT <= 8 ? 2 : 1;
+  static constexpr int kTmemCols = kAcc * kCt;
+};
 
 __device__ unsigned g_sel_status;
 
 template <int D, int KT>
 struct SelTcSmem {
-  static constexpr int kStages = KT <= 8 ? 4 : 3;  // chunk-summary tiles in flight
-  static constexpr int kCap = window_cap<KT>();
-  static constexpr int kCandMax = KT + kCap;
-  static constexpr size_t kTileBytes = (size_t)kStages * kCt * D * 2;
-  static constexpr size_t kQ32Bytes = (size_t)kTok * D * 4;
-  static constexpr size_t kAfterBytes = kQ32Bytes + (size_t)KT * kTok * 8;
-  static constexpr size_t kUnionBytes = kTileBytes > kAfterBytes ? kTileBytes : kAfterBytes;
+  using Cfg = SelCfg<KT>;
+  static constexpr int kStages = Cfg::kStages, kAcc = Cfg::kAcc, kBuf = Cfg::kBuf;
   // barrier slots
   static constexpr int BAR_A = 0, BAR_Q32 = 1, BAR_FULL = 2, BAR_EMPTY = 2 + kStages,
                        BAR_ACC_FULL = 2 + 2 * kStages, BAR_ACC_EMPTY = BAR_ACC_FULL + kAcc,
                        BAR_KN = BAR_ACC_EMPTY + kAcc, kBars = BAR_KN + kAcc;
-  uint16_t A[kTok * D];  // q̂ (bf16) of the block's rows, K-major SW128
-  // chunk-summary tiles while scanning; afterwards the rows' fp32 q̂ (128-byte
-  // swizzled boxes of 32 columns) and the chosen keys [KT][kTok]
-  alignas(1024) unsigned char U[kUnionBytes];
-  float wv[kCandMax][kTok];  // window buffer (upper bounds u_i); then the candidates' exact scores
-  int wi[kCandMax][kTok];    // their chunk indices
-  float knt[kAcc][kCt + 4];  // |K̄_i| of the tile in accumulator ab, then the tile's max
+  // A and B are adjacent: once every MMA is done they hold the rows' fp32 q̂ ([e][row], 128 * D floats)
+  uint16_t A[kTok * D];                  // q̂ (bf16) of the block's rows, K-major SW128
+  uint16_t B[kStages][kCt * D];          // chunk-summary tiles, K-major SW128
+  float bl[kBuf][kTok];                  // second-pass entries: lower bounds, later exact scores
+  float bu[kBuf][kTok];                  //   upper bounds
+  int bi[kBuf][kTok];                    //   chunk indices
+  unsigned long long chosen[KT][kTok];   // the k best exact keys
+  float knt[kAcc][kCt + 4];              // |K̄_i| of the tile in accumulator ab, then the tile's max
   uint64_t bar[kBars];
   uint32_t tmem_base;
   int abort_flag;
 };
 
 struct SelTcArgs {
-  const float* qh32;      // [B*Hkv*L, D] fp32 q̂
+  const float* qh32t;     // [B*Hkv, D, Lp] fp32 q̂, transposed (tokens adjacent)
   const float* qn;        // [B*Hkv*L] |q̂|
   const float* kbar32;    // [B, Nc, Hkv, D]
   const float* kn;        // [B*Hkv, Ncp] |K̄_i|
@@ -86,28 +90,9 @@ struct SelTcArgs {
   float* s_sel;
   unsigned* nflag;        // rows handed to the exact pass
   int32_t* flags;
-  int L, Hkv, Nc, Ncp, topk, n_qt, BH;
+  int L, Lp, Hkv, Nc, Ncp, topk, n_qt, BH;
   float scale_sel;
 };
-
-// Register list sorted by decreasing lower bound l (with the entry's upper
-// bound u and chunk index); l is known to beat v[KT-1].
-template <int KT>
-__device__ __forceinline__ void list_insert(float (&v)[KT], float (&vu)[KT], int (&id)[KT], float l, float u, int c) {
-#pragma unroll
-  for (int i = KT - 1; i > 0; --i) {
-    const bool up = l > v[i - 1];
-    const bool here = l > v[i];
-    v[i] = up ? v[i - 1] : (here ? l : v[i]);
-    vu[i] = up ? vu[i - 1] : (here ? u : vu[i]);
-    id[i] = up ? id[i - 1] : (here ? c : id[i]);
-  }
-  if (l > v[0]) {
-    v[0] = l;
-    vu[0] = u;
-    id[0] = c;
-  }
-}
 
 // x[c] for a run-time c in [0, 32): a five-level select tree.
 __device__ __forceinline__ float pick32(const float (&x)[32], int c) {
@@ -123,37 +108,13 @@ __device__ __forceinline__ float pick32(const float (&x)[32], int c) {
   return (c & 16) ? t[1] : t[0];
 }
 
-// Bitonic sorting network, descending by l, carrying u and c along.
-template <int N>
-__device__ __forceinline__ void sort_desc(float (&l)[N], float (&u)[N], int (&c)[N]) {
-#pragma unroll
-  for (int size = 2; size <= N; size <<= 1)
-#pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1)
-#pragma unroll
-      for (int i = 0; i < N; ++i) {
-        const int j = i ^ stride;
-        if (j > i) {
-          const bool sw = (i & size) == 0 ? (l[i] < l[j]) : (l[i] > l[j]);
-          const float tl = sw ? l[j] : l[i], tu = sw ? u[j] : u[i];
-          const int tc = sw ? c[j] : c[i];
-          l[j] = sw ? l[i] : l[j];
-          u[j] = sw ? u[i] : u[j];
-          c[j] = sw ? c[i] : c[j];
-          l[i] = tl;
-          u[i] = tu;
-          c[i] = tc;
-        }
-      }
-}
-
 template <int D, int KT>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     sel_tc_kernel(SelTcArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
-                  const __grid_constant__ CUtensorMap tmap_q32) {
+                  const __grid_constant__ CUtensorMap tmap_q32t) {
   extern __shared__ unsigned char smem_raw[];
   using Smem = SelTcSmem<D, KT>;
-  constexpr int kStages = Smem::kStages;
+  constexpr int kStages = Smem::kStages, kAcc = Smem::kAcc, kTmemCols = SelCfg<KT>::kTmemCols;
   constexpr int BAR_A = Smem::BAR_A, BAR_Q32 = Smem::BAR_Q32, BAR_FULL = Smem::BAR_FULL, BAR_EMPTY = Smem::BAR_EMPTY,
                 BAR_ACC_FULL = Smem::BAR_ACC_FULL, BAR_ACC_EMPTY = Smem::BAR_ACC_EMPTY, BAR_KN = Smem::BAR_KN;
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
@@ -165,6 +126,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int t_last = min(t0 + kTok, a.L) - 1;
   const int vis_max = min(t_last / kChunk, a.Nc);
   const int ntiles = (vis_max + kCt - 1) / kCt;
+  // Blocks start their sweep at different tiles, so that concurrent blocks of
+  // one (b, g) do not all request the same chunk-summary lines at once.
+  const int rot = ntiles > 0 ? (int)(blockIdx.x % (unsigned)ntiles) : 0;
+  auto tile_of = [&](int it) {
+    const int j = it < ntiles ? it : it - ntiles;
+    return j + rot < ntiles ? j + rot : j + rot - ntiles;
+  };
   auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
   volatile int* abort_flag = &sm.abort_flag;
   unsigned* status = &g_sel_status;
@@ -189,7 +157,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = sm.tmem_base;
-  const uint32_t abase = smem_u32(sm.A), ubase = smem_u32(sm.U);
+  const uint32_t abase = smem_u32(sm.A), ubase = smem_u32(sm.B);
   constexpr uint32_t kStageBytes = kCt * D * 2;
 
   if (warp == 4) {
@@ -199,9 +167,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int kb = 0; kb < D / 64; ++kb)
         tc::tma_load_2d(abase + kb * kTok * 128, &tmap_q, kb * 64, bg * a.L + t0, bar(BAR_A));
-      for (int n = 0; n < ntiles; ++n) {
-        const int s = n % kStages;
-        if (!tc::mbar_wait(bar(BAR_EMPTY + s), ((n / kStages) & 1) ^ 1, abort_flag, status)) break;
+      for (int it = 0; it < 2 * ntiles; ++it) {  // two passes over the tiles
+        const int n = tile_of(it);
+        const int s = it % kStages;
+        if (!tc::mbar_wait(bar(BAR_EMPTY + s), ((it / kStages) & 1) ^ 1, abort_flag, status)) break;
         tc::mbar_arrive_expect_tx(bar(BAR_FULL + s), kStageBytes);
 #pragma unroll
         for (int kb = 0; kb < D / 64; ++kb)
@@ -215,10 +184,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && ntiles > 0) {
       constexpr uint32_t idesc = tc::idesc_bf16(kTok, kCt);
       bool ok = tc::mbar_wait(bar(BAR_A), 0, abort_flag, status);
-      for (int n = 0; ok && n < ntiles; ++n) {
-        const int s = n % kStages, ab = n % kAcc;
-        if (!tc::mbar_wait(bar(BAR_FULL + s), (n / kStages) & 1, abort_flag, status)) break;
-        if (!tc::mbar_wait(bar(BAR_ACC_EMPTY + ab), ((n / kAcc) & 1) ^ 1, abort_flag, status)) break;
+      for (int it = 0; ok && it < 2 * ntiles; ++it) {
+        const int n = tile_of(it);
+        const int s = it % kStages, ab = it % kAcc;
+        if (!tc::mbar_wait(bar(BAR_FULL + s), (it / kStages) & 1, abort_flag, status)) break;
+        if (!tc::mbar_wait(bar(BAR_ACC_EMPTY + ab), ((it / kAcc) & 1) ^ 1, abort_flag, status)) break;
         tc::fence_after_sync();
         // the tile's chunk norms travel with its accumulator (the scan has released both)
         tc::mbar_arrive_expect_tx(bar(BAR_KN + ab), (kCt + 4) * 4);
@@ -242,71 +212,41 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = tid;
     const int t = t0 + r;
     const int vis = t < a.L ? min(t / kChunk, a.Nc) : 0;
-    constexpr int kCap = Smem::kCap;
+    constexpr int kBuf = Smem::kBuf;
     const long long qrow = (long long)bg * a.L + t;
     const float cq = vis > 0 ? kEpsRel * a.qn[qrow] : 0.f;  // eps_i = cq * |K̄_i| + kEpsAbs
-    // slots [KT-k, KT) hold the k largest lower bounds (descending); the slots
-    // above hold +inf and never move, so v[KT-1] is always lambda
-    float v[KT], vu[KT];
-    int id[KT];
+    // First pass: the k-th largest of (max over a group of columns - the
+    // tile's largest eps) is a lower bound of lambda, since each group holds a
+    // chunk whose lower bound is at least its term. Groups of 32 or 8 columns,
+    // or single columns for short rows, keep at least 2k terms per row.
+    const int vis0 = min(t0 / kChunk, a.Nc);
+    const int gsz = vis0 >= 64 * a.topk ? 32 : (vis0 >= 16 * a.topk ? 8 : 1);
+    float bm[KT];  // slots [KT-k, KT): the k largest terms (descending); +inf above
 #pragma unroll
-    for (int i = 0; i < KT; ++i) {
-      v[i] = i < KT - a.topk ? INFINITY : -INFINITY;
-      vu[i] = v[i];
-      id[i] = -1;
-    }
-    float thr = -INFINITY;  // lambda = v[KT-1]
-    bool fresh = true;      // no score of this row seen yet
-    int wcnt = 0;
+    for (int i = 0; i < KT; ++i) bm[i] = i < KT - a.topk ? INFINITY : -INFINITY;
+    auto push = [&](float v) {  // branch-free insertion: bm keeps the k largest
+#pragma unroll
+      for (int i = 0; i < KT; ++i) {
+        const float hi = fmaxf(bm[i], v);
+        v = fminf(bm[i], v);
+        bm[i] = hi;
+      }
+    };
+    float lam_lo = -INFINITY;
+    int cnt = 0;  // second-pass entries
     bool overflow = false;
 
-    auto window_append = [&](float x, int c) {
-      if (wcnt == kCap) {  // drop entries that fell below the window
-        int j = 0;
-        for (int i = 0; i < kCap; ++i) {
-          const float wx = sm.wv[i][r];
-          if (wx >= thr) {
-            sm.wv[j][r] = wx;
-            sm.wi[j][r] = sm.wi[i][r];
-            ++j;
-          }
-        }
-        wcnt = j;
-        if (wcnt == kCap) {
-          overflow = true;
-          thr = INFINITY;
-          return;
-        }
-      }
-      sm.wv[wcnt][r] = x;
-      sm.wi[wcnt][r] = c;
-      ++wcnt;
-    };
-    auto consider = [&](float x, int c, float knc) {
-      const float e = fmaf(cq, knc, kEpsAbs);
-      const float u = x + e;
-      if (!(u >= thr)) return;
-      const float l = x - e;
-      if (l > v[KT - 1]) {
-        const float eu = vu[KT - 1];
-        const int eid = id[KT - 1];
-        list_insert<KT>(v, vu, id, l, u, c);
-        thr = v[KT - 1];
-        if (eid >= 0 && eu >= thr) window_append(eu, eid);
-      } else {
-        window_append(u, c);
-      }
-    };
-
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-    for (int n = 0; n < ntiles; ++n) {
-      const int ab = n % kAcc;
-      if (!tc::mbar_wait(bar(BAR_ACC_FULL + ab), (n / kAcc) & 1, abort_flag, status)) break;
-      if (!tc::mbar_wait(bar(BAR_KN + ab), (n / kAcc) & 1, abort_flag, status)) break;
+    for (int it = 0; it < 2 * ntiles; ++it) {
+      const bool second = it >= ntiles;
+      const int n = tile_of(it);
+      const int ab = it % kAcc;
+      if (it == ntiles) lam_lo = bm[KT - 1];
+      if (!tc::mbar_wait(bar(BAR_ACC_FULL + ab), (it / kAcc) & 1, abort_flag, status)) break;
+      if (!tc::mbar_wait(bar(BAR_KN + ab), (it / kAcc) & 1, abort_flag, status)) break;
       tc::fence_after_sync();
       const float* knt = sm.knt[ab];
-      // coarse filter of the tile: a_i + eps_i >= lambda needs a_i >= lambda - cq * max_tile |K̄_i| - kEpsAbs
-      const float emax = fmaf(cq, knt[kCt], kEpsAbs);
+      const float emax = fmaf(cq, knt[kCt], kEpsAbs);  // the tile's largest eps_i
 #pragma unroll 1
       for (int h = 0; h < kCt / 32; ++h) {
         float x[32];
@@ -316,60 +256,76 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int c0 = n * kCt + h * 32;
         const int lim = vis - c0;
         if (lim <= 0) continue;
-        if (fresh) {
-          // first 32 scores of the row: bounds, one sort, the top k to the list
-          fresh = false;
-          float sl[32], su[32];
-          int sc[32];
+        if (!second) {
+          if (lim < 32) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            const float e = fmaf(cq, knt[h * 32 + c], kEpsAbs);
-            const bool ok = c < lim;
-            sl[c] = ok ? x[c] - e : -INFINITY;
-            su[c] = ok ? x[c] + e : -INFINITY;
-            sc[c] = ok ? c0 + c : -1;
+            for (int c = 0; c < 32; ++c) x[c] = c < lim ? x[c] : -INFINITY;
           }
-          sort_desc<32>(sl, su, sc);
+          if (gsz == 1) {
 #pragma unroll
-          for (int j = 0; j < KT; ++j)
-            if (j < a.topk && sc[j] >= 0) list_insert<KT>(v, vu, id, sl[j], su[j], sc[j]);
-          thr = v[KT - 1];
+            for (int c = 0; c < 32; ++c) push(x[c] - emax);
+          } else {
+            float m8[4];
 #pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (j >= a.topk && sc[j] >= 0 && su[j] >= thr) window_append(su[j], sc[j]);
-          continue;
-        }
-        uint32_t m = 0;
-        const float lo = thr - emax;
+            for (int j = 0; j < 4; ++j) {
+              m8[j] = fmaxf(fmaxf(fmaxf(x[8 * j], x[8 * j + 1]), fmaxf(x[8 * j + 2], x[8 * j + 3])),
+                            fmaxf(fmaxf(x[8 * j + 4], x[8 * j + 5]), fmaxf(x[8 * j + 6], x[8 * j + 7])));
+            }
+            if (gsz == 8) {
 #pragma unroll
-        for (int c = 0; c < 32; ++c) m |= (c < lim && x[c] >= lo) ? (1u << c) : 0u;
-        while (m) {
-          const int c = __ffs(m) - 1;
-          m &= m - 1;
-          const float xc = pick32(x, c);
-          if (xc >= thr - emax) consider(xc, c0 + c, knt[h * 32 + c]);
+              for (int j = 0; j < 4; ++j) push(m8[j] - emax);
+            } else {
+              push(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])) - emax);
+            }
+          }
+        } else {
+          // second pass: every chunk whose upper bound reaches lam_lo
+          uint32_t m = 0;
+          const float lo = lam_lo - emax;
+#pragma unroll
+          for (int c = 0; c < 32; ++c) m |= x[c] >= lo ? (1u << c) : 0u;
+          if (lim < 32) m &= (1u << lim) - 1u;
+          while (m) {
+            const int c = __ffs(m) - 1;
+            m &= m - 1;
+            const float xc = pick32(x, c);
+            const float e = fmaf(cq, knt[h * 32 + c], kEpsAbs);
+            if (xc + e >= lam_lo) {
+              if (cnt < kBuf) {
+                sm.bl[cnt][r] = xc - e;
+                sm.bu[cnt][r] = xc + e;
+                sm.bi[cnt][r] = c0 + c;
+              }
+              ++cnt;
+            }
+          }
         }
       }
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_ACC_EMPTY + ab));
     }
+    if (cnt > kBuf) overflow = true;
+    if (ntiles == 0) cnt = 0;
 
     // ---------------------------------------------------------------- exact rescoring of the candidates
-    // Every MMA has completed once the last accumulator was seen, so the
-    // stage buffers are free: the rows' fp32 q̂ lands there in one TMA load.
+    // Every MMA has completed once the last accumulator was seen, so A and B
+    // are free: the rows' fp32 q̂ lands there in one TMA box ([e][row]).
     if (r == 0 && ntiles > 0 && !*abort_flag) {
       tc::mbar_arrive_expect_tx(bar(BAR_Q32), kTok * D * 4);
-#pragma unroll
-      for (int cb = 0; cb < D / 32; ++cb)
-        tc::tma_load_2d(ubase + cb * kTok * 128, &tmap_q32, cb * 32, bg * a.L + t0, bar(BAR_Q32));
+      tc::tma_load_2d(abase, &tmap_q32t, t0, bg * D, bar(BAR_Q32));
     }
-    // candidates: the window entries whose upper bound still reaches lambda, then the list
+    // lambda itself: the k-th largest lower bound among the entries (they
+    // include every chunk whose lower bound reaches lam_lo); the candidates
+    // are the entries whose upper bound reaches it
     int nc = 0;
-    for (int j = 0; j < wcnt; ++j)
-      if (sm.wv[j][r] >= thr) sm.wi[nc++][r] = sm.wi[j][r];
+    if (!overflow) {
 #pragma unroll
-    for (int i = 0; i < KT; ++i)
-      if (id[i] >= 0) sm.wi[nc++][r] = id[i];
+      for (int i = 0; i < KT; ++i) bm[i] = i < KT - a.topk ? INFINITY : -INFINITY;
+      for (int j = 0; j < cnt; ++j) push(sm.bl[j][r]);
+      const float lam = bm[KT - 1];
+      for (int j = 0; j < cnt; ++j)
+        if (sm.bu[j][r] >= lam) sm.bi[nc++][r] = sm.bi[j][r];
+    }
     const bool q_ok = ntiles == 0 || tc::mbar_wait(bar(BAR_Q32), 0, abort_flag, status);
     if (t < a.L && q_ok && !*abort_flag) {
       const long long p = ((long long)b * a.L + t) * a.Hkv + g;
@@ -379,38 +335,37 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (overflow) {
         a.flags[atomicAdd(a.nflag, 1u)] = (int32_t)p;
       } else {
-        unsigned long long(*chosen)[kTok] = reinterpret_cast<unsigned long long(*)[kTok]>(sm.U + Smem::kQ32Bytes);
-        const unsigned char* qrow_s = sm.U + r * 128;
+        unsigned long long(*chosen)[kTok] = sm.chosen;
+        // q̂ of this row: element e at qs[e * kTok] (a warp's rows are adjacent words)
+        const float* qs = reinterpret_cast<const float*>(sm.A) + r;
         const float* kb = a.kbar32 + ((long long)b * a.Nc * a.Hkv + g) * D;
-        for (int j0 = 0; j0 < nc; j0 += 4) {
-          const float4* k4[4];
-          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        // one candidate at a time: each lane streams one K̄ row, 128 bytes
+        // (eight float4) per step, so a warp keeps 4 KB of lines live in L1
+        for (int j = 0; j < nc; ++j) {
+          const float4* k4 = reinterpret_cast<const float4*>(kb + (long long)sm.bi[j][r] * a.Hkv * D);
+          float acc = 0.f;
+#pragma unroll 1
+          for (int e8 = 0; e8 < D / 32; ++e8) {
+            float4 kv[8];
 #pragma unroll
-          for (int u = 0; u < 4; ++u)
-            k4[u] = reinterpret_cast<const float4*>(kb + (long long)sm.wi[j0 + u < nc ? j0 + u : j0][r] * a.Hkv * D);
-#pragma unroll 4
-          for (int e4 = 0; e4 < D / 4; ++e4) {
-            const float4 qv = *reinterpret_cast<const float4*>(qrow_s + (e4 >> 3) * (kTok * 128) +
-                                                               (((e4 & 7) ^ (r & 7)) << 4));
+            for (int u = 0; u < 8; ++u) kv[u] = __ldg(k4 + e8 * 8 + u);
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const float4 kv = __ldg(k4[u] + e4);
-              acc[u] = fmaf(qv.x, kv.x, acc[u]);
-              acc[u] = fmaf(qv.y, kv.y, acc[u]);
-              acc[u] = fmaf(qv.z, kv.z, acc[u]);
-              acc[u] = fmaf(qv.w, kv.w, acc[u]);
+            for (int u = 0; u < 8; ++u) {
+              const int e = e8 * 32 + 4 * u;
+              acc = fmaf(qs[e * kTok], kv[u].x, acc);
+              acc = fmaf(qs[(e + 1) * kTok], kv[u].y, acc);
+              acc = fmaf(qs[(e + 2) * kTok], kv[u].z, acc);
+              acc = fmaf(qs[(e + 3) * kTok], kv[u].w, acc);
             }
           }
-#pragma unroll
-          for (int u = 0; u < 4; ++u)
-            if (j0 + u < nc) sm.wv[j0 + u][r] = acc[u] * a.scale_sel;
+          sm.bl[j][r] = acc * a.scale_sel;
         }
         // the keff largest keys (keys are distinct: they carry the chunk index)
         unsigned long long prev = ~0ull;
         for (int s = 0; s < keff; ++s) {
           unsigned long long best = 0ull;
           for (int j = 0; j < nc; ++j) {
-            const unsigned long long kj = rank_key(sm.wv[j][r], (uint32_t)sm.wi[j][r]);
+            const unsigned long long kj = rank_key(sm.bl[j][r], (uint32_t)sm.bi[j][r]);
             if (kj < prev && kj > best) best = kj;
           }
           chosen[s][r] = best;
@@ -440,50 +395,58 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// q̂ of every (b, g, t) row: fp32 head-order sum, its bf16 rounding and its norm.
-// Threads D/8 per row, each 8 consecutive elements; rows in [b][g][t] order.
+// q̂ of every (b, g, t) row: the fp32 head-order sum (stored transposed,
+// [b*Hkv+g][e][t], so that the rows a warp rescores are adjacent in memory),
+// its bf16 rounding ([b*Hkv+g][t][e], the MMA operand) and its norm. One
+// block per 32 consecutive tokens of one (b, g).
 template <int D>
 __global__ void __launch_bounds__(256) sel_qhat_kernel(const uint16_t* __restrict__ q, uint16_t* __restrict__ qh16,
-                                                       float* __restrict__ qh32, float* __restrict__ qn,
-                                                       long long rows, int L, int Hq, int Hkv, int G) {
+                                                       float* __restrict__ qh32t, float* __restrict__ qn, int L,
+                                                       int Lp, int Hq, int Hkv, int G) {
+  __shared__ float qs[32][D + 1];
   constexpr int D8 = D / 8;
-  const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  const long long row = u / D8;
-  const int e8 = (int)(u % D8);
-  const bool valid = row < rows;
-  float acc[8];
+  const int bg = blockIdx.y;
+  const int t0 = blockIdx.x * 32;
+  const int b = bg / Hkv, g = bg % Hkv;
+  // the D8 threads of a row are adjacent lanes of one warp (256 and 32 are multiples of D8)
+  for (int u = threadIdx.x; u < 32 * D8; u += 256) {
+    const int rr = u / D8, e8 = u % D8;
+    const int t = t0 + rr;
+    float acc[8];
 #pragma unroll
-  for (int c = 0; c < 8; ++c) acc[c] = 0.f;
-  if (valid) {
-    const int t = (int)(row % L);
-    const long long bg = row / L;
-    const int g = (int)(bg % Hkv);
-    const long long b = bg / Hkv;
-    const uint4* src = reinterpret_cast<const uint4*>(q + ((b * L + t) * Hq + (long long)g * G) * D) + e8;
-    for (int hh = 0; hh < G; ++hh) {
-      const uint4 w = __ldg(src + (long long)hh * D8);
-      acc[0] = acc[0] + bf16_lo(w.x);
-      acc[1] = acc[1] + bf16_hi(w.x);
-      acc[2] = acc[2] + bf16_lo(w.y);
-      acc[3] = acc[3] + bf16_hi(w.y);
-      acc[4] = acc[4] + bf16_lo(w.z);
-      acc[5] = acc[5] + bf16_hi(w.z);
-      acc[6] = acc[6] + bf16_lo(w.w);
-      acc[7] = acc[7] + bf16_hi(w.w);
+    for (int c = 0; c < 8; ++c) acc[c] = 0.f;
+    if (t < L) {
+      const uint4* src = reinterpret_cast<const uint4*>(q + (((long long)b * L + t) * Hq + (long long)g * G) * D) + e8;
+      for (int hh = 0; hh < G; ++hh) {
+        const uint4 w = __ldg(src + (long long)hh * D8);
+        acc[0] = acc[0] + bf16_lo(w.x);
+        acc[1] = acc[1] + bf16_hi(w.x);
+        acc[2] = acc[2] + bf16_lo(w.y);
+        acc[3] = acc[3] + bf16_hi(w.y);
+        acc[4] = acc[4] + bf16_lo(w.z);
+        acc[5] = acc[5] + bf16_hi(w.z);
+        acc[6] = acc[6] + bf16_lo(w.w);
+        acc[7] = acc[7] + bf16_hi(w.w);
+      }
+      *reinterpret_cast<uint4*>(qh16 + ((long long)bg * L + t) * D + e8 * 8) =
+          make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
+                     pack_bf16x2(acc[6], acc[7]));
     }
-    float4* d32 = reinterpret_cast<float4*>(qh32 + row * D + e8 * 8);
-    d32[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
-    d32[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
-    *reinterpret_cast<uint4*>(qh16 + row * D + e8 * 8) =
-        make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
-                   pack_bf16x2(acc[6], acc[7]));
+#pragma unroll
+    for (int c = 0; c < 8; ++c) qs[rr][e8 * 8 + c] = acc[c];
+    float ss = 0.f;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) ss = fmaf(acc[c], acc[c], ss);
+#pragma unroll
+    for (int o = D8 / 2; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
+    if (t < L && e8 == 0) qn[(long long)bg * L + t] = sqrtf(ss);
   }
-  float ss = 0.f;
-#pragma unroll
-  for (int c = 0; c < 8; ++c) ss = fmaf(acc[c], acc[c], ss);
-#pragma unroll
-  for (int o = D8 / 2; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
-  if (valid && e8 == 0) qn[row] = sqrtf(ss);
+  __syncthreads();
+  for (int u = threadIdx.x; u < 32 * D; u += 256) {
+    const int e = u / 32, rr = u % 32;
+    const int t = t0 + rr;
+    if (t < L) qh32t[((long long)bg * D + e) * Lp + t] = qs[rr][e];
+  }
 }
 
 // K̄ in bf16 with rows reordered to [b][g][i], |K̄_i| in fp32 ([b*Hkv+g][Ncp])
@@ -526,15 +489,16 @@ __global__ void __launch_bounds__(256) sel_kbar_kernel(const float* __restrict__
   }
 }
 
-// Exact pass for the rows whose window buffer overflowed: one warp per row,
+// Exact pass for the rows whose candidate buffer overflowed: one warp per row,
 // lanes over chunks, the exact fp32 score chain and a warp-held top-k list.
 template <int D>
-__global__ void __launch_bounds__(256) sel_exact_rows_kernel(const float* __restrict__ qh32,
+__global__ void __launch_bounds__(256) sel_exact_rows_kernel(const float* __restrict__ qh32t,
                                                              const float* __restrict__ kbar32,
                                                              const unsigned* __restrict__ nflag,
                                                              const int32_t* __restrict__ flags,
                                                              int32_t* __restrict__ idx, float* __restrict__ s_sel,
-                                                             int L, int Hkv, int Nc, int topk, float scale_sel) {
+                                                             int L, int Lp, int Hkv, int Nc, int topk,
+                                                             float scale_sel) {
   __shared__ float qs[8][D];
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const unsigned n = *nflag;
@@ -545,9 +509,9 @@ __global__ void __launch_bounds__(256) sel_exact_rows_kernel(const float* __rest
     const int t = (int)(bt % L);
     const long long b = bt / L;
     const int vis = min(t / kChunk, Nc);
-    const float* qrow = qh32 + ((b * Hkv + g) * L + t) * D;
+    const float* qcol = qh32t + (b * Hkv + g) * D * Lp + t;
     __syncwarp();
-    for (int e = lane; e < D; e += 32) qs[wib][e] = qrow[e];
+    for (int e = lane; e < D; e += 32) qs[wib][e] = qcol[(long long)e * Lp];
     __syncwarp();
     unsigned long long lst = 0ull;
     for (int c0 = 0; c0 < vis; c0 += 32) {
@@ -579,6 +543,8 @@ struct SelLayout {
 };
 
 inline int padded_chunks(const Dims& D) { return (D.Nc + kCt - 1) / kCt * kCt; }
+// Row length of the transposed fp32 q̂ (a multiple of 4 tokens: TMA row strides are multiples of 16 bytes).
+inline int padded_tokens(const Dims& D) { return (D.L + 3) / 4 * 4; }
 
 // Row counts of the two bf16 operand matrices, padded to one full box (the
 // padding rows are never selected: they lie past every row's visible range).
@@ -593,7 +559,7 @@ SelLayout sel_layout(const Dims& D) {
   lo.qh16 = o;
   o = align256(o + rows * D.d * 2);
   lo.qh32 = o;
-  o = align256(o + rows * D.d * 4);
+  o = align256(o + (size_t)D.B * D.Hkv * D.d * padded_tokens(D) * 4);
   lo.qn = o;
   o = align256(o + rows * 4);
   lo.kb16 = o;
@@ -624,15 +590,15 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   unsigned* ktmax = (unsigned*)(base + lo.ktmax);
   unsigned* nflag = (unsigned*)(base + lo.nflag);
   int32_t* flags = (int32_t*)(base + lo.flags);
-  const long long rows = (long long)Dm.B * Dm.Hkv * Dm.L;
   const long long krows = (long long)Dm.B * Dm.Nc * Dm.Hkv;
   const int BH = Dm.B * Dm.Hkv;
   cudaError_t e;
   // the tile maxima and the flagged-row counter are adjacent: one clear covers both
   if ((e = cudaMemsetAsync(ktmax, 0, lo.flags - lo.ktmax, st)) != cudaSuccess) return e;
   constexpr int D8 = DD / 8;
-  sel_qhat_kernel<DD><<<(unsigned)((rows * D8 + 255) / 256), 256, 0, st>>>((const uint16_t*)q, qh16, qh32, qn, rows,
-                                                                          Dm.L, Dm.Hq, Dm.Hkv, Dm.G);
+  const int Lp = padded_tokens(Dm);
+  sel_qhat_kernel<DD><<<dim3((unsigned)((Dm.L + 31) / 32), (unsigned)BH), 256, 0, st>>>((const uint16_t*)q, qh16, qh32,
+                                                                                      qn, Dm.L, Lp, Dm.Hq, Dm.Hkv, Dm.G);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int Ncp = padded_chunks(Dm);
@@ -641,15 +607,15 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
-  CUtensorMap tq, tk, tq32;
+  CUtensorMap tq, tk, tq32t;
   memset(&tq, 0, sizeof(tq));
   memset(&tk, 0, sizeof(tk));
-  memset(&tq32, 0, sizeof(tq32));
-  if (!tc::make_rows_tmap_f32(&tq32, qh32, (unsigned long long)q_rows(Dm), DD, kTok)) return cudaErrorNotSupported;
+  memset(&tq32t, 0, sizeof(tq32t));
+  if (!tc::make_plain_tmap_f32(&tq32t, qh32, (unsigned long long)BH * DD, Lp, kTok, DD)) return cudaErrorNotSupported;
   if (!tc::make_rows_tmap(&tq, qh16, (unsigned long long)q_rows(Dm), DD, kTok)) return cudaErrorNotSupported;
   if (!tc::make_rows_tmap(&tk, kb16, (unsigned long long)k_rows(Dm), DD, kCt)) return cudaErrorNotSupported;
   SelTcArgs a;
-  a.qh32 = qh32;
+  a.qh32t = qh32;
   a.qn = qn;
   a.kbar32 = kbar32;
   a.kn = kn;
@@ -659,6 +625,7 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   a.nflag = nflag;
   a.flags = flags;
   a.L = Dm.L;
+  a.Lp = Lp;
   a.Hkv = Dm.Hkv;
   a.Nc = Dm.Nc;
   a.Ncp = Ncp;
@@ -671,11 +638,11 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
       cudaSuccess)
     return e;
   const long long blocks = (long long)a.n_qt * BH;
-  sel_tc_kernel<DD, KT><<<(unsigned)blocks, kThreads, smem, st>>>(a, tq, tk, tq32);
+  sel_tc_kernel<DD, KT><<<(unsigned)blocks, kThreads, smem, st>>>(a, tq, tk, tq32t);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  sel_exact_rows_kernel<DD><<<2 * 152, 256, 0, st>>>(qh32, kbar32, nflag, flags, idx, s_sel, Dm.L, Dm.Hkv, Dm.Nc,
-                                                     Dm.topk, Dm.scale_sel);
+  sel_exact_rows_kernel<DD><<<2 * 152, 256, 0, st>>>(qh32, kbar32, nflag, flags, idx, s_sel, Dm.L, Lp, Dm.Hkv,
+                                                     Dm.Nc, Dm.topk, Dm.scale_sel);
   note_launches(1);
   return cudaGetLastError();
 }

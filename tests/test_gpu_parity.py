@@ -127,6 +127,24 @@ def test_exact_score_ties_break_toward_lower_chunk():
     assert (ref["gap"] == 0).any()
 
 
+@pytest.mark.parametrize("topk", [8, 16])
+def test_selection_many_equal_chunks_takes_the_exact_pass(topk):
+    # every complete chunk is a copy of chunk 0: all scores of a row tie, the
+    # per-row candidate buffer of the tensor-core selection overflows and the
+    # rows go through the exact pass; ties rank the lower chunk index first
+    w = synth.Workload("all-equal", 48, B=1, L=64 * 120 + 17, S=64, Hq=8, Hkv=2, d=64, topk=topk)
+    bits = host_inputs(w)
+    K = bits["K"]
+    for c in range(1, w.L // 64):
+        K[:, c * 64:(c + 1) * 64] = K[:, 0:64]
+    got, ref = check_prefill(w, bits=bits)
+    idx = got["idx"].cpu().numpy()
+    vis = np.minimum(np.arange(w.L) // 64, w.Nc)
+    for t in (200, 64 * 70, w.L - 1):
+        keff = min(topk, vis[t])
+        assert list(idx[0, t, 0, :keff]) == list(range(keff - 1, -1, -1)), t
+
+
 def test_backward_is_deterministic():
     w = synth.WORKLOADS[2].with_(B=2, L=2048)
     bits = host_inputs(w)

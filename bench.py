@@ -52,7 +52,11 @@ def select_workload(number, batch):
 # kernel from one ncu capture, keyed by the source file it was compiled from
 # and that file's sha256 at capture time (reported as null once the source
 # has changed).
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {
+    # bwd_delta + bwd_chunk + bwd_dq_merge at the long-context workload (B=2, L=32768), one launch each
+    "hsa_backward": {"bytes_per_launch": 15075620096, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
+                     "sha256": "abfbeaf8dd1418c3cc8654fe0238e8d36f783348f1f64ae5ae4a0088febb9904"},
+}
 
 
 def log(*a):

@@ -130,8 +130,12 @@ hsa_status_t hsa_chunk_pool(const hsa_shape_t* shape, const void* K, float* kbar
  *   s_sel  [B, L, Hkv, topk] fp32, output: their scores, -inf padded.
  * Scores are fp32: q̂ = fp32 sum of the group's heads in head order,
  * dot = fused multiply-add chain over d in order, s = dot * c_sel. The score
- * matrix is never written to memory. ws may be NULL when the workspace size
- * is 0.
+ * matrix is never written to memory. For topk <= 16 the scan runs as bf16
+ * tensor-core products whose rounding error is bounded per score; only the
+ * chunks the bound cannot rule out are rescored with the fp32 chain, so idx
+ * and s_sel are exactly those of the definition above. That path needs
+ * workspace HSA_OP_SELECT; for topk > 16 every score is computed with the
+ * fp32 chain and the workspace size is 0 (ws may then be NULL).
  */
 hsa_status_t hsa_select_topk(const hsa_shape_t* shape, const void* q, const float* kbar32, int32_t* idx,
                              float* s_sel, void* ws, size_t ws_bytes, cudaStream_t stream);

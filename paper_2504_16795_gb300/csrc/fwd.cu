@@ -27,10 +27,11 @@ __device__ unsigned g_fwd_status;
 
 template <int D>
 struct FwdSmem {
-  uint16_t Q[kQStages][kRows * D];  // gathered query rows, K-major SW128
+  uint16_t Q[kQStages][kRows * D];  // gathered query rows, grouped K-major SW128 (tc::grp_offset)
   uint16_t K[kChunk * D];           // chunk keys [s][d]
   uint16_t Vt[D * kChunk];          // chunk values transposed [d][s]
   uint16_t P[2][kRows * kChunk];    // normalised probabilities (bf16)
+  uint16_t Ostage[kRows * D];       // TMA path: the step's O' rows (grouped layout) on their way out
   int slot_row[kQStages][kRows];    // cp.async path: first q row of each slot (-1: past the list)
   uint64_t bar[16];
   uint32_t tmem_base;
@@ -61,7 +62,8 @@ struct FwdArgs {
 };
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const __grid_constant__ CUtensorMap tmap_q) {
+__global__ void __launch_bounds__(kThreads, 1)
+    fwd_chunk_kernel(FwdArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_o) {
   extern __shared__ unsigned char smem_raw[];
   FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
@@ -120,32 +122,30 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
 
   if (warp == 8) {
     // ---------------------------------------------------------------- loader warp
-    // TMA path: the next tile's slot rows are resolved before waiting for the
-    // current tile's stage, so the dependent global loads are off the critical path.
-    auto slot_y = [&](int i) {
+    // TMA path: the slot ids of a tile are loaded two tiles ahead and turned
+    // into query rows one tile ahead, so no dependent global load sits on the
+    // loader's critical path.
+    auto load_p = [&](int i) {
       const int e = i * epi + lane;
-      int y = a.n_rows;  // past the list: the box reads zeros
-      if (lane < epi && e < cnt) {
-        const int p = a.entries[off + e];
-        const int t = (p / slot_div) % a.L;
-        y = ((b * a.L + t) * a.Hq) + g * a.G;
-      }
-      return y;
+      return (a.use_tma && lane < epi && e < cnt) ? a.entries[off + e] : -1;
     };
-    int y_next = a.use_tma ? slot_y(0) : 0;
+    auto row_of = [&](int p) {  // past the list: rows past the tensor read zeros
+      return p < 0 ? a.n_rows : ((b * a.L + (p / slot_div) % a.L) * a.Hq) + g * a.G;
+    };
+    int p_cur = load_p(0), p_next = load_p(1);
     for (int i = 0; i < niter; ++i) {
       const int st = i % kQStages;
-      const int y = y_next;
-      if (a.use_tma && i + 1 < niter) y_next = slot_y(i + 1);
+      const int y = row_of(p_cur);
+      p_cur = p_next;
+      p_next = load_p(i + 2);
       tc::mbar_wait(bar(BAR_Q_EMPTY + st), ((i / kQStages) & 1) ^ 1, abort_flag, status);
       const uint32_t base = smem_u32(sm.Q[st]);
       if (a.use_tma) {
-        // lane l < epi gathers slot l's G rows as one box per 64 columns; the
+        // lane l < epi gathers slot l's G rows, one box per 8-row group; the
         // single expected arrival carries the byte count
         if (lane < epi) {
-#pragma unroll
-          for (int kb = 0; kb < D / 64; ++kb)
-            tc::tma_load_2d(base + kb * kRows * 128 + lane * a.G * 128, &tmap_q, kb * 64, y, bar(BAR_Q_FULL + st));
+          for (int j = 0; j < (a.G >> 3); ++j)
+            tc::tma_load_3d(base + (lane * (a.G >> 3) + j) * (16 * D), &tmap_q, 0, y + 8 * j, 0, bar(BAR_Q_FULL + st));
         }
         if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_Q_FULL + st), kRows * D * 2);
         continue;
@@ -164,7 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
       for (int u = lane; u < kRows * D8; u += 32) {
         const int r = u / D8, ch = u % D8;
         const int row = sm.slot_row[st][r >> a.log2G];
-        const uint32_t dst = base + tc::sw128_offset(kRows, r, ch * 8);
+        const uint32_t dst = base + tc::grp_offset(D, r, ch * 8);
         if (row >= 0) {
           cp_async16(dst, a.q + ((long long)(row + (r & (a.G - 1)))) * D + ch * 8);
         } else {
@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t blk = kk >> 2, w = kk & 3;
-          tc::mma_bf16_ss(tmem + sb * kChunk, tc::sdesc_sw128(qbase + blk * kRows * 128 + w * 32),
+          tc::mma_bf16_ss(tmem + sb * kChunk, tc::sdesc_sw128_sbo(qbase + blk * 1024 + w * 32, 16 * D),
                           tc::sdesc_sw128(kbase + blk * kChunk * 128 + w * 32), idS, kk > 0);
         }
         tc::mma_commit(bar(BAR_S_FULL + sb));
@@ -283,32 +283,55 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_chunk_kernel(FwdArgs a, const
     // ---------------------------------------------------------------- epilogue (thread = row)
     const int r = tid - 128;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    // TMA path (G >= 8): each warp writes its 32 rows into the staging tile
+    // (swizzled, conflict-free) and the first lane of every slot stores the
+    // slot's G rows with one TMA box per 8 rows. Otherwise rows go out directly.
+    const bool issuer = a.use_tma && (r & (a.G - 1)) == 0;
+    const uint32_t stage = smem_u32(sm.Ostage);
     int p_next = r >> a.log2G < cnt ? a.entries[off + (r >> a.log2G)] : -1;
     for (int j = 0; j < niter; ++j) {
       const int pj = p_next;
       const int en = (j + 1) * epi + (r >> a.log2G);
       p_next = en < cnt ? a.entries[off + en] : -1;  // prefetch the next step's slot
       const int ob = j & 1;
+      if (a.use_tma) {  // the previous step's stores have read this warp's part of the staging tile
+        if (issuer) tc::bulk_wait_read();
+        __syncwarp();
+      }
       tc::mbar_wait(bar(BAR_O_FULL + ob), (j >> 1) & 1, abort_flag, status);
       tc::fence_after_sync();
-      uint16_t* dst = pj >= 0 ? a.Opart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
+      uint16_t* dst = (!a.use_tma && pj >= 0) ? a.Opart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
 #pragma unroll
       for (int h = 0; h < D / 32; ++h) {
         float o[32];
         tc::tmem_ld32(tmem + lane_base + 2 * kChunk + ob * D + h * 32, o);
         tc::tmem_wait_ld();
-        if (dst) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + h * 32);
 #pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4)
-            d4[q4] = make_uint4(pack_bf16x2(o[8 * q4], o[8 * q4 + 1]), pack_bf16x2(o[8 * q4 + 2], o[8 * q4 + 3]),
-                                pack_bf16x2(o[8 * q4 + 4], o[8 * q4 + 5]),
-                                pack_bf16x2(o[8 * q4 + 6], o[8 * q4 + 7]));
+        for (int q4 = 0; q4 < 4; ++q4) {
+          const uint4 v = make_uint4(pack_bf16x2(o[8 * q4], o[8 * q4 + 1]), pack_bf16x2(o[8 * q4 + 2], o[8 * q4 + 3]),
+                                     pack_bf16x2(o[8 * q4 + 4], o[8 * q4 + 5]),
+                                     pack_bf16x2(o[8 * q4 + 6], o[8 * q4 + 7]));
+          if (a.use_tma) {
+            asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(stage + tc::grp_offset(D, r, h * 32 + 8 * q4)),
+                         "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w));
+          } else if (dst) {
+            reinterpret_cast<uint4*>(dst + h * 32)[q4] = v;
+          }
         }
       }
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_O_EMPTY + ob));
+      if (a.use_tma) {
+        tc::fence_proxy_async_smem();
+        __syncwarp();
+        if (issuer && pj >= 0) {
+          for (int jj = 0; jj < (a.G >> 3); ++jj)
+            tc::tma_store_3d(&tmap_o, 0, pj * a.G + 8 * jj, 0, stage + ((r >> 3) + jj) * (16 * D));
+          tc::bulk_commit();
+        }
+      }
     }
+    if (issuer) tc::bulk_wait_all();
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -400,12 +423,15 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     const size_t smem = sizeof(FwdSmem<D>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(fwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    CUtensorMap tq;
+    CUtensorMap tq, to;
     memset(&tq, 0, sizeof(tq));
+    memset(&to, 0, sizeof(to));
     a.n_rows = Dm.B * Dm.L * Dm.Hq;
     a.use_tma = Dm.G >= 8 ? 1 : 0;
-    if (a.use_tma && !tc::make_rows_tmap(&tq, q, (unsigned long long)a.n_rows, D, Dm.G)) return cudaErrorNotSupported;
-    fwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq);
+    if (a.use_tma && !tc::make_group8_tmap(&tq, q, (unsigned long long)a.n_rows, D)) return cudaErrorNotSupported;
+    if (a.use_tma && !tc::make_group8_tmap(&to, Opart, (unsigned long long)Dm.slots() * Dm.G, D))
+      return cudaErrorNotSupported;
+    fwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq, to);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

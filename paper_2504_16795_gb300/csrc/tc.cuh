@@ -73,6 +73,28 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
 // 2-D tiled bulk copy global -> shared (async proxy); completion is counted
 // in bytes on `bar`. x (the innermost coordinate) must be a multiple of 8
 // bf16 elements; rows beyond the tensor are filled with zeros.
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+      : "memory");
+}
+// 3-D tiled bulk copy shared -> global (async proxy), tracked by the issuing
+// thread's bulk group: commit with bulk_commit, and before the shared source
+// is written again wait with bulk_wait_read.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, int x, int y, int z, uint32_t src) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// The shared sources of all committed bulk groups have been read.
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// All committed bulk groups have completed (writes visible).
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
@@ -196,6 +218,25 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
                : "memory");
 }
 
+// K-major, 128-byte swizzle, 8-row groups `sbo` bytes apart (the start
+// address gives the 64-column block inside a group).
+__device__ __forceinline__ uint64_t sdesc_sw128_sbo(uint32_t addr, uint32_t sbo) {
+  return (uint64_t)((addr & 0x3FFFFu) >> 4)      // start address
+         | ((uint64_t)1 << 16)                   // leading byte offset (unused by swizzled K-major)
+         | ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32)  // stride byte offset: next 8-row group
+         | ((uint64_t)1 << 46)                   // descriptor version
+         | ((uint64_t)2 << 61);                  // 128-byte swizzle
+}
+
+// Grouped layout of a gathered tile of `cols` bf16 columns: rows in groups of
+// 8, group j at j * 16 * cols bytes, holding one 1024-byte swizzled atom
+// (8 rows x 64 columns) per 64-column block. One TMA box of 8 rows x all
+// columns fills one group. For cols = 64 it is the plain stacked layout.
+__device__ __forceinline__ uint32_t grp_offset(int cols, int row, int col) {
+  return (uint32_t)((row >> 3) * 16 * cols + (col >> 6) * 1024 + (row & 7) * 128 +
+                    ((((col >> 3) & 7) ^ (row & 7)) << 4) + ((col & 7) << 1));
+}
+
 // Byte offset of (row, col) in a K-major 128-byte-swizzled tile of `rows` rows
 // (bf16 elements; col may exceed 63: 64-column blocks are stacked).
 __device__ __forceinline__ uint32_t sw128_offset(int rows, int row, int col) {
@@ -227,6 +268,21 @@ inline bool make_rows_tmap(CUtensorMap* map, const void* base, unsigned long lon
   const cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
   const cuuint32_t estr[2] = {1u, 1u};
   return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// A bf16 matrix of `rows` x `cols` read 8 rows at a time into the grouped
+// layout (grp_offset): a 3-D view {64 columns, rows, cols/64 blocks} with box
+// {64, 8, cols/64} and the 128-byte swizzle.
+inline bool make_group8_tmap(CUtensorMap* map, const void* base, unsigned long long rows, int cols) {
+  PFN_cuTensorMapEncodeTiled_v12000 encode = tmap_encoder();
+  if (encode == nullptr) return false;
+  const cuuint64_t dims[3] = {64u, (cuuint64_t)rows, (cuuint64_t)(cols / 64)};
+  const cuuint64_t strides[2] = {(cuuint64_t)cols * 2, 128u};
+  const cuuint32_t box[3] = {64u, 8u, (cuuint32_t)(cols / 64)};
+  const cuuint32_t estr[3] = {1u, 1u, 1u};
+  return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }

@@ -48,8 +48,8 @@ __device__ unsigned g_bwd_status;
 
 template <int D>
 struct BwdSmem {
-  uint16_t Q[2][kRows * D];       // gathered query rows (K-major SW128)
-  uint16_t dO[2][kRows * D];      // gathered output gradients
+  uint16_t Q[2][kRows * D];       // gathered query rows (grouped K-major SW128, tc::grp_offset)
+  uint16_t dO[2][kRows * D];      // gathered output gradients (same layout)
   uint16_t K[kChunk * D];         // chunk keys [s][d]
   uint16_t V[kChunk * D];         // chunk values [s][d]
   uint16_t P[kRows * kChunk];     // w * P
@@ -173,28 +173,32 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 8) {
     // ---------------------------------------------------------------- loader warp
-    // The slot data of tile i+1 (entries -> token -> weight, Δ) is fetched
-    // before waiting for tile i's stage, so its dependent global loads are off
-    // the critical path.
+    // The slot data of a tile is fetched in two stages ahead of use: the slot
+    // ids two tiles ahead, the token, weight and Δ one tile ahead, so no
+    // dependent global load sits on the loader's critical path.
+    auto load_p = [&](int i) {
+      const int e = i * epi + lane;
+      return (epi <= 32 && lane < epi && e < cnt) ? a.entries[off + e] : -1;
+    };
     int n_row = -1, n_p = -1;
     float n_w = 0.f, n_dl = 0.f;
-    auto fetch = [&](int i) {
-      n_row = -1, n_p = -1, n_w = 0.f, n_dl = 0.f;
-      const int e = i * epi + lane;
-      if (lane < epi && e < cnt) {
-        n_p = a.entries[off + e];
-        const int t = (n_p / slot_div) % a.L;
+    auto resolve = [&](int p) {  // slot id -> query row, weight, Δ (loads issued, used an iteration later)
+      n_p = p, n_row = -1, n_w = 0.f, n_dl = 0.f;
+      if (p >= 0) {
+        const int t = (p / slot_div) % a.L;
         n_row = ((b * a.L + t) * a.Hq) + g * a.G;
-        n_w = a.w[n_p];
+        n_w = a.w[p];
         n_dl = a.delta[((long long)b * a.L + t) * a.Hkv + g];
       }
     };
-    fetch(0);
+    resolve(load_p(0));
+    int p_ahead = load_p(1);
     for (int i = 0; i < niter; ++i) {
       const int st = i & 1;
       const int c_row = n_row, c_p = n_p;
       const float c_w = n_w, c_dl = n_dl;
-      if (i + 1 < niter && epi <= 32) fetch(i + 1);
+      resolve(p_ahead);
+      p_ahead = load_p(i + 2);
       // cp.async path: publish tile i-1 before waiting for tile i's stage (that
       // stage is freed by the second half of step i-2, which the MMA thread
       // issues only after the first half of step i-1, which needs tile i-1)
@@ -236,11 +240,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // publishes the slot tables written above
         if (lane < epi) {
           const int y = c_row >= 0 ? c_row : a.n_rows;  // past the list: zeros
-#pragma unroll
-          for (int kb = 0; kb < D / 64; ++kb) {
-            const uint32_t o = kb * kRows * 128 + lane * a.G * 128;
-            tc::tma_load_2d(qb + o, &tmap_q, kb * 64, y, bar(BAR_QD_FULL + st));
-            tc::tma_load_2d(ob + o, &tmap_do, kb * 64, y, bar(BAR_QD_FULL + st));
+          for (int j = 0; j < (a.G >> 3); ++j) {  // one box per 8-row group
+            const uint32_t o = (lane * (a.G >> 3) + j) * (16 * D);
+            tc::tma_load_3d(qb + o, &tmap_q, 0, y + 8 * j, 0, bar(BAR_QD_FULL + st));
+            tc::tma_load_3d(ob + o, &tmap_do, 0, y + 8 * j, 0, bar(BAR_QD_FULL + st));
           }
         }
         __syncwarp();
@@ -251,7 +254,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = lane; u < kRows * D8; u += 32) {
         const int r = u / D8, ch = u % D8;
         const int row = sm.slot_row[st][r >> a.log2G];
-        const uint32_t o = tc::sw128_offset(kRows, r, ch * 8);
+        const uint32_t o = tc::grp_offset(D, r, ch * 8);
         if (row >= 0) {
           const long long src = ((long long)(row + (r & (a.G - 1)))) * D + ch * 8;
           cp_async16(qb + o, a.q + src);
@@ -274,9 +277,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idSP = tc::idesc_bf16(kRows, kChunk);                // S, dP': Q K^T, dO V^T
       constexpr uint32_t idDQ = tc::idesc_bf16(kRows, D, false, true);        // dq = dSq K   (K as MN-major B)
       constexpr uint32_t idKV = tc::idesc_bf16(kRows, kChunk, true, true);    // dV^T, dK^T  (both MN-major)
-      // head-dim operands of M = 128: the second 64-block sits one tile block
-      // further; with D = 64 it repeats the first (rows 64..127 are unused)
-      constexpr uint32_t kMnQ = D == 128 ? (uint32_t)kRows * 128 : 0u;
+      // head-dim operands of M = 128 from the grouped Q / dO tiles: the second
+      // 64-block of a group sits 1024 bytes further, 8-row groups 16 * D apart;
+      // with D = 64 it repeats the first block (rows 64..127 are unused)
+      constexpr uint32_t kMnQ = D == 128 ? 1024u : 0u;
+      constexpr uint32_t kGrp = 16 * D;
       constexpr uint32_t kMnK = (uint32_t)kChunk * 128;
       const uint32_t kbase = smem_u32(sm.K), vbase = smem_u32(sm.V);
       const uint32_t pbase = smem_u32(sm.P), dsq = smem_u32(sm.dSq), dsk = smem_u32(sm.dSk);
@@ -287,11 +292,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t blk = kk >> 2, wq = kk & 3;
-          const uint32_t ao = blk * kRows * 128 + wq * 32, bo = blk * kChunk * 128 + wq * 32;
-          tc::mma_bf16_ss(tmem + Cols<D>::S + sb * kChunk, tc::sdesc_sw128(qb + ao), tc::sdesc_sw128(kbase + bo),
-                          idSP, kk > 0);
-          tc::mma_bf16_ss(tmem + Cols<D>::dP + sb * kChunk, tc::sdesc_sw128(ob + ao), tc::sdesc_sw128(vbase + bo),
-                          idSP, kk > 0);
+          const uint32_t ao = blk * 1024 + wq * 32, bo = blk * kChunk * 128 + wq * 32;
+          tc::mma_bf16_ss(tmem + Cols<D>::S + sb * kChunk, tc::sdesc_sw128_sbo(qb + ao, kGrp),
+                          tc::sdesc_sw128(kbase + bo), idSP, kk > 0);
+          tc::mma_bf16_ss(tmem + Cols<D>::dP + sb * kChunk, tc::sdesc_sw128_sbo(ob + ao, kGrp),
+                          tc::sdesc_sw128(vbase + bo), idSP, kk > 0);
         }
         tc::mma_commit(bar(BAR_S_FULL + sb));
       };
@@ -309,9 +314,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < kRows / 16; ++kk) {
           const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
-          tc::mma_bf16_ss(tmem + Cols<D>::dVt, tc::sdesc_sw128_mn(ob + kk * 2048, kMnQ),
+          tc::mma_bf16_ss(tmem + Cols<D>::dVt, tc::sdesc_sw128_mn(ob + kk * 2 * kGrp, kMnQ, kGrp),
                           tc::sdesc_sw128_mn(pbase + kk * 2048, 0), idKV, acc);
-          tc::mma_bf16_ss(tmem + Cols<D>::dKt, tc::sdesc_sw128_mn(qb + kk * 2048, kMnQ),
+          tc::mma_bf16_ss(tmem + Cols<D>::dKt, tc::sdesc_sw128_mn(qb + kk * 2 * kGrp, kMnQ, kGrp),
                           tc::sdesc_sw128_mn(dsk + kk * 2048, 0), idKV, acc);
         }
         tc::mma_commit(bar(BAR_QD_EMPTY + st));
@@ -604,8 +609,8 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     memset(&tdo, 0, sizeof(tdo));
     a.n_rows = Dm.B * Dm.L * Dm.Hq;
     a.use_tma = Dm.G >= 8 ? 1 : 0;
-    if (a.use_tma && (!tc::make_rows_tmap(&tq, q, (unsigned long long)a.n_rows, D, Dm.G) ||
-                      !tc::make_rows_tmap(&tdo, dO, (unsigned long long)a.n_rows, D, Dm.G)))
+    if (a.use_tma && (!tc::make_group8_tmap(&tq, q, (unsigned long long)a.n_rows, D) ||
+                      !tc::make_group8_tmap(&tdo, dO, (unsigned long long)a.n_rows, D)))
       return cudaErrorNotSupported;
     bwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq, tdo);
     note_launches(1);

@@ -195,10 +195,10 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t addr) {
 // K) and the next 64 M/N elements start `mn_block_bytes` further on. A
 // K-major tile [k-row][64 columns] read this way is its own transpose, so
 // the same shared tile serves both operand orientations.
-__device__ __forceinline__ uint64_t sdesc_sw128_mn(uint32_t addr, uint32_t mn_block_bytes) {
+__device__ __forceinline__ uint64_t sdesc_sw128_mn(uint32_t addr, uint32_t mn_block_bytes, uint32_t k8_bytes = 1024) {
   return (uint64_t)((addr & 0x3FFFFu) >> 4)                     // start address
          | ((uint64_t)((mn_block_bytes >> 4) & 0x3FFFu) << 16)  // leading byte offset: next 64 M/N elements
-         | ((uint64_t)(1024 >> 4) << 32)                        // stride byte offset: next 8 K-rows
+         | ((uint64_t)((k8_bytes >> 4) & 0x3FFFu) << 32)        // stride byte offset: next 8 K-rows
          | ((uint64_t)1 << 46)                                  // descriptor version
          | ((uint64_t)2 << 61);                                 // 128-byte swizzle
 }

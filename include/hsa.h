@@ -197,6 +197,38 @@ hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const vo
                         const float* kbar32, void* O, int32_t* idx, float* s_sel, float* w, void* ws,
                         size_t ws_bytes, cudaStream_t stream);
 
+/*
+ * Decode index of a resident memory, built once per memory and reused by
+ * every hsa_decode_indexed call (§3.2 "Inference": the chunk summaries are
+ * what each decoding step scans). It holds the summaries rounded to bf16 in
+ * [Hkv][n_chunks][d] order, |K̄_i| per chunk and its maximum over every 64
+ * chunks. Size from hsa_decode_index_size (0 when topk > 16 or n_chunks = 0:
+ * hsa_decode_indexed then needs no index). Only shape's Hkv, d, n_chunks and
+ * topk matter; Bq may be 0.
+ *   kbar32 [n_chunks, Hkv, d] fp32 (hsa_chunk_pool of the memory, B = 1).
+ *   index  device memory, caller-owned, 16-byte aligned.
+ */
+size_t hsa_decode_index_size(const hsa_decode_shape_t* shape);
+hsa_status_t hsa_decode_index(const hsa_decode_shape_t* shape, const float* kbar32, void* index, size_t index_bytes,
+                              cudaStream_t stream);
+
+/* Workspace bytes of hsa_decode_indexed for `shape`. */
+size_t hsa_decode_indexed_workspace_size(const hsa_decode_shape_t* shape);
+
+/*
+ * hsa_decode with the memory index: same arguments and results (idx and s_sel
+ * identical, O and w to fp32 rounding), with the scan of the summaries on the
+ * tensor cores. Blocks over ranges of the memory score bf16 summaries against
+ * the group query; per query and range, the scores' rounding error is bounded
+ * (|error| < 2^-7 |q̂| |K̄_i|), so only the chunks that bound cannot rule out
+ * are kept, and those are rescored with the fp32 chain of hsa_select_topk
+ * before the top-k is taken. For topk > 16 it falls back to hsa_decode's scan
+ * (index may then be NULL).
+ */
+hsa_status_t hsa_decode_indexed(const hsa_decode_shape_t* shape, const void* q, const void* K_mem, const void* V_mem,
+                                const float* kbar32, const void* index, void* O, int32_t* idx, float* s_sel, float* w,
+                                void* ws, size_t ws_bytes, cudaStream_t stream);
+
 /* Size of the scratch array behind hsa_decode_noalloc (one per device): 8 MiB. */
 #define HSA_DECODE_NOALLOC_SCRATCH_BYTES (8u << 20)
 

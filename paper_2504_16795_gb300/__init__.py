@@ -18,6 +18,8 @@ from .binding import (  # noqa: F401
     build_index,
     chunk_pool,
     decode,
+    decode_index,
+    decode_indexed,
     decode_noalloc,
     decode_workspace_size,
     device_check,

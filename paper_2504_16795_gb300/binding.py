@@ -115,8 +115,14 @@ def load():
     L.hsa_backward.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     L.hsa_decode.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     L.hsa_decode_noalloc.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+    L.hsa_decode_index_size.restype = sz
+    L.hsa_decode_index_size.argtypes = [dp]
+    L.hsa_decode_index.argtypes = [dp, vp, vp, sz, vp]
+    L.hsa_decode_indexed_workspace_size.restype = sz
+    L.hsa_decode_indexed_workspace_size.argtypes = [dp]
+    L.hsa_decode_indexed.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     for f in (L.hsa_chunk_pool, L.hsa_select_topk, L.hsa_build_index, L.hsa_forward, L.hsa_backward,
-              L.hsa_decode, L.hsa_decode_noalloc):
+              L.hsa_decode, L.hsa_decode_noalloc, L.hsa_decode_index, L.hsa_decode_indexed):
         f.restype = i
     _lib = L
     return L
@@ -281,6 +287,36 @@ def decode_noalloc(shape: DecodeShape, q, K_mem, V_mem, kbar32, O, idx, s_sel, w
     s = shape.c()
     _check(load().hsa_decode_noalloc(ctypes.byref(s), _ptr(q), _ptr(K_mem), _ptr(V_mem), _ptr(kbar32), _ptr(O),
                                      _ptr(idx), _ptr(s_sel), _ptr(w), _stream(q.device)), "hsa_decode_noalloc")
+    return O, idx, s_sel, w
+
+
+def decode_index(shape: DecodeShape, kbar32, index=None):
+    """The memory index of hsa_decode_indexed (built once per memory); None when not needed."""
+    s = shape.c()
+    nb = int(load().hsa_decode_index_size(ctypes.byref(s)))
+    if nb == 0:
+        return None
+    dev = kbar32.device
+    index = torch.empty(nb, dtype=torch.uint8, device=dev) if index is None else index
+    _check(load().hsa_decode_index(ctypes.byref(s), _ptr(kbar32), _ptr(index), nb, _stream(dev)), "hsa_decode_index")
+    return index
+
+
+def decode_indexed(shape: DecodeShape, q, K_mem, V_mem, kbar32, index, O=None, idx=None, s_sel=None, w=None,
+                   ws=None):
+    _need(q, "q", torch.bfloat16, (shape.Bq, shape.Hq, shape.d))
+    dev = q.device
+    O = torch.empty_like(q) if O is None else O
+    out = (shape.Bq, shape.Hkv, shape.topk)
+    idx = torch.empty(out, dtype=torch.int32, device=dev) if idx is None else idx
+    s_sel = torch.empty(out, dtype=torch.float32, device=dev) if s_sel is None else s_sel
+    w = torch.empty(out, dtype=torch.float32, device=dev) if w is None else w
+    s = shape.c()
+    nb = int(load().hsa_decode_indexed_workspace_size(ctypes.byref(s)))
+    wsp = _workspace(nb, dev, ws)
+    _check(load().hsa_decode_indexed(ctypes.byref(s), _ptr(q), _ptr(K_mem), _ptr(V_mem), _ptr(kbar32), _ptr(index),
+                                     _ptr(O), _ptr(idx), _ptr(s_sel), _ptr(w), _ptr(wsp), nb, _stream(dev)),
+           "hsa_decode_indexed")
     return O, idx, s_sel, w
 
 

@@ -256,6 +256,58 @@ hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const vo
   return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, ws, stream));
 }
 
+size_t hsa_decode_index_size(const hsa_decode_shape_t* shape) {
+  hsa::DecodeDims D;
+  if (resolve_decode(shape, &D) != HSA_OK || !hsa::decode_tc_applies(D)) return 0;
+  return hsa::decode_index_bytes(D);
+}
+
+hsa_status_t hsa_decode_index(const hsa_decode_shape_t* shape, const float* kbar32, void* index, size_t index_bytes,
+                              cudaStream_t stream) {
+  hsa::DecodeDims D;
+  hsa_status_t st = resolve_decode(shape, &D);
+  if (st != HSA_OK) return st;
+  if (!hsa::decode_tc_applies(D)) return D.Nc == 0 ? HSA_OK : HSA_ERR_UNSUPPORTED;
+  HSA_REQUIRE_PTR(kbar32);
+  const size_t need = hsa::decode_index_bytes(D);
+  if (index_bytes < need || index == nullptr || !aligned16(index)) return HSA_ERR_WORKSPACE;
+  return cuda_status(hsa::launch_decode_index(D, kbar32, index, stream));
+}
+
+size_t hsa_decode_indexed_workspace_size(const hsa_decode_shape_t* shape) {
+  hsa::DecodeDims D;
+  if (resolve_decode(shape, &D) != HSA_OK || D.Bq == 0) return 0;
+  return hsa::decode_tc_applies(D) ? hsa::decode_tc_workspace(D) : hsa::decode_workspace(D);
+}
+
+hsa_status_t hsa_decode_indexed(const hsa_decode_shape_t* shape, const void* q, const void* K_mem, const void* V_mem,
+                                const float* kbar32, const void* index, void* O, int32_t* idx, float* s_sel, float* w,
+                                void* ws, size_t ws_bytes, cudaStream_t stream) {
+  hsa::DecodeDims D;
+  hsa_status_t st = resolve_decode(shape, &D);
+  if (st != HSA_OK) return st;
+  if (D.Bq == 0) return HSA_OK;
+  HSA_REQUIRE_PTR(q);
+  HSA_REQUIRE_PTR(O);
+  HSA_REQUIRE_PTR(idx);
+  HSA_REQUIRE_PTR(s_sel);
+  HSA_REQUIRE_PTR(w);
+  if (D.Nc > 0) {
+    HSA_REQUIRE_PTR(K_mem);
+    HSA_REQUIRE_PTR(V_mem);
+    HSA_REQUIRE_PTR(kbar32);
+  }
+  if (!hsa::decode_tc_applies(D)) {  // k > 16 or an empty memory: the CUDA-core scan of hsa_decode
+    const size_t need = hsa::decode_workspace(D);
+    if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+    return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, ws, stream));
+  }
+  HSA_REQUIRE_PTR(index);
+  const size_t need = hsa::decode_tc_workspace(D);
+  if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+  return cuda_status(hsa::launch_decode_tc(D, q, K_mem, V_mem, kbar32, index, O, idx, s_sel, w, ws, stream));
+}
+
 }  // extern "C"
 
 hsa_status_t hsa::resolve_decode_shape(const hsa_decode_shape_t* s, hsa::DecodeDims* out) {

@@ -196,6 +196,17 @@ struct DecodeDims {
 size_t decode_workspace(const DecodeDims& D);
 cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
                           void* O, int32_t* idx, float* s_sel, float* w, void* ws, cudaStream_t st);
+// Token-level attention over the selected chunks and the weighted sum (the last two decode steps).
+cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void* K, const void* V,
+                                 const int32_t* idx, const float* w, void* O, float* opart, cudaStream_t st);
+// Decode over a memory index (bf16 summaries, norms): tensor-core scan with exact rescoring (topk <= 16).
+bool decode_tc_applies(const DecodeDims& D);
+size_t decode_index_bytes(const DecodeDims& D);
+cudaError_t launch_decode_index(const DecodeDims& D, const float* kbar32, void* index, cudaStream_t st);
+size_t decode_tc_workspace(const DecodeDims& D);
+cudaError_t launch_decode_tc(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
+                             const void* index, void* O, int32_t* idx, float* s_sel, float* w, void* ws,
+                             cudaStream_t st);
 // The decode shape check of hsa_decode, shared with the entry point that owns its scratch.
 hsa_status_t resolve_decode_shape(const hsa_decode_shape_t* s, DecodeDims* out);
 }  // namespace hsa

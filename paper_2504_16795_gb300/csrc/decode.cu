@@ -280,6 +280,33 @@ cudaError_t run(const DecodeDims& D, const void* q, const void* K, const void* V
 
 size_t decode_workspace(const DecodeDims& D) { return dec_layout(D).total; }
 
+cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void* K, const void* V,
+                                 const int32_t* idx, const float* w, void* O, float* opart, cudaStream_t st) {
+  const int rows = D.Bq * D.Hkv;
+  cudaError_t e;
+  if (D.d == 64) {
+    if ((e = cudaFuncSetAttribute(dec_attend_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)sizeof(AttSmem<64>))) != cudaSuccess)
+      return e;
+    dec_attend_kernel<64><<<rows * D.topk, kThreads, sizeof(AttSmem<64>), st>>>(
+        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk, D.scale_attn);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    dec_out_kernel<64><<<rows, 256, 0, st>>>(opart, w, (uint16_t*)O, D.G, D.topk);
+  } else {
+    if ((e = cudaFuncSetAttribute(dec_attend_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)sizeof(AttSmem<128>))) != cudaSuccess)
+      return e;
+    dec_attend_kernel<128><<<rows * D.topk, kThreads, sizeof(AttSmem<128>), st>>>(
+        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk, D.scale_attn);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    dec_out_kernel<128><<<rows, 256, 0, st>>>(opart, w, (uint16_t*)O, D.G, D.topk);
+  }
+  note_launches(1);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
                           void* O, int32_t* idx, float* s_sel, float* w, void* ws, cudaStream_t st) {
   return D.d == 64 ? run<64>(D, q, K, V, kbar32, O, idx, s_sel, w, ws, st)

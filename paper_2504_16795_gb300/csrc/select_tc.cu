@@ -7,15 +7,17 @@
 // The score matrix q̂ K̄^T is a dense contraction, so it runs as bf16 tcgen05
 // MMAs (q̂ and K̄ rounded to bf16, fp32 accumulation in tensor memory). A
 // bf16 score a_i differs from the exact dot product by less than
-//   eps_i = 2^-7 * |q̂| * |K̄_i|
-// (each bf16 rounding moves a factor by at most 2^-9 of itself, so the
-// product sum moves by at most about 2^-8 * sum|q̂_e||K̄_ie| <= 2^-8 |q̂||K̄_i|
-// by Cauchy-Schwarz; the fp32 accumulation errors of both sides are far
-// below the remaining factor of two). So l_i = a_i - eps_i and
-// u_i = a_i + eps_i bracket the exact score: if lambda is the k-th largest
-// lower bound, the exact k-th score is at least lambda, and a chunk with
-// u_i < lambda is strictly below it (with room to spare for the final
-// rounding by c_sel, so no tie can be created).
+//   eps_i = 2^-7 * (9/8) * |q̂| * |K̄_i|.
+// Rounding to bf16 (8 significant bits, to nearest) moves a factor by at
+// most 2^-8 of itself, so the exact product sum moves by at most
+// (2^-7 + 2^-16) * sum|q̂_e||K̄_ie|; the products of bf16 factors are exact in
+// fp32, and the fp32 sums of both sides (the tensor core's, allowed up to
+// 2^-12 relative, and the reference chain's, about 2^-17) add less than
+// 2^-11 of the same sum. Cauchy-Schwarz bounds the sum by |q̂||K̄_i|. So
+// l_i = a_i - eps_i and u_i = a_i + eps_i bracket the exact score: if lambda
+// is the k-th largest lower bound, the exact k-th score is at least lambda,
+// and a chunk with u_i < lambda is strictly below it, with margin enough
+// (2^-10 |q̂||K̄_i|) that the final rounding by c_sel cannot create a tie.
 //
 // Per block: 128 consecutive tokens of one (b, g) against tiles of 64 chunk
 // summaries, in two passes over the tiles (the MMAs run twice). Thread r of
@@ -27,7 +29,9 @@
 //   buffer (typically k plus a few); it holds every chunk whose lower bound
 //   reaches lambda, so lambda is the k-th largest lower bound in the buffer.
 // The buffer entries whose upper bound reaches lambda are rescored exactly in
-// fp32 and the top k emitted. A row whose buffer overflows is handed to an
+// fp32 and the top k emitted. A full buffer keeps the entries with the
+// largest upper bounds and remembers the largest upper bound it dropped; a
+// row is certified when that value is below its lambda, and otherwise handed to an
 // exact warp-per-row pass. The L x (L/S) score matrix never leaves the chip.
 #include <algorithm>
 #include <cstring>
@@ -40,7 +44,7 @@ namespace {
 constexpr int kTok = 128;      // token rows per block (MMA M, tensor-memory lanes)
 constexpr int kCt = 64;        // chunk summaries per tile (MMA N)
 constexpr int kThreads = 192;  // warps 0-3 scan (thread = row), 4 loader, 5 MMA
-constexpr float kEpsRel = 1.f / 128.f;
+constexpr float kEpsRel = 9.f / 1024.f;  // 2^-7 * 9/8
 // Absolute floor of eps_i: covers products the tensor core may flush to zero
 // (operands below the normal range), far below any score it could reorder.
 constexpr float kEpsAbs = 1e-25f;
@@ -92,6 +96,15 @@ struct SelTcArgs {
   int32_t* flags;
   int L, Lp, Hkv, Nc, Ncp, topk, n_qt, BH;
   float scale_sel;
+  // decode against a resident memory: rows are query tokens (all chunks
+  // visible); block (split, g, query tile) scans chunks [split*range, +range)
+  // and exports, per row, the chunks whose upper bound reaches its own lambda
+  int Bq, n_split, range;
+  float* cand_l;   // [Hkv, Bq, n_split, kBuf] lower bounds
+  float* cand_u;   //                          upper bounds
+  int32_t* cand_c; //                          chunk indices
+  int32_t* cand_n; // [Hkv, Bq, n_split] entry count
+  float* cand_d;   // [Hkv, Bq, n_split] largest upper bound the row's buffer dropped (-inf: none)
 };
 
 // x[c] for a run-time c in [0, 32): a five-level select tree.
@@ -108,7 +121,7 @@ __device__ __forceinline__ float pick32(const float (&x)[32], int c) {
   return (c & 16) ? t[1] : t[0];
 }
 
-template <int D, int KT>
+template <int D, int KT, bool DEC>
 __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     sel_tc_kernel(SelTcArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                   const __grid_constant__ CUtensorMap tmap_q32t) {
@@ -119,16 +132,24 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
                 BAR_ACC_FULL = Smem::BAR_ACC_FULL, BAR_ACC_EMPTY = Smem::BAR_ACC_EMPTY, BAR_KN = Smem::BAR_KN;
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int qt = a.n_qt - 1 - (int)(blockIdx.x / a.BH);  // late (heavy) token tiles first
-  const int bg = (int)(blockIdx.x % a.BH);
+  int qt, bg, split = 0, c_begin = 0, vis_max;
+  if constexpr (DEC) {
+    split = (int)blockIdx.x;
+    bg = (int)blockIdx.y;  // the memory has one batch row: bg = g
+    qt = (int)blockIdx.z;
+    c_begin = split * a.range;
+    vis_max = max(min(c_begin + a.range, a.Nc) - c_begin, 0);
+  } else {
+    qt = a.n_qt - 1 - (int)(blockIdx.x / a.BH);  // late (heavy) token tiles first
+    bg = (int)(blockIdx.x % a.BH);
+    vis_max = min((min(qt * kTok + kTok, a.L) - 1) / kChunk, a.Nc);
+  }
   const int b = bg / a.Hkv, g = bg % a.Hkv;
   const int t0 = qt * kTok;
-  const int t_last = min(t0 + kTok, a.L) - 1;
-  const int vis_max = min(t_last / kChunk, a.Nc);
   const int ntiles = (vis_max + kCt - 1) / kCt;
-  // Blocks start their sweep at different tiles, so that concurrent blocks of
-  // one (b, g) do not all request the same chunk-summary lines at once.
-  const int rot = ntiles > 0 ? (int)(blockIdx.x % (unsigned)ntiles) : 0;
+  // Prefill blocks start their sweep at different tiles, so that concurrent
+  // blocks of one (b, g) do not all request the same summary lines at once.
+  const int rot = (!DEC && ntiles > 0) ? (int)(blockIdx.x % (unsigned)ntiles) : 0;
   auto tile_of = [&](int it) {
     const int j = it < ntiles ? it : it - ntiles;
     return j + rot < ntiles ? j + rot : j + rot - ntiles;
@@ -166,7 +187,8 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       tc::mbar_arrive_expect_tx(bar(BAR_A), kTok * D * 2);
 #pragma unroll
       for (int kb = 0; kb < D / 64; ++kb)
-        tc::tma_load_2d(abase + kb * kTok * 128, &tmap_q, kb * 64, bg * a.L + t0, bar(BAR_A));
+        tc::tma_load_2d(abase + kb * kTok * 128, &tmap_q, kb * 64, DEC ? (g * a.n_qt + qt) * kTok : bg * a.L + t0,
+                        bar(BAR_A));
       for (int it = 0; it < 2 * ntiles; ++it) {  // two passes over the tiles
         const int n = tile_of(it);
         const int s = it % kStages;
@@ -174,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
         tc::mbar_arrive_expect_tx(bar(BAR_FULL + s), kStageBytes);
 #pragma unroll
         for (int kb = 0; kb < D / 64; ++kb)
-          tc::tma_load_2d(ubase + s * kStageBytes + kb * kCt * 128, &tmap_k, kb * 64, bg * a.Nc + n * kCt,
+          tc::tma_load_2d(ubase + s * kStageBytes + kb * kCt * 128, &tmap_k, kb * 64, bg * a.Nc + c_begin + n * kCt,
                           bar(BAR_FULL + s));
       }
     }
@@ -192,9 +214,10 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
         tc::fence_after_sync();
         // the tile's chunk norms travel with its accumulator (the scan has released both)
         tc::mbar_arrive_expect_tx(bar(BAR_KN + ab), (kCt + 4) * 4);
-        tc::bulk_load(smem_u32(sm.knt[ab]), a.kn + (long long)bg * a.Ncp + n * kCt, kCt * 4, bar(BAR_KN + ab));
-        tc::bulk_load(smem_u32(&sm.knt[ab][kCt]), a.ktmax + ((long long)bg * (a.Ncp / kCt) + n) * 4, 16,
+        tc::bulk_load(smem_u32(sm.knt[ab]), a.kn + (long long)bg * a.Ncp + c_begin + n * kCt, kCt * 4,
                       bar(BAR_KN + ab));
+        tc::bulk_load(smem_u32(&sm.knt[ab][kCt]),
+                      a.ktmax + ((long long)bg * (a.Ncp / kCt) + c_begin / kCt + n) * 4, 16, bar(BAR_KN + ab));
         const uint32_t bbase = ubase + s * kStageBytes;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
@@ -211,15 +234,16 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     // ---------------------------------------------------------------- scan (thread = token row)
     const int r = tid;
     const int t = t0 + r;
-    const int vis = t < a.L ? min(t / kChunk, a.Nc) : 0;
+    const bool row_ok = DEC ? t < a.Bq : t < a.L;
+    const int vis = !row_ok ? 0 : (DEC ? vis_max : min(t / kChunk, a.Nc));
     constexpr int kBuf = Smem::kBuf;
-    const long long qrow = (long long)bg * a.L + t;
+    const long long qrow = DEC ? (long long)t * a.Hkv + g : (long long)bg * a.L + t;
     const float cq = vis > 0 ? kEpsRel * a.qn[qrow] : 0.f;  // eps_i = cq * |K̄_i| + kEpsAbs
     // First pass: the k-th largest of (max over a group of columns - the
     // tile's largest eps) is a lower bound of lambda, since each group holds a
     // chunk whose lower bound is at least its term. Groups of 32 or 8 columns,
     // or single columns for short rows, keep at least 2k terms per row.
-    const int vis0 = min(t0 / kChunk, a.Nc);
+    const int vis0 = DEC ? vis_max : min(t0 / kChunk, a.Nc);
     const int gsz = vis0 >= 64 * a.topk ? 32 : (vis0 >= 16 * a.topk ? 8 : 1);
     float bm[KT];  // slots [KT-k, KT): the k largest terms (descending); +inf above
 #pragma unroll
@@ -234,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     };
     float lam_lo = -INFINITY;
     int cnt = 0;  // second-pass entries
-    bool overflow = false;
+    float u_drop = -INFINITY;  // largest upper bound a full buffer dropped
 
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
     for (int it = 0; it < 2 * ntiles; ++it) {
@@ -291,12 +315,29 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
             const float xc = pick32(x, c);
             const float e = fmaf(cq, knt[h * 32 + c], kEpsAbs);
             if (xc + e >= lam_lo) {
+              const float lv = xc - e, uv = xc + e;
+              int slot = cnt;
               if (cnt < kBuf) {
-                sm.bl[cnt][r] = xc - e;
-                sm.bu[cnt][r] = xc + e;
-                sm.bi[cnt][r] = c0 + c;
+                ++cnt;
+              } else {  // full: replace the entry with the smallest upper bound, if smaller
+                float um = sm.bu[0][r];
+                slot = 0;
+                for (int j = 1; j < kBuf; ++j) {
+                  const float uj = sm.bu[j][r];
+                  if (uj < um) um = uj, slot = j;
+                }
+                if (uv > um) {
+                  u_drop = fmaxf(u_drop, um);
+                } else {
+                  u_drop = fmaxf(u_drop, uv);
+                  slot = -1;
+                }
               }
-              ++cnt;
+              if (slot >= 0) {
+                sm.bl[slot][r] = lv;
+                sm.bu[slot][r] = uv;
+                sm.bi[slot][r] = c_begin + c0 + c;
+              }
             }
           }
         }
@@ -304,8 +345,33 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_ACC_EMPTY + ab));
     }
-    if (cnt > kBuf) overflow = true;
     if (ntiles == 0) cnt = 0;
+    // lambda of the kept entries: at most the row's true lambda (a subset's k-th largest)
+#pragma unroll
+    for (int i = 0; i < KT; ++i) bm[i] = i < KT - a.topk ? INFINITY : -INFINITY;
+    for (int j = 0; j < cnt; ++j) push(sm.bl[j][r]);
+    const float lam_keep = bm[KT - 1];
+
+    if constexpr (DEC) {
+      // export the entries whose upper bound reaches this range's lambda, and
+      // the largest upper bound the buffer dropped (the merge checks it against
+      // the lambda of the whole memory)
+      if (row_ok && !*abort_flag) {
+        const long long crow = ((long long)g * a.Bq + t) * a.n_split + split;
+        int ne = 0;
+        for (int j = 0; j < cnt; ++j) {
+          const float u = sm.bu[j][r];
+          if (u >= lam_keep) {
+            a.cand_l[crow * kBuf + ne] = sm.bl[j][r];
+            a.cand_u[crow * kBuf + ne] = u;
+            a.cand_c[crow * kBuf + ne] = sm.bi[j][r];
+            ++ne;
+          }
+        }
+        a.cand_n[crow] = ne;
+        a.cand_d[crow] = u_drop;
+      }
+    } else {
 
     // ---------------------------------------------------------------- exact rescoring of the candidates
     // Every MMA has completed once the last accumulator was seen, so A and B
@@ -314,18 +380,15 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       tc::mbar_arrive_expect_tx(bar(BAR_Q32), kTok * D * 4);
       tc::tma_load_2d(abase, &tmap_q32t, t0, bg * D, bar(BAR_Q32));
     }
-    // lambda itself: the k-th largest lower bound among the entries (they
-    // include every chunk whose lower bound reaches lam_lo); the candidates
-    // are the entries whose upper bound reaches it
+    // lambda: the k-th largest lower bound among the kept entries (they
+    // include every chunk whose lower bound reaches lam_lo, unless the buffer
+    // dropped entries, whose upper bounds must then stay below it); the
+    // candidates are the entries whose upper bound reaches it
+    const bool overflow = u_drop > -INFINITY && !(u_drop < lam_keep);
     int nc = 0;
-    if (!overflow) {
-#pragma unroll
-      for (int i = 0; i < KT; ++i) bm[i] = i < KT - a.topk ? INFINITY : -INFINITY;
-      for (int j = 0; j < cnt; ++j) push(sm.bl[j][r]);
-      const float lam = bm[KT - 1];
+    if (!overflow)
       for (int j = 0; j < cnt; ++j)
-        if (sm.bu[j][r] >= lam) sm.bi[nc++][r] = sm.bi[j][r];
-    }
+        if (sm.bu[j][r] >= lam_keep) sm.bi[nc++][r] = sm.bi[j][r];
     const bool q_ok = ntiles == 0 || tc::mbar_wait(bar(BAR_Q32), 0, abort_flag, status);
     if (t < a.L && q_ok && !*abort_flag) {
       const long long p = ((long long)b * a.L + t) * a.Hkv + g;
@@ -386,6 +449,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
         }
       }
     }
+    }  // prefill
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -536,6 +600,200 @@ __global__ void __launch_bounds__(256) sel_exact_rows_kernel(const float* __rest
   }
 }
 
+// Decode queries: q̂ in fp32 ([Bq * Hkv, D], head order), in bf16 as the MMA
+// operand ([Hkv, n_qt * 128, D], rows past Bq zero) and its norm. Threads
+// D/8 per row.
+template <int D>
+__global__ void __launch_bounds__(256) dtc_qhat_kernel(const uint16_t* __restrict__ q, float* __restrict__ qh32,
+                                                       uint16_t* __restrict__ qh16, float* __restrict__ qn, int Bq,
+                                                       int Hq, int Hkv, int G, int n_qt) {
+  constexpr int D8 = D / 8;
+  const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const long long row = u / D8;  // g * n_qt * 128 + b
+  const int e8 = (int)(u % D8);
+  const long long rows = (long long)Hkv * n_qt * kTok;
+  const int g = (int)(row / ((long long)n_qt * kTok));
+  const int b = (int)(row % ((long long)n_qt * kTok));
+  const bool in = row < rows;
+  const bool valid = in && b < Bq;
+  float acc[8];
+#pragma unroll
+  for (int c = 0; c < 8; ++c) acc[c] = 0.f;
+  if (valid) {
+    const uint4* src = reinterpret_cast<const uint4*>(q + ((long long)b * Hq + (long long)g * G) * D) + e8;
+    for (int hh = 0; hh < G; ++hh) {
+      const uint4 w = __ldg(src + (long long)hh * D8);
+      acc[0] = acc[0] + bf16_lo(w.x);
+      acc[1] = acc[1] + bf16_hi(w.x);
+      acc[2] = acc[2] + bf16_lo(w.y);
+      acc[3] = acc[3] + bf16_hi(w.y);
+      acc[4] = acc[4] + bf16_lo(w.z);
+      acc[5] = acc[5] + bf16_hi(w.z);
+      acc[6] = acc[6] + bf16_lo(w.w);
+      acc[7] = acc[7] + bf16_hi(w.w);
+    }
+    float4* d32 = reinterpret_cast<float4*>(qh32 + ((long long)b * Hkv + g) * D + e8 * 8);
+    d32[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    d32[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+  }
+  if (in)
+    *reinterpret_cast<uint4*>(qh16 + row * D + e8 * 8) =
+        make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]), pack_bf16x2(acc[4], acc[5]),
+                   pack_bf16x2(acc[6], acc[7]));
+  float ss = 0.f;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) ss = fmaf(acc[c], acc[c], ss);
+#pragma unroll
+  for (int o = D8 / 2; o > 0; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
+  if (valid && e8 == 0) qn[(long long)b * Hkv + g] = sqrtf(ss);
+}
+
+// Exact score chain of one chunk summary (dot product in dimension order, from 0).
+template <int D>
+__device__ __forceinline__ float exact_dot(const float* __restrict__ qs, const float* __restrict__ krow) {
+  const float4* k4 = reinterpret_cast<const float4*>(krow);
+  float acc = 0.f;
+#pragma unroll 8
+  for (int e4 = 0; e4 < D / 4; ++e4) {
+    const float4 kv = __ldg(k4 + e4);
+    acc = fmaf(qs[4 * e4], kv.x, acc);
+    acc = fmaf(qs[4 * e4 + 1], kv.y, acc);
+    acc = fmaf(qs[4 * e4 + 2], kv.z, acc);
+    acc = fmaf(qs[4 * e4 + 3], kv.w, acc);
+  }
+  return acc;
+}
+
+// Decode merge: one block (8 warps) per (query, group). lambda = the k-th
+// largest lower bound over the entries every scan block exported, at most the
+// true lambda. A block whose buffer dropped an entry with upper bound at or
+// above lambda cannot vouch for its range: those ranges are scored exactly
+// (rare). The candidates (entries with upper bound at or above lambda, and
+// the exactly scored chunks at or above it) are ranked by the exact chain,
+// (score desc, chunk index asc). Each warp keeps a top-k list over its share;
+// warp 0 combines the eight.
+template <int D>
+__global__ void __launch_bounds__(256) dtc_merge_kernel(const float* __restrict__ cand_l,
+                                                        const float* __restrict__ cand_u,
+                                                        const int32_t* __restrict__ cand_c,
+                                                        const int32_t* __restrict__ cand_n,
+                                                        const float* __restrict__ cand_d, int kbuf,
+                                                        const float* __restrict__ qh32,
+                                                        const float* __restrict__ kbar32, int32_t* __restrict__ idx,
+                                                        float* __restrict__ s_sel, float* __restrict__ w, int Bq,
+                                                        int Hkv, int Nc, int n_split, int range, int topk,
+                                                        float scale_sel) {
+  __shared__ float qs[D];
+  __shared__ unsigned long long lists[8][32];
+  __shared__ float lam_s;
+  __shared__ int any_unsure;
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  const int row = blockIdx.x;  // b * Hkv + g
+  const int b = row / Hkv, g = row % Hkv;
+  const long long cbase = ((long long)g * Bq + b) * n_split;
+  if (threadIdx.x == 0) any_unsure = 0;
+  for (int e = threadIdx.x; e < D; e += 256) qs[e] = qh32[(long long)row * D + e];
+  __syncthreads();
+  const long long total = (long long)n_split * kbuf;  // entry slots of the row
+  auto krow = [&](int c) { return kbar32 + ((long long)c * Hkv + g) * D; };
+  auto combine = [&](unsigned long long mine) {  // top-k of the eight warp lists, in warp 0
+    lists[wib][lane] = mine;
+    __syncthreads();
+    unsigned long long all = 0ull;
+    if (wib == 0)
+      for (int k = 0; k < 8; ++k) warp_topk_offer(all, lane < topk ? lists[k][lane] : 0ull, topk, lane);
+    __syncthreads();
+    return all;
+  };
+  // ---- lambda: every warp walks slots wib*32 + lane, step 256, four batches
+  // at a time (loads first, then the list updates)
+  unsigned long long lst = 0ull;
+  for (long long base = (long long)wib * 32; base < total; base += 4 * 256) {
+    float lv[4];
+    bool ok[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const long long slot = base + u * 256 + lane;
+      ok[u] = slot < total && cand_n[cbase + slot / kbuf] > (int)(slot % kbuf);
+      lv[u] = ok[u] ? cand_l[cbase * kbuf + slot] : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const long long slot = base + u * 256 + lane;
+      const unsigned long long key = ok[u] ? ((unsigned long long)order_bits(lv[u]) << 32) | (uint32_t)slot : 0ull;
+      warp_topk_offer(lst, key, topk, lane);
+    }
+  }
+  {
+    const unsigned long long all = combine(lst);
+    if (wib == 0) {
+      const unsigned long long kth = __shfl_sync(0xFFFFFFFFu, all, topk - 1);
+      if (lane == 0) lam_s = kth != 0ull ? order_bits_to_float((uint32_t)(kth >> 32)) : -INFINITY;
+    }
+    __syncthreads();
+  }
+  const float lam = lam_s;
+  for (int sp = threadIdx.x; sp < n_split; sp += 256)
+    if (cand_d[cbase + sp] >= lam) any_unsure = 1;
+  __syncthreads();
+  const bool unsure = any_unsure != 0;
+  // ---- the candidates, exactly
+  unsigned long long fin = 0ull;
+  for (long long base = (long long)wib * 32; base < total; base += 4 * 256) {
+    float uv[4];
+    bool ok[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const long long slot = base + u * 256 + lane;
+      ok[u] = slot < total && cand_n[cbase + slot / kbuf] > (int)(slot % kbuf);
+      uv[u] = ok[u] ? cand_u[cbase * kbuf + slot] : -INFINITY;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const long long slot = base + u * 256 + lane;
+      unsigned long long key = 0ull;
+      if (ok[u] && uv[u] >= lam) {
+        const int c = cand_c[cbase * kbuf + slot];
+        key = rank_key(exact_dot<D>(qs, krow(c)) * scale_sel, (uint32_t)c);
+      }
+      warp_topk_offer(fin, key, topk, lane);
+    }
+  }
+  for (int sp = 0; unsure && sp < n_split; ++sp) {
+    if (!(cand_d[cbase + sp] >= lam)) continue;  // uniform across the block
+    // this range's exported entries are scored again below the whole range:
+    // skip them there to keep every chunk once
+    const int cb = sp * range, ce = min(cb + range, Nc);
+    const int n = cand_n[cbase + sp];
+    for (int c0 = cb + wib * 32; c0 < ce; c0 += 256) {
+      const int c = c0 + lane;
+      unsigned long long key = 0ull;
+      if (c < ce) {
+        bool exported = false;
+        for (int j = 0; j < n; ++j) exported |= cand_c[(cbase + sp) * kbuf + j] == c && cand_u[(cbase + sp) * kbuf + j] >= lam;
+        const float dot = exact_dot<D>(qs, krow(c));
+        if (!exported && dot >= lam) key = rank_key(dot * scale_sel, (uint32_t)c);
+      }
+      warp_topk_offer(fin, key, topk, lane);
+    }
+  }
+  const unsigned long long all = combine(fin);
+  if (wib != 0) return;
+  const long long o = (long long)row * topk;
+  warp_emit_selection(all, topk, lane, idx + o, s_sel + o);
+  __syncwarp();
+  bool valid = false;
+  float sv = -INFINITY;
+  if (lane < topk) {
+    valid = idx[o + lane] >= 0;
+    if (valid) sv = s_sel[o + lane];
+  }
+  const float m = warp_max(sv);
+  const float ex = valid ? expf(sv - m) : 0.f;
+  const float z = warp_sum(ex);
+  if (lane < topk) w[o + lane] = valid ? ex / z : 0.f;
+}
+
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 struct SelLayout {
@@ -614,7 +872,7 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   if (!tc::make_plain_tmap_f32(&tq32t, qh32, (unsigned long long)BH * DD, Lp, kTok, DD)) return cudaErrorNotSupported;
   if (!tc::make_rows_tmap(&tq, qh16, (unsigned long long)q_rows(Dm), DD, kTok)) return cudaErrorNotSupported;
   if (!tc::make_rows_tmap(&tk, kb16, (unsigned long long)k_rows(Dm), DD, kCt)) return cudaErrorNotSupported;
-  SelTcArgs a;
+  SelTcArgs a{};
   a.qh32t = qh32;
   a.qn = qn;
   a.kbar32 = kbar32;
@@ -634,11 +892,11 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   a.BH = BH;
   a.scale_sel = Dm.scale_sel;
   const size_t smem = sizeof(SelTcSmem<DD, KT>) + 1024;
-  if ((e = cudaFuncSetAttribute(sel_tc_kernel<DD, KT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
-      cudaSuccess)
+  if ((e = cudaFuncSetAttribute(sel_tc_kernel<DD, KT, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)smem)) != cudaSuccess)
     return e;
   const long long blocks = (long long)a.n_qt * BH;
-  sel_tc_kernel<DD, KT><<<(unsigned)blocks, kThreads, smem, st>>>(a, tq, tk, tq32t);
+  sel_tc_kernel<DD, KT, false><<<(unsigned)blocks, kThreads, smem, st>>>(a, tq, tk, tq32t);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   sel_exact_rows_kernel<DD><<<2 * 152, 256, 0, st>>>(qh32, kbar32, nflag, flags, idx, s_sel, Dm.L, Lp, Dm.Hkv,
@@ -648,6 +906,170 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
 }
 
 }  // namespace
+
+// ---------------------------------------------------------------- decode against a resident memory
+namespace {
+
+struct DecIndexLayout {
+  size_t kb16, kn, ktmax, total;
+};
+
+DecIndexLayout dec_index_layout(const DecodeDims& D) {
+  const size_t ncp = (size_t)((D.Nc + kCt - 1) / kCt * kCt);
+  const size_t krows = std::max<size_t>((size_t)D.Hkv * D.Nc, kCt);
+  DecIndexLayout lo{};
+  size_t o = 0;
+  lo.kb16 = o;
+  o = align256(o + krows * D.d * 2);
+  lo.kn = o;
+  o = align256(o + (size_t)D.Hkv * ncp * 4);
+  lo.ktmax = o;
+  o = align256(o + (size_t)D.Hkv * (ncp / kCt) * 16);
+  lo.total = o;
+  return lo;
+}
+
+struct DecTcLayout {
+  size_t qh32, qh16, qn, cl, cu, cc, cn, cd, opart, total;
+  int n_qt, n_split, range;
+};
+
+template <int KT>
+DecTcLayout dec_tc_layout(const DecodeDims& D) {
+  DecTcLayout lo{};
+  lo.n_qt = (D.Bq + kTok - 1) / kTok;
+  const long long want = (2LL * 152) / ((long long)D.Hkv * lo.n_qt);
+  lo.n_split = (int)std::max<long long>(1, std::min<long long>(want, (D.Nc + kCt - 1) / kCt));
+  const long long per = (D.Nc + lo.n_split - 1) / lo.n_split;
+  lo.range = (int)((per + kCt - 1) / kCt * kCt);
+  lo.n_split = (int)((D.Nc + lo.range - 1) / lo.range);
+  const size_t rows = (size_t)D.Bq * D.Hkv;
+  const size_t nc = rows * lo.n_split * SelCfg<KT>::kBuf;
+  size_t o = 0;
+  lo.qh32 = o;
+  o = align256(o + rows * D.d * 4);
+  lo.qh16 = o;
+  o = align256(o + (size_t)D.Hkv * lo.n_qt * kTok * D.d * 2);
+  lo.qn = o;
+  o = align256(o + rows * 4);
+  lo.cl = o;
+  o = align256(o + nc * 4);
+  lo.cu = o;
+  o = align256(o + nc * 4);
+  lo.cc = o;
+  o = align256(o + nc * 4);
+  lo.cn = o;
+  o = align256(o + rows * lo.n_split * 4);
+  lo.cd = o;
+  o = align256(o + rows * lo.n_split * 4);
+  lo.opart = o;
+  o = align256(o + rows * D.topk * D.G * D.d * 4);
+  lo.total = o;
+  return lo;
+}
+
+template <int DD, int KT>
+cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, const void* V, const float* kbar32,
+                          const void* index, void* O, int32_t* idx, float* s_sel, float* w, void* ws,
+                          cudaStream_t st) {
+  const DecTcLayout lo = dec_tc_layout<KT>(Dm);
+  const DecIndexLayout ix = dec_index_layout(Dm);
+  char* base = (char*)ws;
+  float* qh32 = (float*)(base + lo.qh32);
+  uint16_t* qh16 = (uint16_t*)(base + lo.qh16);
+  float* qn = (float*)(base + lo.qn);
+  const char* ib = (const char*)index;
+  cudaError_t e;
+  constexpr int D8 = DD / 8;
+  const long long qrows = (long long)Dm.Hkv * lo.n_qt * kTok;
+  dtc_qhat_kernel<DD><<<(unsigned)((qrows * D8 + 255) / 256), 256, 0, st>>>((const uint16_t*)q, qh32, qh16, qn, Dm.Bq,
+                                                                           Dm.Hq, Dm.Hkv, Dm.G, lo.n_qt);
+  note_launches(1);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  CUtensorMap tq, tk, unused;
+  memset(&tq, 0, sizeof(tq));
+  memset(&tk, 0, sizeof(tk));
+  memset(&unused, 0, sizeof(unused));
+  const unsigned long long krows = std::max<unsigned long long>((unsigned long long)Dm.Hkv * Dm.Nc, kCt);
+  if (!tc::make_rows_tmap(&tq, qh16, (unsigned long long)qrows, DD, kTok)) return cudaErrorNotSupported;
+  if (!tc::make_rows_tmap(&tk, ib + ix.kb16, krows, DD, kCt)) return cudaErrorNotSupported;
+  SelTcArgs a{};
+  a.qn = qn;
+  a.kbar32 = kbar32;
+  a.kn = (const float*)(ib + ix.kn);
+  a.ktmax = (const float*)(ib + ix.ktmax);
+  a.L = 1;
+  a.Hkv = Dm.Hkv;
+  a.Nc = (int)Dm.Nc;
+  a.Ncp = (int)((Dm.Nc + kCt - 1) / kCt * kCt);
+  a.topk = Dm.topk;
+  a.n_qt = lo.n_qt;
+  a.BH = Dm.Hkv;
+  a.scale_sel = Dm.scale_sel;
+  a.Bq = Dm.Bq;
+  a.n_split = lo.n_split;
+  a.range = lo.range;
+  a.cand_l = (float*)(base + lo.cl);
+  a.cand_u = (float*)(base + lo.cu);
+  a.cand_c = (int32_t*)(base + lo.cc);
+  a.cand_n = (int32_t*)(base + lo.cn);
+  a.cand_d = (float*)(base + lo.cd);
+  const size_t smem = sizeof(SelTcSmem<DD, KT>) + 1024;
+  if ((e = cudaFuncSetAttribute(sel_tc_kernel<DD, KT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)smem)) != cudaSuccess)
+    return e;
+  sel_tc_kernel<DD, KT, true><<<dim3((unsigned)lo.n_split, (unsigned)Dm.Hkv, (unsigned)lo.n_qt), kThreads, smem, st>>>(
+      a, tq, tk, unused);
+  note_launches(1);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const int rows = Dm.Bq * Dm.Hkv;
+  dtc_merge_kernel<DD><<<(unsigned)rows, 256, 0, st>>>(
+      a.cand_l, a.cand_u, a.cand_c, a.cand_n, a.cand_d, SelCfg<KT>::kBuf, qh32, kbar32, idx, s_sel, w, Dm.Bq, Dm.Hkv,
+      (int)Dm.Nc, lo.n_split, lo.range, Dm.topk, Dm.scale_sel);
+  note_launches(1);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  return launch_decode_attend(Dm, q, K, V, idx, w, O, (float*)(base + lo.opart), st);
+}
+
+}  // namespace
+
+bool decode_tc_applies(const DecodeDims& D) { return D.topk <= 16 && D.Nc > 0 && D.Nc * (long long)D.Hkv < (1LL << 31); }
+
+size_t decode_index_bytes(const DecodeDims& D) { return D.Nc > 0 ? dec_index_layout(D).total : 0; }
+
+cudaError_t launch_decode_index(const DecodeDims& Dm, const float* kbar32, void* index, cudaStream_t st) {
+  if (Dm.Nc == 0) return cudaSuccess;
+  const DecIndexLayout ix = dec_index_layout(Dm);
+  char* base = (char*)index;
+  const int Ncp = (int)((Dm.Nc + kCt - 1) / kCt * kCt);
+  cudaError_t e;
+  if ((e = cudaMemsetAsync(base + ix.ktmax, 0, ix.total - ix.ktmax, st)) != cudaSuccess) return e;
+  const long long krows = Dm.Nc * Dm.Hkv;  // input rows (i, g) of the one-batch memory
+  if (Dm.d == 64)
+    sel_kbar_kernel<64><<<(unsigned)((krows * 8 + 255) / 256), 256, 0, st>>>(
+        kbar32, (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows, (int)Dm.Nc,
+        Ncp, Dm.Hkv);
+  else
+    sel_kbar_kernel<128><<<(unsigned)((krows * 16 + 255) / 256), 256, 0, st>>>(
+        kbar32, (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows, (int)Dm.Nc,
+        Ncp, Dm.Hkv);
+  note_launches(1);
+  return cudaGetLastError();
+}
+
+size_t decode_tc_workspace(const DecodeDims& D) {
+  if (!decode_tc_applies(D) || D.Bq == 0) return 0;
+  return D.topk <= 8 ? dec_tc_layout<8>(D).total : dec_tc_layout<16>(D).total;
+}
+
+cudaError_t launch_decode_tc(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
+                             const void* index, void* O, int32_t* idx, float* s_sel, float* w, void* ws,
+                             cudaStream_t st) {
+  if (D.d == 64) return D.topk <= 8 ? run_decode_tc<64, 8>(D, q, K, V, kbar32, index, O, idx, s_sel, w, ws, st)
+                                    : run_decode_tc<64, 16>(D, q, K, V, kbar32, index, O, idx, s_sel, w, ws, st);
+  return D.topk <= 8 ? run_decode_tc<128, 8>(D, q, K, V, kbar32, index, O, idx, s_sel, w, ws, st)
+                     : run_decode_tc<128, 16>(D, q, K, V, kbar32, index, O, idx, s_sel, w, ws, st);
+}
 
 bool select_tc_applies(const Dims& D) { return D.topk <= 16 && D.Nc > 0; }
 

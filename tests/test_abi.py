@@ -138,6 +138,21 @@ def test_decode_noalloc_rejects_shapes_beyond_its_scratch(lib):
     assert lib.hsa_decode_noalloc(ctypes.byref(c), *[vp(FAKE + 8)] * 8, None) == INVALID
 
 
+def test_decode_index_sizes_and_fallback(lib):
+    vp = ctypes.c_void_p
+    s = hsa.DecodeShape(Bq=64, Hq=8, Hkv=1, d=128, n_chunks=1 << 20, topk=8)
+    c = s.c()
+    # bf16 summaries + one fp32 norm per chunk + one max per 64 chunks
+    assert lib.hsa_decode_index_size(ctypes.byref(c)) >= (1 << 20) * (128 * 2 + 4)
+    assert lib.hsa_decode_indexed_workspace_size(ctypes.byref(c)) > 0
+    big_k = hsa.DecodeShape(Bq=64, Hq=8, Hkv=1, d=128, n_chunks=1 << 20, topk=20).c()
+    assert lib.hsa_decode_index_size(ctypes.byref(big_k)) == 0
+    assert lib.hsa_decode_index(ctypes.byref(big_k), vp(FAKE), vp(FAKE), 0, None) == UNSUPPORTED
+    assert lib.hsa_decode_index(ctypes.byref(c), vp(FAKE), vp(FAKE), 16, None) == WORKSPACE
+    # a missing index is an invalid argument (checked before any launch)
+    assert lib.hsa_decode_indexed(ctypes.byref(c), *[vp(FAKE)] * 4, vp(0), *[vp(FAKE)] * 5, 1 << 40, None) == INVALID
+
+
 def test_workspace_sizes_scale_with_the_problem(lib):
     s = shape(B=2, L=32768, Hq=32, Hkv=4)
     slots = 2 * 32768 * 4 * 8

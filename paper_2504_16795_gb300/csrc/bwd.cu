@@ -55,6 +55,7 @@ struct BwdSmem {
   uint16_t P[kRows * kChunk];     // w * P
   uint16_t dSq[kRows * kChunk];   // c_att * w * P∘(dP' - D)            (feeds dq)
   uint16_t dSk[kRows * kChunk];   // dSq + c_sel * ds / S               (feeds dK: attention + mean pool)
+  uint16_t dqstage[4][32 * 32];   // TMA path: per epilogue warp, 32 rows x 32 columns of dq' (64-byte swizzle)
   float kbar[D];
   int slot_row[2][kRows];         // first q row of each slot (-1: past the list)
   int slot_p[2][kRows];
@@ -111,7 +112,8 @@ struct Cols {
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
-    bwd_chunk_kernel(BwdArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_do) {
+    bwd_chunk_kernel(BwdArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_do,
+                     const __grid_constant__ CUtensorMap tmap_dq) {
   extern __shared__ unsigned char smem_raw[];
   BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
@@ -440,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int pj = sm.row_p[sb][r];
       tc::mbar_wait(bar(BAR_DQ_FULL), j & 1, abort_flag, status);
       tc::fence_after_sync();
-      uint16_t* dst = pj >= 0 ? a.dqpart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
+      uint16_t* dst = (!a.use_tma && pj >= 0) ? a.dqpart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
       const float cs = a.scale_sel * dsj;
       float v[D];
 #pragma unroll
@@ -448,7 +450,33 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::tmem_wait_ld();
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_DQ_EMPTY));
-      if (dst) {
+      if (a.use_tma) {
+        // 32 columns at a time through the warp's staging tile; the lane of
+        // every 8-row group stores the group with one TMA box
+        const uint32_t stage = smem_u32(sm.dqstage[warp & 3]) + (lane >> 3) * 512 + (lane & 7) * 64;
+        const uint32_t swz = (lane >> 1) & 3;
+        const bool issuer = (lane & 7) == 0 && pj >= 0;
+#pragma unroll
+        for (int h = 0; h < D / 32; ++h) {
+          if ((lane & 7) == 0) tc::bulk_wait_read();  // the previous round's boxes have left the tile
+          __syncwarp();
+#pragma unroll
+          for (int q8 = 0; q8 < 4; ++q8) {
+            float o[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) o[k] = v[h * 32 + 8 * q8 + k] + cs * sm.kbar[h * 32 + 8 * q8 + k];
+            asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(stage + ((q8 ^ swz) << 4)),
+                         "r"(pack_bf16x2(o[0], o[1])), "r"(pack_bf16x2(o[2], o[3])), "r"(pack_bf16x2(o[4], o[5])),
+                         "r"(pack_bf16x2(o[6], o[7])));
+          }
+          tc::fence_proxy_async_smem();
+          __syncwarp();
+          if (issuer) {
+            tc::tma_store_2d(&tmap_dq, h * 32, pj * a.G + (r & (a.G - 1)), stage);
+            tc::bulk_commit();
+          }
+        }
+      } else if (dst) {
         uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
         for (int q8 = 0; q8 < D / 8; ++q8) {
@@ -460,6 +488,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    if (a.use_tma && (lane & 7) == 0) tc::bulk_wait_all();
     // dK, dV of the chunk: TMEM lane = head dim, column = chunk row
     tc::mbar_wait(bar(BAR_ACC_DONE), 0, abort_flag, status);
     tc::fence_after_sync();
@@ -604,15 +633,17 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     if ((e = cudaFuncSetAttribute(bwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
         cudaSuccess)
       return e;
-    CUtensorMap tq, tdo;
+    CUtensorMap tq, tdo, tdq;
     memset(&tq, 0, sizeof(tq));
     memset(&tdo, 0, sizeof(tdo));
+    memset(&tdq, 0, sizeof(tdq));
     a.n_rows = Dm.B * Dm.L * Dm.Hq;
     a.use_tma = Dm.G >= 8 ? 1 : 0;
     if (a.use_tma && (!tc::make_group8_tmap(&tq, q, (unsigned long long)a.n_rows, D) ||
-                      !tc::make_group8_tmap(&tdo, dO, (unsigned long long)a.n_rows, D)))
+                      !tc::make_group8_tmap(&tdo, dO, (unsigned long long)a.n_rows, D) ||
+                      !tc::make_rows32_sw64_tmap(&tdq, dqpart, (unsigned long long)Dm.slots() * Dm.G, D)))
       return cudaErrorNotSupported;
-    bwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq, tdo);
+    bwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq, tdo, tdq);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

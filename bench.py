@@ -54,8 +54,8 @@ def select_workload(number, batch):
 # has changed).
 NCU_TRAFFIC = {
     # bwd_delta + bwd_chunk + bwd_dq_merge at the long-context workload (B=2, L=32768), one launch each
-    "hsa_backward": {"bytes_per_launch": 15075620096, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
-                     "sha256": "abfbeaf8dd1418c3cc8654fe0238e8d36f783348f1f64ae5ae4a0088febb9904"},
+    "hsa_backward": {"bytes_per_launch": 15407138304, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
+                     "sha256": "dff8a9b920f1c01b0fc423ea3badf2353e8992233ffdb569294e1bf13cd389a0"},
 }
 
 
@@ -493,6 +493,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", type=int, default=3, help="prefill workload number (3 is the headline)")
     ap.add_argument("--batch", type=int, default=0, help="override the workload's batch (profiling)")
+    ap.add_argument("--decode-only", action="store_true",
+                    help="run only the decode sub-benchmark and print its object (profiling)")
     args = ap.parse_args()
     select_workload(args.workload, args.batch)
     rank = int(os.environ.get("RANK", "0"))
@@ -500,6 +502,18 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.decode_only:
+        import torch
+
+        import paper_2504_16795_gb300 as hsa
+
+        hsa.build()
+        hsa.load()
+        dev = torch.device("cuda", local_rank)
+        torch.cuda.set_device(dev)
+        d = run_decode(args, dev, 1, peaks(), torch.cuda.synchronize, lambda x: x, hsa)
+        print(json.dumps({"decode": d}), flush=True)
         return
     import torch.distributed as dist
 

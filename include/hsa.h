@@ -220,7 +220,7 @@ size_t hsa_decode_indexed_workspace_size(const hsa_decode_shape_t* shape);
  * identical, O and w to fp32 rounding), with the scan of the summaries on the
  * tensor cores. Blocks over ranges of the memory score bf16 summaries against
  * the group query; per query and range, the scores' rounding error is bounded
- * (|error| < 2^-7 |q̂| |K̄_i|), so only the chunks that bound cannot rule out
+ * (|error| < 2^-7 * 9/8 * |q̂| |K̄_i|), so only the chunks that bound cannot rule out
  * are kept, and those are rescored with the fp32 chain of hsa_select_topk
  * before the top-k is taken. For topk > 16 it falls back to hsa_decode's scan
  * (index may then be NULL).

@@ -16,7 +16,9 @@
 // The mean-pool term reaches every row s of the chunk equally, and q̂_t is
 // the sum of the slot's G query rows, so adding c_sel ds_j / S to every
 // element of the slot's rows of the dS tile that feeds dK = dS^T Q produces
-// dK̄_I / S inside the same tensor-core product.
+// dK̄_I / S inside the same tensor-core product. The same tile also yields the
+// selection term of dq: K̄_I is the mean of the chunk's S key rows, so
+// (da c_att + c_sel ds_j / S) K_I = c_att da K_I + c_sel ds_j K̄_I.
 //
 // Chunk-major and deterministic: one block per (b, g, chunk) owns that
 // chunk's dK/dV rows, walks the chunk's slots (from the inverse index) in
@@ -27,12 +29,15 @@
 //
 // Per 128-row step on the 5th-generation tensor core (one issuing thread):
 //   S = Q K^T, dP' = dO V^T            (M = 128 rows, N = 64, K = d)
-//   dq' = dSq K                        (K read as an MN-major operand)
 //   dV^T += dO^T (wP), dK^T += Q^T dSk (M = d, N = 64, K = 128 rows; the
 //                                       row-major tiles read MN-major)
-// Warps 0-3 (one thread per row) turn S, dP' into P, dSq, dSk; warps 4-7
-// store dq' (plus the selection term) and finally dK, dV; warp 8 gathers the
-// Q and dO rows of the next tiles; one thread of warp 9 issues the MMAs.
+//   dq' = dSk K                        (K read as an MN-major operand)
+// The dK/dV products come first, so the Q/dO stage is released before the
+// dq product runs. Warps 0-3 (one thread per row) turn S, dP' into P and
+// dSk; warps 4-7 store dq' and finally dK, dV; warps 8 and 10 gather the Q
+// and dO rows of the next tiles (a TMA issue costs each issuing warp tens of
+// nanoseconds per box, so the two tensors go out from two warps); one thread
+// of warp 9 issues the MMAs.
 #include <cstring>
 
 #include "tc.cuh"
@@ -41,7 +46,7 @@ namespace hsa {
 namespace {
 
 constexpr int kRows = 128;     // query rows per step (tensor-core M)
-constexpr int kThreads = 320;  // warps 0-3 softmax/gradients, 4-7 epilogue, 8 loader, 9 MMA
+constexpr int kThreads = 352;  // warps 0-3 softmax/gradients, 4-7 epilogue, 8 and 10 loaders, 9 MMA
 constexpr int kTmemCols = 512;
 
 __device__ unsigned g_bwd_status;
@@ -53,16 +58,13 @@ struct BwdSmem {
   uint16_t K[kChunk * D];         // chunk keys [s][d]
   uint16_t V[kChunk * D];         // chunk values [s][d]
   uint16_t P[kRows * kChunk];     // w * P
-  uint16_t dSq[kRows * kChunk];   // c_att * w * P∘(dP' - D)            (feeds dq)
-  uint16_t dSk[kRows * kChunk];   // dSq + c_sel * ds / S               (feeds dK: attention + mean pool)
-  uint16_t dqstage[4][32 * 32];   // TMA path: per epilogue warp, 32 rows x 32 columns of dq' (64-byte swizzle)
-  float kbar[D];
+  uint16_t dSk[kRows * kChunk];   // c_att * w * P∘(dP' - D) + c_sel * ds / S  (feeds dK and dq)
+  uint16_t dqstage[kRows * 64];   // TMA path: 64 columns of dq' (8-row atoms, 128-byte swizzle; 4 KB per warp)
   int slot_row[2][kRows];         // first q row of each slot (-1: past the list)
   int slot_p[2][kRows];
   float slot_w[2][kRows];
   float slot_delta[2][kRows];
-  float row_ds[2][kRows];         // softmax -> epilogue: ds of the row's slot
-  int row_p[2][kRows];            // softmax -> epilogue: the row's slot id (-1: none)
+  int row_p[3][kRows];            // softmax -> epilogue: the row's slot id (-1: none)
   uint64_t bar[16];
   uint32_t tmem_base;
   int abort_flag;
@@ -78,7 +80,7 @@ enum {
   BAR_DQ_FULL = 10,  // dq accumulator ready (commit)
   BAR_DQ_EMPTY = 11, // dq read (128 arrivals)
   BAR_ACC_DONE = 12, // last dK^T / dV^T update finished (commit)
-  BAR_DS_FULL = 13   // 2: row_ds / row_p of a step written (128 arrivals)
+  BAR_DS_FULL = 13   // 3: row_p of a step written (128 arrivals)
 };
 
 struct BwdArgs {
@@ -86,7 +88,6 @@ struct BwdArgs {
   const uint16_t* K;
   const uint16_t* V;
   const uint16_t* dO;
-  const float* kbar32;
   const float* w;
   const float* delta;  // [B, L, Hkv]
   const int32_t* offsets;
@@ -141,12 +142,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (tid == 0) {
     for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(bar(BAR_QD_FULL + i), a.use_tma ? 1 : 32);
+      tc::mbar_init(bar(BAR_QD_FULL + i), a.use_tma ? 2 : 32);
       tc::mbar_init(bar(BAR_QD_EMPTY + i), 1);
       tc::mbar_init(bar(BAR_S_FULL + i), 1);
       tc::mbar_init(bar(BAR_S_EMPTY + i), 128);
-      tc::mbar_init(bar(BAR_DS_FULL + i), 128);
     }
+    for (int i = 0; i < 3; ++i) tc::mbar_init(bar(BAR_DS_FULL + i), 128);
     tc::mbar_init(bar(BAR_P_FULL), 128);
     tc::mbar_init(bar(BAR_P_EMPTY), 1);
     tc::mbar_init(bar(BAR_DQ_FULL), 1);
@@ -163,7 +164,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       cp_async16(smem_u32(sm.K) + tc::sw128_offset(kChunk, srow, ch * 8), a.K + src);
       cp_async16(smem_u32(sm.V) + tc::sw128_offset(kChunk, srow, ch * 8), a.V + src);
     }
-    for (int u = tid; u < D; u += 256) sm.kbar[u] = a.kbar32[(((long long)b * a.Nc + c) * a.Hkv + g) * D + u];
     cp_async_commit();
     cp_async_wait<0>();
     tc::fence_proxy_async_smem();
@@ -237,19 +237,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
       if (a.use_tma) {
-        // lane l < epi gathers slot l's G rows of q and dO (one box per 64
-        // columns); the single expected arrival carries the byte count and
-        // publishes the slot tables written above
+        // lane l < epi gathers slot l's G rows of q (one box per 8-row
+        // group); this warp's expected arrival carries the byte count and
+        // publishes the slot tables written above (warp 10 brings dO)
         if (lane < epi) {
           const int y = c_row >= 0 ? c_row : a.n_rows;  // past the list: zeros
-          for (int j = 0; j < (a.G >> 3); ++j) {  // one box per 8-row group
-            const uint32_t o = (lane * (a.G >> 3) + j) * (16 * D);
-            tc::tma_load_3d(qb + o, &tmap_q, 0, y + 8 * j, 0, bar(BAR_QD_FULL + st));
-            tc::tma_load_3d(ob + o, &tmap_do, 0, y + 8 * j, 0, bar(BAR_QD_FULL + st));
-          }
+          for (int j = 0; j < (a.G >> 3); ++j)
+            tc::tma_load_3d(qb + (lane * (a.G >> 3) + j) * (16 * D), &tmap_q, 0, y + 8 * j, 0, bar(BAR_QD_FULL + st));
         }
         __syncwarp();
-        if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), 2 * kRows * D * 2);
+        if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), kRows * D * 2);
         continue;
       }
       __syncwarp();
@@ -286,7 +283,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t kGrp = 16 * D;
       constexpr uint32_t kMnK = (uint32_t)kChunk * 128;
       const uint32_t kbase = smem_u32(sm.K), vbase = smem_u32(sm.V);
-      const uint32_t pbase = smem_u32(sm.P), dsq = smem_u32(sm.dSq), dsk = smem_u32(sm.dSk);
+      const uint32_t pbase = smem_u32(sm.P), dsk = smem_u32(sm.dSk);
       auto issue_SdP = [&](int i) {
         const int st = i & 1, sb = i & 1;
         tc::fence_after_sync();
@@ -302,15 +299,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc::mma_commit(bar(BAR_S_FULL + sb));
       };
-      auto issue_rest = [&](int i) {
+      auto issue_KV = [&](int i) {
         const int st = i & 1;
         tc::fence_after_sync();
-        // dq' = dSq K : M = 128 rows, N = D, K = 64 chunk rows
-#pragma unroll
-        for (int kk = 0; kk < kChunk / 16; ++kk)
-          tc::mma_bf16_ss(tmem + Cols<D>::dq, tc::sdesc_sw128(dsq + kk * 32),
-                          tc::sdesc_sw128_mn(kbase + kk * 2048, kMnK), idDQ, kk > 0);
-        tc::mma_commit(bar(BAR_DQ_FULL));
         // dV^T += dO^T (wP), dK^T += Q^T dSk : M = head dim, N = 64, K = 128 rows
         const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
 #pragma unroll
@@ -322,24 +313,36 @@ __global__ void __launch_bounds__(kThreads, 1)
                           tc::sdesc_sw128_mn(dsk + kk * 2048, 0), idKV, acc);
         }
         tc::mma_commit(bar(BAR_QD_EMPTY + st));
+      };
+      auto issue_DQ = [&]() {
+        // dq' = dSk K : M = 128 rows, N = D, K = 64 chunk rows
+#pragma unroll
+        for (int kk = 0; kk < kChunk / 16; ++kk)
+          tc::mma_bf16_ss(tmem + Cols<D>::dq, tc::sdesc_sw128(dsk + kk * 32),
+                          tc::sdesc_sw128_mn(kbase + kk * 2048, kMnK), idDQ, kk > 0);
+        tc::mma_commit(bar(BAR_DQ_FULL));
         tc::mma_commit(bar(BAR_P_EMPTY));
       };
       // Event loop: issue whichever is ready — S/dP' of step nS (tile landed,
-      // accumulator buffer read) or the second half of step nR (P tiles written,
-      // dq accumulator read). Neither barrier can run a phase past the one
-      // polled before the corresponding issue, so parity polling is exact.
-      int nS = 0, nR = 0;
+      // accumulator buffer read), dK/dV of step nK (P tiles written) or dq of
+      // step nQ (dq accumulator read). Neither barrier can run a phase past the
+      // one polled before the corresponding issue, so parity polling is exact.
+      int nS = 0, nK = 0, nQ = 0;
       unsigned long long t0 = tc::globaltimer();
-      while (nR < niter) {
+      while (nQ < niter) {
         bool progressed = false;
-        if (nS < niter && nS < nR + 2 && tc::mbar_try_wait(bar(BAR_QD_FULL + (nS & 1)), (nS >> 1) & 1) &&
-            tc::mbar_try_wait(bar(BAR_S_EMPTY + (nS & 1)), ((nS >> 1) & 1) ^ 1)) {
+        if (nS < niter && nS < nQ + 2 && tc::mbar_test_wait(bar(BAR_QD_FULL + (nS & 1)), (nS >> 1) & 1) &&
+            tc::mbar_test_wait(bar(BAR_S_EMPTY + (nS & 1)), ((nS >> 1) & 1) ^ 1)) {
           issue_SdP(nS++);
           progressed = true;
         }
-        if (nR < nS && tc::mbar_try_wait(bar(BAR_P_FULL), nR & 1) &&
-            tc::mbar_try_wait(bar(BAR_DQ_EMPTY), (nR & 1) ^ 1)) {
-          issue_rest(nR++);
+        if (nK < nS && tc::mbar_test_wait(bar(BAR_P_FULL), nK & 1)) {
+          issue_KV(nK++);
+          progressed = true;
+        }
+        if (nQ < nK && tc::mbar_test_wait(bar(BAR_DQ_EMPTY), (nQ & 1) ^ 1)) {
+          issue_DQ();
+          ++nQ;
           progressed = true;
         }
         if (progressed) {
@@ -351,6 +354,32 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mma_commit(bar(BAR_ACC_DONE));
     }
     __syncwarp();
+  } else if (warp == 10) {
+    // ---------------------------------------------------------------- second loader warp (TMA path: dO)
+    if (a.use_tma) {
+      auto load_p = [&](int i) {
+        const int e = i * epi + lane;
+        return (lane < epi && e < cnt) ? a.entries[off + e] : -1;
+      };
+      auto row_of = [&](int p) {  // past the list: rows past the tensor read zeros
+        return p < 0 ? a.n_rows : ((b * a.L + (p / slot_div) % a.L) * a.Hq) + g * a.G;
+      };
+      int p_cur = load_p(0), p_next = load_p(1);
+      for (int i = 0; i < niter; ++i) {
+        const int st = i & 1;
+        const int y = row_of(p_cur);
+        p_cur = p_next;
+        p_next = load_p(i + 2);
+        tc::mbar_wait(bar(BAR_QD_EMPTY + st), ((i >> 1) & 1) ^ 1, abort_flag, status);
+        const uint32_t ob = smem_u32(sm.dO[st]);
+        if (lane < epi) {
+          for (int j = 0; j < (a.G >> 3); ++j)
+            tc::tma_load_3d(ob + (lane * (a.G >> 3) + j) * (16 * D), &tmap_do, 0, y + 8 * j, 0, bar(BAR_QD_FULL + st));
+        }
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), kRows * D * 2);
+      }
+    }
   } else if (warp < 4) {
     // ---------------------------------------------------------------- softmax / gradient rows (thread = row)
     const int r = tid;
@@ -400,31 +429,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       float dw = Drow;  // sum over the G rows of the slot (consecutive lanes)
       for (int o = 1; o < a.G; o <<= 1) dw += __shfl_xor_sync(0xFFFFFFFFu, dw, o);
       const float dsv = wv * (dw - dl);
-      // hand ds and the slot id to the epilogue warps (double-buffered: the
-      // buffer of step i is rewritten at step i+2, after the epilogue of step i
-      // has released the dq accumulator that step i+1's dq product waits for)
-      sm.row_ds[sb][r] = dsv;
-      sm.row_p[sb][r] = pv;
-      tc::mbar_arrive(bar(BAR_DS_FULL + sb));
+      // hand the slot id to the epilogue warps (three buffers: step i+3 runs
+      // after S of step i+3, which the MMA thread issues only after the dK/dV
+      // products of step i+1, which wait for the epilogue of step i to have
+      // read the dq accumulator, and so its slot ids)
+      sm.row_p[i % 3][r] = pv;
+      tc::mbar_arrive(bar(BAR_DS_FULL + i % 3));
       const float ca = a.scale_attn * wv, pool = a.scale_sel * dsv * inv_S;
       tc::mbar_wait(bar(BAR_P_EMPTY), (i & 1) ^ 1, abort_flag, status);
-      const uint32_t prow = smem_u32(sm.P), qrow = smem_u32(sm.dSq), krow = smem_u32(sm.dSk);
+      const uint32_t prow = smem_u32(sm.P), krow = smem_u32(sm.dSk);
 #pragma unroll
       for (int c16 = 0; c16 < 8; ++c16) {
         const uint32_t o = tc::sw128_offset(kRows, r, c16 * 8);
-        uint32_t pp[4], gq[4], gk[4];
+        uint32_t pp[4], gk[4];
 #pragma unroll
         for (int h = 0; h < 4; ++h) {
           const int k0 = 8 * c16 + 2 * h;
-          const float g0 = ca * x[k0] * (y[k0] - Drow), g1 = ca * x[k0 + 1] * (y[k0 + 1] - Drow);
           pp[h] = pack_bf16x2(wv * x[k0], wv * x[k0 + 1]);
-          gq[h] = pack_bf16x2(g0, g1);
-          gk[h] = pack_bf16x2(g0 + pool, g1 + pool);
+          gk[h] = pack_bf16x2(fmaf(ca * x[k0], y[k0] - Drow, pool), fmaf(ca * x[k0 + 1], y[k0 + 1] - Drow, pool));
         }
         asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(prow + o), "r"(pp[0]), "r"(pp[1]), "r"(pp[2]),
                      "r"(pp[3]));
-        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(qrow + o), "r"(gq[0]), "r"(gq[1]), "r"(gq[2]),
-                     "r"(gq[3]));
         asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(krow + o), "r"(gk[0]), "r"(gk[1]), "r"(gk[2]),
                      "r"(gk[3]));
       }
@@ -436,14 +461,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = tid - 128;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     for (int j = 0; j < niter; ++j) {
-      const int sb = j & 1;
-      tc::mbar_wait(bar(BAR_DS_FULL + sb), (j >> 1) & 1, abort_flag, status);
-      const float dsj = sm.row_ds[sb][r];
-      const int pj = sm.row_p[sb][r];
+      tc::mbar_wait(bar(BAR_DS_FULL + j % 3), (j / 3) & 1, abort_flag, status);
+      const int pj = sm.row_p[j % 3][r];
       tc::mbar_wait(bar(BAR_DQ_FULL), j & 1, abort_flag, status);
       tc::fence_after_sync();
       uint16_t* dst = (!a.use_tma && pj >= 0) ? a.dqpart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
-      const float cs = a.scale_sel * dsj;
       float v[D];
 #pragma unroll
       for (int h = 0; h < D / 32; ++h) tc::tmem_ld32(tmem + lane_base + Cols<D>::dq + h * 32, *reinterpret_cast<float(*)[32]>(&v[h * 32]));
@@ -451,28 +473,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_DQ_EMPTY));
       if (a.use_tma) {
-        // 32 columns at a time through the warp's staging tile; the lane of
-        // every 8-row group stores the group with one TMA box
-        const uint32_t stage = smem_u32(sm.dqstage[warp & 3]) + (lane >> 3) * 512 + (lane & 7) * 64;
-        const uint32_t swz = (lane >> 1) & 3;
+        // 64 columns at a time through the warp's staging atoms (one 1 KB
+        // atom per 8 rows, 128-byte swizzle); the first lane of every 8-row
+        // group stores the group with one TMA box
+        const uint32_t atom = smem_u32(sm.dqstage) + (warp & 3) * 4096 + (lane >> 3) * 1024;
+        const uint32_t row = atom + (lane & 7) * 128, swz = lane & 7;
         const bool issuer = (lane & 7) == 0 && pj >= 0;
 #pragma unroll
-        for (int h = 0; h < D / 32; ++h) {
-          if ((lane & 7) == 0) tc::bulk_wait_read();  // the previous round's boxes have left the tile
+        for (int h = 0; h < D / 64; ++h) {
+          if ((lane & 7) == 0) tc::bulk_wait_read();  // the previous round's boxes have left the atoms
           __syncwarp();
 #pragma unroll
-          for (int q8 = 0; q8 < 4; ++q8) {
-            float o[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) o[k] = v[h * 32 + 8 * q8 + k] + cs * sm.kbar[h * 32 + 8 * q8 + k];
-            asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(stage + ((q8 ^ swz) << 4)),
+          for (int c8 = 0; c8 < 8; ++c8) {
+            const float* o = &v[h * 64 + 8 * c8];
+            asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(row + ((c8 ^ swz) << 4)),
                          "r"(pack_bf16x2(o[0], o[1])), "r"(pack_bf16x2(o[2], o[3])), "r"(pack_bf16x2(o[4], o[5])),
                          "r"(pack_bf16x2(o[6], o[7])));
           }
           tc::fence_proxy_async_smem();
           __syncwarp();
           if (issuer) {
-            tc::tma_store_2d(&tmap_dq, h * 32, pj * a.G + (r & (a.G - 1)), stage);
+            tc::tma_store_2d(&tmap_dq, h * 64, pj * a.G + (r & (a.G - 1)), atom);
             tc::bulk_commit();
           }
         }
@@ -480,9 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
         for (int q8 = 0; q8 < D / 8; ++q8) {
-          float o[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) o[k] = v[8 * q8 + k] + cs * sm.kbar[8 * q8 + k];
+          const float* o = &v[8 * q8];
           d4[q8] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
                               pack_bf16x2(o[6], o[7]));
         }
@@ -611,7 +630,6 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.K = (const uint16_t*)K;
     a.V = (const uint16_t*)V;
     a.dO = (const uint16_t*)dO;
-    a.kbar32 = kbar32;
     a.w = w;
     a.delta = delta;
     a.offsets = offsets;
@@ -641,7 +659,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.use_tma = Dm.G >= 8 ? 1 : 0;
     if (a.use_tma && (!tc::make_group8_tmap(&tq, q, (unsigned long long)a.n_rows, D) ||
                       !tc::make_group8_tmap(&tdo, dO, (unsigned long long)a.n_rows, D) ||
-                      !tc::make_rows32_sw64_tmap(&tdq, dqpart, (unsigned long long)Dm.slots() * Dm.G, D)))
+                      !tc::make_rows_tmap(&tdq, dqpart, (unsigned long long)Dm.slots() * Dm.G, D, 8)))
       return cudaErrorNotSupported;
     bwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq, tdo, tdq);
     note_launches(1);

@@ -219,13 +219,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       unsigned long long t0 = tc::globaltimer();
       while (nO < niter) {
         bool progressed = false;
-        if (nS < niter && nS < nO + 2 && tc::mbar_try_wait(bar(BAR_Q_FULL + nS % kQStages), (nS / kQStages) & 1) &&
-            tc::mbar_try_wait(bar(BAR_S_EMPTY + (nS & 1)), ((nS >> 1) & 1) ^ 1)) {
+        if (nS < niter && nS < nO + 2 && tc::mbar_test_wait(bar(BAR_Q_FULL + nS % kQStages), (nS / kQStages) & 1) &&
+            tc::mbar_test_wait(bar(BAR_S_EMPTY + (nS & 1)), ((nS >> 1) & 1) ^ 1)) {
           issue_S(nS++);
           progressed = true;
         }
-        if (nO < nS && tc::mbar_try_wait(bar(BAR_P_FULL + (nO & 1)), (nO >> 1) & 1) &&
-            tc::mbar_try_wait(bar(BAR_O_EMPTY + (nO & 1)), ((nO >> 1) & 1) ^ 1)) {
+        if (nO < nS && tc::mbar_test_wait(bar(BAR_P_FULL + (nO & 1)), (nO >> 1) & 1) &&
+            tc::mbar_test_wait(bar(BAR_O_EMPTY + (nO & 1)), ((nO >> 1) & 1) ^ 1)) {
           issue_O(nO++);
           progressed = true;
         }

@@ -34,10 +34,8 @@
 //   dq' = dSk K                        (K read as an MN-major operand)
 // The dK/dV products come first, so the Q/dO stage is released before the
 // dq product runs. Warps 0-3 (one thread per row) turn S, dP' into P and
-// dSk; warps 4-7 store dq' and finally dK, dV; warps 8 and 10 gather the Q
-// and dO rows of the next tiles (a TMA issue costs each issuing warp tens of
-// nanoseconds per box, so the two tensors go out from two warps); one thread
-// of warp 9 issues the MMAs.
+// dSk; warps 4-7 store dq' and finally dK, dV; warps 8, 10 and 11 gather the
+// Q and dO rows of the next tiles; one thread of warp 9 issues the MMAs.
 #include <cstring>
 
 #include "tc.cuh"
@@ -46,7 +44,8 @@ namespace hsa {
 namespace {
 
 constexpr int kRows = 128;     // query rows per step (tensor-core M)
-constexpr int kThreads = 352;  // warps 0-3 softmax/gradients, 4-7 epilogue, 8 and 10 loaders, 9 MMA
+constexpr int kThreads = 384;  // warps 0-3 softmax/gradients, 4-7 epilogue, 8, 10, 11 loaders, 9 MMA
+constexpr int kLoaders = 3;
 constexpr int kTmemCols = 512;
 
 __device__ unsigned g_bwd_status;
@@ -142,7 +141,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (tid == 0) {
     for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(bar(BAR_QD_FULL + i), a.use_tma ? 2 : 32);
+      tc::mbar_init(bar(BAR_QD_FULL + i), a.use_tma ? kLoaders : 32);
       tc::mbar_init(bar(BAR_QD_EMPTY + i), 1);
       tc::mbar_init(bar(BAR_S_FULL + i), 1);
       tc::mbar_init(bar(BAR_S_EMPTY + i), 128);
@@ -173,14 +172,30 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::fence_after_sync();
   const uint32_t tmem = sm.tmem_base;
 
-  if (warp == 8) {
-    // ---------------------------------------------------------------- loader warp
-    // The slot data of a tile is fetched in two stages ahead of use: the slot
-    // ids two tiles ahead, the token, weight and Δ one tile ahead, so no
-    // dependent global load sits on the loader's critical path.
-    auto load_p = [&](int i) {
+  if (warp == 8 || warp >= 10) {
+    // ---------------------------------------------------------------- loader warps
+    // TMA path: a tile's 2 * epi gathers (item s < epi: the q rows of slot s;
+    // item epi + s: the dO rows of slot s) are spread over warps 8, 10 and 11,
+    // lane l of loader li taking item li + 3 l, since a TMA issue costs the
+    // issuing warp tens of nanoseconds per box. Warp 8 also fills the slot
+    // tables and runs the cp.async path alone. Slot data is fetched in two
+    // stages ahead of use: the slot ids two tiles ahead, the token, weight and
+    // Δ one tile ahead, so no dependent global load sits on the critical path.
+    const int li = warp == 8 ? 0 : warp - 9;
+    const int item = li + kLoaders * lane;
+    const bool has_item = a.use_tma && item < 2 * epi;
+    const int islot = item < epi ? item : item - epi;
+    const uint32_t item_bytes = (uint32_t)((2 * epi - li + kLoaders - 1) / kLoaders) * a.G * D * 2;
+    auto load_ip = [&](int i) {
+      const int e = i * epi + islot;
+      return (has_item && e < cnt) ? a.entries[off + e] : -1;
+    };
+    auto row_of = [&](int p) {  // past the list: rows past the tensor read zeros
+      return p < 0 ? a.n_rows : ((b * a.L + (p / slot_div) % a.L) * a.Hq) + g * a.G;
+    };
+    auto load_p = [&](int i) {  // warp 8's slot tables: lane l holds slot l
       const int e = i * epi + lane;
-      return (epi <= 32 && lane < epi && e < cnt) ? a.entries[off + e] : -1;
+      return (li == 0 && epi <= 32 && lane < epi && e < cnt) ? a.entries[off + e] : -1;
     };
     int n_row = -1, n_p = -1;
     float n_w = 0.f, n_dl = 0.f;
@@ -193,82 +208,90 @@ __global__ void __launch_bounds__(kThreads, 1)
         n_dl = a.delta[((long long)b * a.L + t) * a.Hkv + g];
       }
     };
-    resolve(load_p(0));
-    int p_ahead = load_p(1);
-    for (int i = 0; i < niter; ++i) {
-      const int st = i & 1;
-      const int c_row = n_row, c_p = n_p;
-      const float c_w = n_w, c_dl = n_dl;
-      resolve(p_ahead);
-      p_ahead = load_p(i + 2);
-      // cp.async path: publish tile i-1 before waiting for tile i's stage (that
-      // stage is freed by the second half of step i-2, which the MMA thread
-      // issues only after the first half of step i-1, which needs tile i-1)
-      if (i >= 1 && !a.use_tma) {
-        cp_async_wait<0>();
-        tc::fence_proxy_async_smem();
-        tc::mbar_arrive(bar(BAR_QD_FULL + ((i - 1) & 1)));
-      }
-      tc::mbar_wait(bar(BAR_QD_EMPTY + st), ((i >> 1) & 1) ^ 1, abort_flag, status);
-      if (epi <= 32) {
-        if (lane < epi) {
-          sm.slot_row[st][lane] = c_row;
-          sm.slot_p[st][lane] = c_p;
-          sm.slot_w[st][lane] = c_w;
-          sm.slot_delta[st][lane] = c_dl;
+    if (li == 0 || a.use_tma) {
+      int ip_cur = load_ip(0), ip_next = load_ip(1);
+      resolve(load_p(0));
+      int p_ahead = load_p(1);
+      for (int i = 0; i < niter; ++i) {
+        const int st = i & 1;
+        const int yi = row_of(ip_cur);
+        ip_cur = ip_next;
+        ip_next = load_ip(i + 2);
+        const int c_row = n_row, c_p = n_p;
+        const float c_w = n_w, c_dl = n_dl;
+        resolve(p_ahead);
+        p_ahead = load_p(i + 2);
+        // cp.async path: publish tile i-1 before waiting for tile i's stage (that
+        // stage is freed by the dK/dV products of step i-2, which the MMA thread
+        // issues only after S/dP' of step i-1, which needs tile i-1)
+        if (i >= 1 && !a.use_tma) {
+          cp_async_wait<0>();
+          tc::fence_proxy_async_smem();
+          tc::mbar_arrive(bar(BAR_QD_FULL + ((i - 1) & 1)));
         }
-      } else {
-        for (int sl = lane; sl < epi; sl += 32) {
-          const int e = i * epi + sl;
-          int row = -1, p = -1;
-          float wv = 0.f, dl = 0.f;
-          if (e < cnt) {
-            p = a.entries[off + e];
-            const int t = (p / slot_div) % a.L;
-            row = ((b * a.L + t) * a.Hq) + g * a.G;
-            wv = a.w[p];
-            dl = a.delta[((long long)b * a.L + t) * a.Hkv + g];
+        tc::mbar_wait(bar(BAR_QD_EMPTY + st), ((i >> 1) & 1) ^ 1, abort_flag, status);
+        if (li == 0) {
+          if (epi <= 32) {
+            if (lane < epi) {
+              sm.slot_row[st][lane] = c_row;
+              sm.slot_p[st][lane] = c_p;
+              sm.slot_w[st][lane] = c_w;
+              sm.slot_delta[st][lane] = c_dl;
+            }
+          } else {
+            for (int sl = lane; sl < epi; sl += 32) {
+              const int e = i * epi + sl;
+              int row = -1, p = -1;
+              float wv = 0.f, dl = 0.f;
+              if (e < cnt) {
+                p = a.entries[off + e];
+                const int t = (p / slot_div) % a.L;
+                row = ((b * a.L + t) * a.Hq) + g * a.G;
+                wv = a.w[p];
+                dl = a.delta[((long long)b * a.L + t) * a.Hkv + g];
+              }
+              sm.slot_row[st][sl] = row;
+              sm.slot_p[st][sl] = p;
+              sm.slot_w[st][sl] = wv;
+              sm.slot_delta[st][sl] = dl;
+            }
           }
-          sm.slot_row[st][sl] = row;
-          sm.slot_p[st][sl] = p;
-          sm.slot_w[st][sl] = wv;
-          sm.slot_delta[st][sl] = dl;
         }
-      }
-      const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
-      if (a.use_tma) {
-        // lane l < epi gathers slot l's G rows of q (one box per 8-row
-        // group); this warp's expected arrival carries the byte count and
-        // publishes the slot tables written above (warp 10 brings dO)
-        if (lane < epi) {
-          const int y = c_row >= 0 ? c_row : a.n_rows;  // past the list: zeros
-          for (int j = 0; j < (a.G >> 3); ++j)
-            tc::tma_load_3d(qb + (lane * (a.G >> 3) + j) * (16 * D), &tmap_q, 0, y + 8 * j, 0, bar(BAR_QD_FULL + st));
+        const uint32_t qb = smem_u32(sm.Q[st]), ob = smem_u32(sm.dO[st]);
+        if (a.use_tma) {
+          // one box per 8-row group of the lane's item; each loader's expected
+          // arrival carries its byte count (warp 8's also publishes the tables)
+          if (has_item) {
+            const uint32_t dst = (item < epi ? qb : ob) + islot * (a.G >> 3) * (16 * D);
+            const CUtensorMap* m = item < epi ? &tmap_q : &tmap_do;
+            for (int j = 0; j < (a.G >> 3); ++j)
+              tc::tma_load_3d(dst + j * (16 * D), m, 0, yi + 8 * j, 0, bar(BAR_QD_FULL + st));
+          }
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), item_bytes);
+          continue;
         }
         __syncwarp();
-        if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), kRows * D * 2);
-        continue;
-      }
-      __syncwarp();
-      for (int u = lane; u < kRows * D8; u += 32) {
-        const int r = u / D8, ch = u % D8;
-        const int row = sm.slot_row[st][r >> a.log2G];
-        const uint32_t o = tc::grp_offset(D, r, ch * 8);
-        if (row >= 0) {
-          const long long src = ((long long)(row + (r & (a.G - 1)))) * D + ch * 8;
-          cp_async16(qb + o, a.q + src);
-          cp_async16(ob + o, a.dO + src);
-        } else {
-          asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(qb + o), "r"(0));
-          asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(ob + o), "r"(0));
+        for (int u = lane; u < kRows * D8; u += 32) {
+          const int r = u / D8, ch = u % D8;
+          const int row = sm.slot_row[st][r >> a.log2G];
+          const uint32_t o = tc::grp_offset(D, r, ch * 8);
+          if (row >= 0) {
+            const long long src = ((long long)(row + (r & (a.G - 1)))) * D + ch * 8;
+            cp_async16(qb + o, a.q + src);
+            cp_async16(ob + o, a.dO + src);
+          } else {
+            asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(qb + o), "r"(0));
+            asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(ob + o), "r"(0));
+          }
         }
+        cp_async_commit();
       }
-      cp_async_commit();
-    }
-    if (!a.use_tma) {
-      cp_async_wait<0>();
-      tc::fence_proxy_async_smem();
-      tc::mbar_arrive(bar(BAR_QD_FULL + ((niter - 1) & 1)));
+      if (!a.use_tma) {
+        cp_async_wait<0>();
+        tc::fence_proxy_async_smem();
+        tc::mbar_arrive(bar(BAR_QD_FULL + ((niter - 1) & 1)));
+      }
     }
   } else if (warp == 9) {
     // ---------------------------------------------------------------- MMA issue (one thread)
@@ -354,32 +377,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mma_commit(bar(BAR_ACC_DONE));
     }
     __syncwarp();
-  } else if (warp == 10) {
-    // ---------------------------------------------------------------- second loader warp (TMA path: dO)
-    if (a.use_tma) {
-      auto load_p = [&](int i) {
-        const int e = i * epi + lane;
-        return (lane < epi && e < cnt) ? a.entries[off + e] : -1;
-      };
-      auto row_of = [&](int p) {  // past the list: rows past the tensor read zeros
-        return p < 0 ? a.n_rows : ((b * a.L + (p / slot_div) % a.L) * a.Hq) + g * a.G;
-      };
-      int p_cur = load_p(0), p_next = load_p(1);
-      for (int i = 0; i < niter; ++i) {
-        const int st = i & 1;
-        const int y = row_of(p_cur);
-        p_cur = p_next;
-        p_next = load_p(i + 2);
-        tc::mbar_wait(bar(BAR_QD_EMPTY + st), ((i >> 1) & 1) ^ 1, abort_flag, status);
-        const uint32_t ob = smem_u32(sm.dO[st]);
-        if (lane < epi) {
-          for (int j = 0; j < (a.G >> 3); ++j)
-            tc::tma_load_3d(ob + (lane * (a.G >> 3) + j) * (16 * D), &tmap_do, 0, y + 8 * j, 0, bar(BAR_QD_FULL + st));
-        }
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), kRows * D * 2);
-      }
-    }
   } else if (warp < 4) {
     // ---------------------------------------------------------------- softmax / gradient rows (thread = row)
     const int r = tid;

@@ -20,7 +20,8 @@ namespace {
 
 constexpr int kRows = 128;     // query rows per step (tensor-core M)
 constexpr int kQStages = 3;    // gathered query tiles in flight
-constexpr int kThreads = 320;  // warps 0-3 softmax, 4-7 epilogue, 8 loader, 9 MMA
+constexpr int kThreads = 384;  // warps 0-3 softmax, 4-7 epilogue, 8, 10, 11 loaders, 9 MMA
+constexpr int kLoaders = 3;    // a TMA issue costs the issuing warp tens of ns per box: spread the boxes
 constexpr int kTmemCols = 512;
 
 __device__ unsigned g_fwd_status;
@@ -83,7 +84,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (tid == 0) {
     for (int i = 0; i < 3; ++i) {
-      tc::mbar_init(bar(BAR_Q_FULL + i), a.use_tma ? 1 : 32);
+      tc::mbar_init(bar(BAR_Q_FULL + i), a.use_tma ? kLoaders : 32);
       tc::mbar_init(bar(BAR_Q_EMPTY + i), 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -120,68 +121,76 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::fence_after_sync();
   const uint32_t tmem = sm.tmem_base;
 
-  if (warp == 8) {
-    // ---------------------------------------------------------------- loader warp
-    // TMA path: the slot ids of a tile are loaded two tiles ahead and turned
-    // into query rows one tile ahead, so no dependent global load sits on the
-    // loader's critical path.
-    auto load_p = [&](int i) {
-      const int e = i * epi + lane;
-      return (a.use_tma && lane < epi && e < cnt) ? a.entries[off + e] : -1;
-    };
-    auto row_of = [&](int p) {  // past the list: rows past the tensor read zeros
-      return p < 0 ? a.n_rows : ((b * a.L + (p / slot_div) % a.L) * a.Hq) + g * a.G;
-    };
-    int p_cur = load_p(0), p_next = load_p(1);
-    for (int i = 0; i < niter; ++i) {
-      const int st = i % kQStages;
-      const int y = row_of(p_cur);
-      p_cur = p_next;
-      p_next = load_p(i + 2);
-      tc::mbar_wait(bar(BAR_Q_EMPTY + st), ((i / kQStages) & 1) ^ 1, abort_flag, status);
-      const uint32_t base = smem_u32(sm.Q[st]);
-      if (a.use_tma) {
-        // lane l < epi gathers slot l's G rows, one box per 8-row group; the
-        // single expected arrival carries the byte count
-        if (lane < epi) {
-          for (int j = 0; j < (a.G >> 3); ++j)
-            tc::tma_load_3d(base + (lane * (a.G >> 3) + j) * (16 * D), &tmap_q, 0, y + 8 * j, 0, bar(BAR_Q_FULL + st));
+  if (warp == 8 || warp >= 10) {
+    // ---------------------------------------------------------------- loader warps
+    // TMA path: loader li (warps 8, 10, 11) gathers the slots li, li + 3, ...
+    // of every tile, lane l slot li + 3 l. The slot ids of a tile are loaded
+    // two tiles ahead and turned into query rows one tile ahead, so no
+    // dependent global load sits on the loader's critical path. The cp.async
+    // path runs on warp 8 alone.
+    const int li = warp == 8 ? 0 : warp - 9;
+    if (li == 0 || a.use_tma) {
+      const int my_slot = li + kLoaders * lane;
+      const int my_slots = (epi - li + kLoaders - 1) / kLoaders;
+      auto load_p = [&](int i) {
+        const int e = i * epi + my_slot;
+        return (a.use_tma && my_slot < epi && e < cnt) ? a.entries[off + e] : -1;
+      };
+      auto row_of = [&](int p) {  // past the list: rows past the tensor read zeros
+        return p < 0 ? a.n_rows : ((b * a.L + (p / slot_div) % a.L) * a.Hq) + g * a.G;
+      };
+      int p_cur = load_p(0), p_next = load_p(1);
+      for (int i = 0; i < niter; ++i) {
+        const int st = i % kQStages;
+        const int y = row_of(p_cur);
+        p_cur = p_next;
+        p_next = load_p(i + 2);
+        tc::mbar_wait(bar(BAR_Q_EMPTY + st), ((i / kQStages) & 1) ^ 1, abort_flag, status);
+        const uint32_t base = smem_u32(sm.Q[st]);
+        if (a.use_tma) {
+          // one box per 8-row group of the lane's slot; each loader's expected
+          // arrival carries its byte count
+          if (my_slot < epi) {
+            for (int j = 0; j < (a.G >> 3); ++j)
+              tc::tma_load_3d(base + (my_slot * (a.G >> 3) + j) * (16 * D), &tmap_q, 0, y + 8 * j, 0,
+                              bar(BAR_Q_FULL + st));
+          }
+          if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_Q_FULL + st), my_slots * a.G * D * 2);
+          continue;
         }
-        if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_Q_FULL + st), kRows * D * 2);
-        continue;
-      }
-      for (int sl = lane; sl < epi; sl += 32) {
-        const int e = i * epi + sl;
-        int row = -1;
-        if (e < cnt) {
-          const int p = a.entries[off + e];
-          const int t = (p / slot_div) % a.L;
-          row = ((b * a.L + t) * a.Hq) + g * a.G;
+        for (int sl = lane; sl < epi; sl += 32) {
+          const int e = i * epi + sl;
+          int row = -1;
+          if (e < cnt) {
+            const int p = a.entries[off + e];
+            const int t = (p / slot_div) % a.L;
+            row = ((b * a.L + t) * a.Hq) + g * a.G;
+          }
+          sm.slot_row[st][sl] = row;
         }
-        sm.slot_row[st][sl] = row;
-      }
-      __syncwarp();
-      for (int u = lane; u < kRows * D8; u += 32) {
-        const int r = u / D8, ch = u % D8;
-        const int row = sm.slot_row[st][r >> a.log2G];
-        const uint32_t dst = base + tc::grp_offset(D, r, ch * 8);
-        if (row >= 0) {
-          cp_async16(dst, a.q + ((long long)(row + (r & (a.G - 1)))) * D + ch * 8);
-        } else {
-          asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(dst), "r"(0));
+        __syncwarp();
+        for (int u = lane; u < kRows * D8; u += 32) {
+          const int r = u / D8, ch = u % D8;
+          const int row = sm.slot_row[st][r >> a.log2G];
+          const uint32_t dst = base + tc::grp_offset(D, r, ch * 8);
+          if (row >= 0) {
+            cp_async16(dst, a.q + ((long long)(row + (r & (a.G - 1)))) * D + ch * 8);
+          } else {
+            asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};\n" ::"r"(dst), "r"(0));
+          }
+        }
+        cp_async_commit();
+        if (i >= 1) {
+          cp_async_wait<1>();
+          tc::fence_proxy_async_smem();
+          tc::mbar_arrive(bar(BAR_Q_FULL + (i - 1) % kQStages));
         }
       }
-      cp_async_commit();
-      if (i >= 1) {
-        cp_async_wait<1>();
+      if (!a.use_tma) {
+        cp_async_wait<0>();
         tc::fence_proxy_async_smem();
-        tc::mbar_arrive(bar(BAR_Q_FULL + (i - 1) % kQStages));
+        tc::mbar_arrive(bar(BAR_Q_FULL + (niter - 1) % kQStages));
       }
-    }
-    if (!a.use_tma) {
-      cp_async_wait<0>();
-      tc::fence_proxy_async_smem();
-      tc::mbar_arrive(bar(BAR_Q_FULL + (niter - 1) % kQStages));
     }
   } else if (warp == 9) {
     // ---------------------------------------------------------------- MMA issue (one thread)

@@ -69,6 +69,9 @@ struct BwdSmem {
   int abort_flag;
 };
 
+// one block per SM: the layout plus the 1024-byte alignment slack must fit the 227 KB opt-in limit
+static_assert(sizeof(BwdSmem<128>) + 1024 <= 232448, "shared memory layout too large");
+
 enum {
   BAR_QD_FULL = 0,   // 2: Q and dO tiles landed
   BAR_QD_EMPTY = 2,  // 2: every MMA reading the tiles finished (commit)
@@ -186,6 +189,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool has_item = a.use_tma && item < 2 * epi;
     const int islot = item < epi ? item : item - epi;
     const uint32_t item_bytes = (uint32_t)((2 * epi - li + kLoaders - 1) / kLoaders) * a.G * D * 2;
+    const uint64_t keep = tc::l2_evict_last();
     auto load_ip = [&](int i) {
       const int e = i * epi + islot;
       return (has_item && e < cnt) ? a.entries[off + e] : -1;
@@ -265,7 +269,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t dst = (item < epi ? qb : ob) + islot * (a.G >> 3) * (16 * D);
             const CUtensorMap* m = item < epi ? &tmap_q : &tmap_do;
             for (int j = 0; j < (a.G >> 3); ++j)
-              tc::tma_load_3d(dst + j * (16 * D), m, 0, yi + 8 * j, 0, bar(BAR_QD_FULL + st));
+              tc::tma_load_3d_hint(dst + j * (16 * D), m, 0, yi + 8 * j, 0, bar(BAR_QD_FULL + st), keep);
           }
           __syncwarp();
           if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_QD_FULL + st), item_bytes);
@@ -351,7 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // step nQ (dq accumulator read). Neither barrier can run a phase past the
       // one polled before the corresponding issue, so parity polling is exact.
       int nS = 0, nK = 0, nQ = 0;
-      unsigned long long t0 = tc::globaltimer();
+      tc::SpinLimit spin;
       while (nQ < niter) {
         bool progressed = false;
         if (nS < niter && nS < nQ + 2 && tc::mbar_test_wait(bar(BAR_QD_FULL + (nS & 1)), (nS >> 1) & 1) &&
@@ -369,8 +373,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           progressed = true;
         }
         if (progressed) {
-          t0 = tc::globaltimer();
-        } else if (!tc::within_limit(t0, abort_flag, status)) {
+          spin.busy();
+        } else if (!spin.idle(abort_flag, status)) {
           break;
         }
       }
@@ -457,6 +461,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------------- epilogue (thread = row, then head dim)
     const int r = tid - 128;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    const uint64_t stream = tc::l2_evict_first();
     for (int j = 0; j < niter; ++j) {
       tc::mbar_wait(bar(BAR_DS_FULL + j % 3), (j / 3) & 1, abort_flag, status);
       const int pj = sm.row_p[j % 3][r];
@@ -490,7 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::fence_proxy_async_smem();
           __syncwarp();
           if (issuer) {
-            tc::tma_store_2d(&tmap_dq, h * 64, pj * a.G + (r & (a.G - 1)), atom);
+            tc::tma_store_2d_hint(&tmap_dq, h * 64, pj * a.G + (r & (a.G - 1)), atom, stream);
             tc::bulk_commit();
           }
         }

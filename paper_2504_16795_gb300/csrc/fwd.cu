@@ -7,7 +7,8 @@
 // rows of every selection slot that chose the chunk (from the inverse index),
 // 128 rows (= 128/G slots of G heads) per step, through two small dense
 // tensor-core products: S = Q K^T (128 x 64 x d) and O' = softmax(S) V
-// (128 x d x 64). Each chunk is complete, so its softmax needs no online
+// (128 x d x 64), the probabilities going back into tensor memory as the A
+// operand of the second product (no shared-memory round trip). Each chunk is complete, so its softmax needs no online
 // rescaling. The normalised per-slot result O' (bf16) goes to a workspace
 // and a second kernel forms O_t = sum_j w_j O'_{t,j} with the chunk weights
 // w = softmax_j(s_sel) (the "w/o s.b." variant of §4.1), slots in order j.
@@ -31,20 +32,22 @@ struct FwdSmem {
   uint16_t Q[kQStages][kRows * D];  // gathered query rows, grouped K-major SW128 (tc::grp_offset)
   uint16_t K[kChunk * D];           // chunk keys [s][d]
   uint16_t Vt[D * kChunk];          // chunk values transposed [d][s]
-  uint16_t P[2][kRows * kChunk];    // normalised probabilities (bf16)
-  uint16_t Ostage[kRows * D];       // TMA path: the step's O' rows (grouped layout) on their way out
+  uint16_t Ostage[2][kRows * D];    // TMA path: a step's O' rows (grouped layout) on their way out, two steps
   int slot_row[kQStages][kRows];    // cp.async path: first q row of each slot (-1: past the list)
   uint64_t bar[16];
   uint32_t tmem_base;
   int abort_flag;
 };
 
+// one block per SM: the layout plus the 1024-byte alignment slack must fit the 227 KB opt-in limit
+static_assert(sizeof(FwdSmem<128>) + 1024 <= 232448, "shared memory layout too large");
+
 enum {
   BAR_Q_FULL = 0,   // 3: tile landed
   BAR_Q_EMPTY = 3,  // 3: S MMA of the tile finished (commit)
   BAR_S_FULL = 6,   // 2: S accumulator ready (commit)
   BAR_S_EMPTY = 8,  // 2: S read by the softmax warps (128 arrivals)
-  BAR_P_FULL = 10,  // 2: P tile written (128 arrivals)
+  BAR_P_FULL = 10,  // 2: P written to tensor memory (128 arrivals)
   BAR_O_FULL = 12,  // 2: O accumulator ready (commit)
   BAR_O_EMPTY = 14  // 2: O read by the epilogue warps (128 arrivals)
 };
@@ -68,6 +71,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ unsigned char smem_raw[];
   FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
+  constexpr uint32_t kColP = 2 * kChunk + 2 * D;  // tensor memory: S x2 | O' x2 | P x2 (32 columns each)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int key = blockIdx.x;
   const int c = key % a.Nc, bg = key / a.Nc;
@@ -132,6 +136,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (li == 0 || a.use_tma) {
       const int my_slot = li + kLoaders * lane;
       const int my_slots = (epi - li + kLoaders - 1) / kLoaders;
+      const uint64_t keep = tc::l2_evict_last();
       auto load_p = [&](int i) {
         const int e = i * epi + my_slot;
         return (a.use_tma && my_slot < epi && e < cnt) ? a.entries[off + e] : -1;
@@ -152,8 +157,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           // arrival carries its byte count
           if (my_slot < epi) {
             for (int j = 0; j < (a.G >> 3); ++j)
-              tc::tma_load_3d(base + (my_slot * (a.G >> 3) + j) * (16 * D), &tmap_q, 0, y + 8 * j, 0,
-                              bar(BAR_Q_FULL + st));
+              tc::tma_load_3d_hint(base + (my_slot * (a.G >> 3) + j) * (16 * D), &tmap_q, 0, y + 8 * j, 0,
+                                   bar(BAR_Q_FULL + st), keep);
           }
           if (lane == 0) tc::mbar_arrive_expect_tx(bar(BAR_Q_FULL + st), my_slots * a.G * D * 2);
           continue;
@@ -214,10 +219,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue_O = [&](int i) {
         const int pb = i & 1;
         tc::fence_after_sync();
-        const uint32_t pbase = smem_u32(sm.P[pb]);
 #pragma unroll
         for (int kk = 0; kk < kChunk / 16; ++kk)
-          tc::mma_bf16_ss(tmem + 2 * kChunk + pb * D, tc::sdesc_sw128(pbase + kk * 32),
+          tc::mma_bf16_ts(tmem + 2 * kChunk + pb * D, tmem + kColP + pb * (kChunk / 2) + kk * 8,
                           tc::sdesc_sw128(vbase + kk * 32), idO, kk > 0);
         tc::mma_commit(bar(BAR_O_FULL + pb));
       };
@@ -225,7 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // nO (P written, O buffer read), whichever is ready. Neither barrier can
       // run a phase past the polled one before the corresponding issue.
       int nS = 0, nO = 0;
-      unsigned long long t0 = tc::globaltimer();
+      tc::SpinLimit spin;
       while (nO < niter) {
         bool progressed = false;
         if (nS < niter && nS < nO + 2 && tc::mbar_test_wait(bar(BAR_Q_FULL + nS % kQStages), (nS / kQStages) & 1) &&
@@ -239,8 +243,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           progressed = true;
         }
         if (progressed) {
-          t0 = tc::globaltimer();
-        } else if (!tc::within_limit(t0, abort_flag, status)) {
+          spin.busy();
+        } else if (!spin.idle(abort_flag, status)) {
           break;
         }
       }
@@ -275,17 +279,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         zz[k & 7] += x[k];
       }
       const float inv = 1.f / (((zz[0] + zz[1]) + (zz[2] + zz[3])) + ((zz[4] + zz[5]) + (zz[6] + zz[7])));
-      const uint32_t prow = smem_u32(sm.P[sb]);
+      // P into tensor memory: the row's 64 probabilities as 32 bf16 pairs
+      uint32_t pk[kChunk / 2];
 #pragma unroll
-      for (int c16 = 0; c16 < 8; ++c16) {
-        const uint32_t dst = prow + tc::sw128_offset(kRows, r, c16 * 8);
-        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(dst),
-                     "r"(pack_bf16x2(x[8 * c16] * inv, x[8 * c16 + 1] * inv)),
-                     "r"(pack_bf16x2(x[8 * c16 + 2] * inv, x[8 * c16 + 3] * inv)),
-                     "r"(pack_bf16x2(x[8 * c16 + 4] * inv, x[8 * c16 + 5] * inv)),
-                     "r"(pack_bf16x2(x[8 * c16 + 6] * inv, x[8 * c16 + 7] * inv)));
-      }
-      tc::fence_proxy_async_smem();
+      for (int k2 = 0; k2 < kChunk / 2; ++k2) pk[k2] = pack_bf16x2(x[2 * k2] * inv, x[2 * k2 + 1] * inv);
+      tc::tmem_st32(tmem + lane_base + kColP + sb * (kChunk / 2), pk);
+      tc::tmem_wait_st();
+      tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_P_FULL + sb));
     }
   } else {
@@ -296,35 +296,37 @@ __global__ void __launch_bounds__(kThreads, 1)
     // (swizzled, conflict-free) and the first lane of every slot stores the
     // slot's G rows with one TMA box per 8 rows. Otherwise rows go out directly.
     const bool issuer = a.use_tma && (r & (a.G - 1)) == 0;
-    const uint32_t stage = smem_u32(sm.Ostage);
+    const uint64_t stream = tc::l2_evict_first();
     int p_next = r >> a.log2G < cnt ? a.entries[off + (r >> a.log2G)] : -1;
     for (int j = 0; j < niter; ++j) {
       const int pj = p_next;
       const int en = (j + 1) * epi + (r >> a.log2G);
       p_next = en < cnt ? a.entries[off + en] : -1;  // prefetch the next step's slot
       const int ob = j & 1;
-      if (a.use_tma) {  // the previous step's stores have read this warp's part of the staging tile
-        if (issuer) tc::bulk_wait_read();
+      const uint32_t stage = smem_u32(sm.Ostage[ob]);
+      if (a.use_tma) {  // the stores of step j-2 have read this warp's part of the staging tile
+        if (issuer) tc::bulk_wait_read_but1();
         __syncwarp();
       }
       tc::mbar_wait(bar(BAR_O_FULL + ob), (j >> 1) & 1, abort_flag, status);
       tc::fence_after_sync();
       uint16_t* dst = (!a.use_tma && pj >= 0) ? a.Opart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
 #pragma unroll
-      for (int h = 0; h < D / 32; ++h) {
-        float o[32];
-        tc::tmem_ld32(tmem + lane_base + 2 * kChunk + ob * D + h * 32, o);
+      for (int h = 0; h < D / 64; ++h) {  // 64 columns per tensor-memory wait
+        float o[64];
+        tc::tmem_ld32(tmem + lane_base + 2 * kChunk + ob * D + h * 64, *reinterpret_cast<float(*)[32]>(&o[0]));
+        tc::tmem_ld32(tmem + lane_base + 2 * kChunk + ob * D + h * 64 + 32, *reinterpret_cast<float(*)[32]>(&o[32]));
         tc::tmem_wait_ld();
 #pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
+        for (int q4 = 0; q4 < 8; ++q4) {
           const uint4 v = make_uint4(pack_bf16x2(o[8 * q4], o[8 * q4 + 1]), pack_bf16x2(o[8 * q4 + 2], o[8 * q4 + 3]),
                                      pack_bf16x2(o[8 * q4 + 4], o[8 * q4 + 5]),
                                      pack_bf16x2(o[8 * q4 + 6], o[8 * q4 + 7]));
           if (a.use_tma) {
-            asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(stage + tc::grp_offset(D, r, h * 32 + 8 * q4)),
+            asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(stage + tc::grp_offset(D, r, h * 64 + 8 * q4)),
                          "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w));
           } else if (dst) {
-            reinterpret_cast<uint4*>(dst + h * 32)[q4] = v;
+            reinterpret_cast<uint4*>(dst + h * 64)[q4] = v;
           }
         }
       }
@@ -333,9 +335,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (a.use_tma) {
         tc::fence_proxy_async_smem();
         __syncwarp();
-        if (issuer && pj >= 0) {
-          for (int jj = 0; jj < (a.G >> 3); ++jj)
-            tc::tma_store_3d(&tmap_o, 0, pj * a.G + 8 * jj, 0, stage + ((r >> 3) + jj) * (16 * D));
+        if (issuer) {  // one bulk group per step, empty past the list, so "all but the last" means step j-2
+          if (pj >= 0)
+            for (int jj = 0; jj < (a.G >> 3); ++jj)
+              tc::tma_store_3d_hint(&tmap_o, 0, pj * a.G + 8 * jj, 0, stage + ((r >> 3) + jj) * (16 * D), stream);
           tc::bulk_commit();
         }
       }

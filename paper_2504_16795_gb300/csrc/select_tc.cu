@@ -83,6 +83,9 @@ struct SelTcSmem {
   uint32_t tmem_base;
   int abort_flag;
 };
+// the rescoring stages 32 fp32 K̄ rows per scan warp in A and B
+static_assert(sizeof(SelTcSmem<128, 8>::A) + sizeof(SelTcSmem<128, 8>::B) >= 4 * 32 * 128 * 4, "staging");
+static_assert(sizeof(SelTcSmem<64, 8>::A) + sizeof(SelTcSmem<64, 8>::B) >= 4 * 32 * 64 * 4, "staging");
 
 struct SelTcArgs {
   const float* qh32t;     // [B*Hkv, D, Lp] fp32 q̂, transposed (tokens adjacent)
@@ -119,6 +122,44 @@ __device__ __forceinline__ float pick32(const float (&x)[32], int c) {
 #pragma unroll
   for (int i = 0; i < 2; ++i) t[i] = (c & 8) ? t[2 * i + 1] : t[2 * i];
   return (c & 16) ? t[1] : t[0];
+}
+
+// Exact rescoring in shared memory. Each lane of a warp names one chunk (c < 0:
+// none); the warp copies the 32 fp32 K̄ rows with coalesced 16-byte cp.async
+// (lane j brings float4 j of every row) into `stage`, row l at l * D floats
+// with float4 j at slot j ^ (l & 7), so that the lanes' reads of their own
+// rows below hit distinct banks.
+template <int D>
+__device__ __forceinline__ void stage_kbar_rows(uint32_t stage, const float* kb, long long row_stride, int c,
+                                                int lane) {
+#pragma unroll 4
+  for (int l = 0; l < 32; ++l) {
+    const int cl = __shfl_sync(0xFFFFFFFFu, c, l);
+    if (cl >= 0 && lane < D / 4)
+      cp_async16(stage + (uint32_t)(l * D + ((lane ^ (l & 7)) << 2)) * 4u, kb + (long long)cl * row_stride + lane * 4);
+  }
+  cp_async_commit();
+  cp_async_wait<0>();
+  __syncwarp();
+}
+// The exact chain of the selection score over the lane's staged row: fused
+// multiply-adds in element order from 0 (the caller scales by c_sel).
+template <int D>
+__device__ __forceinline__ float staged_dot(const float (&q)[D], uint32_t stage, int lane) {
+  const uint32_t row = stage + (uint32_t)(lane * D) * 4u;
+  float acc = 0.f;
+#pragma unroll
+  for (int j = 0; j < D / 4; ++j) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(row + ((uint32_t)(j ^ (lane & 7)) << 4)));
+    acc = fmaf(q[4 * j], v.x, acc);
+    acc = fmaf(q[4 * j + 1], v.y, acc);
+    acc = fmaf(q[4 * j + 2], v.z, acc);
+    acc = fmaf(q[4 * j + 3], v.w, acc);
+  }
+  return acc;
 }
 
 template <int D, int KT, bool DEC>
@@ -390,7 +431,29 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       for (int j = 0; j < cnt; ++j)
         if (sm.bu[j][r] >= lam_keep) sm.bi[nc++][r] = sm.bi[j][r];
     const bool q_ok = ntiles == 0 || tc::mbar_wait(bar(BAR_Q32), 0, abort_flag, status);
-    if (t < a.L && q_ok && !*abort_flag) {
+    const bool live = t < a.L && q_ok && !*abort_flag;
+    // the row's fp32 q̂ into registers (element e at qs[e * kTok]; a warp's rows
+    // are adjacent words), after which the scan warps reuse A and B as staging
+    float qr[D];
+    {
+      const float* qs = reinterpret_cast<const float*>(sm.A) + r;
+#pragma unroll
+      for (int e = 0; e < D; ++e) qr[e] = qs[e * kTok];
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    {
+      const int my_n = (live && !overflow) ? nc : 0;
+      const int rounds = __reduce_max_sync(0xFFFFFFFFu, (unsigned)my_n);
+      const float* kb = a.kbar32 + ((long long)b * a.Nc * a.Hkv + g) * D;
+      const uint32_t stage = abase + (uint32_t)(warp * 32 * D) * 4u;  // 32 rows per warp inside A and B
+      for (int j = 0; j < rounds; ++j) {
+        const int c = j < my_n ? sm.bi[j][r] : -1;
+        stage_kbar_rows<D>(stage, kb, (long long)a.Hkv * D, c, lane);
+        if (c >= 0) sm.bl[j][r] = staged_dot<D>(qr, stage, lane) * a.scale_sel;
+        __syncwarp();
+      }
+    }
+    if (live) {
       const long long p = ((long long)b * a.L + t) * a.Hkv + g;
       int32_t* out_i = a.idx + p * a.topk;
       float* out_s = a.s_sel + p * a.topk;
@@ -399,30 +462,6 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
         a.flags[atomicAdd(a.nflag, 1u)] = (int32_t)p;
       } else {
         unsigned long long(*chosen)[kTok] = sm.chosen;
-        // q̂ of this row: element e at qs[e * kTok] (a warp's rows are adjacent words)
-        const float* qs = reinterpret_cast<const float*>(sm.A) + r;
-        const float* kb = a.kbar32 + ((long long)b * a.Nc * a.Hkv + g) * D;
-        // one candidate at a time: each lane streams one K̄ row, 128 bytes
-        // (eight float4) per step, so a warp keeps 4 KB of lines live in L1
-        for (int j = 0; j < nc; ++j) {
-          const float4* k4 = reinterpret_cast<const float4*>(kb + (long long)sm.bi[j][r] * a.Hkv * D);
-          float acc = 0.f;
-#pragma unroll 1
-          for (int e8 = 0; e8 < D / 32; ++e8) {
-            float4 kv[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u) kv[u] = __ldg(k4 + e8 * 8 + u);
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-              const int e = e8 * 32 + 4 * u;
-              acc = fmaf(qs[e * kTok], kv[u].x, acc);
-              acc = fmaf(qs[(e + 1) * kTok], kv[u].y, acc);
-              acc = fmaf(qs[(e + 2) * kTok], kv[u].z, acc);
-              acc = fmaf(qs[(e + 3) * kTok], kv[u].w, acc);
-            }
-          }
-          sm.bl[j][r] = acc * a.scale_sel;
-        }
         // the keff largest keys (keys are distinct: they carry the chunk index)
         unsigned long long prev = ~0ull;
         for (int s = 0; s < keff; ++s) {
@@ -553,20 +592,25 @@ __global__ void __launch_bounds__(256) sel_kbar_kernel(const float* __restrict__
   }
 }
 
-// Exact pass for the rows whose candidate buffer overflowed: one warp per row,
-// lanes over chunks, the exact fp32 score chain and a warp-held top-k list.
+// Rows whose candidate buffer could not be certified: every visible chunk is
+// scored with the exact chain. One block per flagged row (grid-stride); its
+// eight warps take 32 chunks at a time, staging the fp32 K̄ rows in shared
+// memory with coalesced copies, and keep running top-k lists that warp 0
+// merges at the end.
+constexpr int kExactWarps = 8;
 template <int D>
-__global__ void __launch_bounds__(256) sel_exact_rows_kernel(const float* __restrict__ qh32t,
-                                                             const float* __restrict__ kbar32,
-                                                             const unsigned* __restrict__ nflag,
-                                                             const int32_t* __restrict__ flags,
-                                                             int32_t* __restrict__ idx, float* __restrict__ s_sel,
-                                                             int L, int Lp, int Hkv, int Nc, int topk,
-                                                             float scale_sel) {
-  __shared__ float qs[8][D];
+__global__ void __launch_bounds__(kExactWarps * 32) sel_exact_rows_kernel(
+    const float* __restrict__ qh32t, const float* __restrict__ kbar32, const unsigned* __restrict__ nflag,
+    const int32_t* __restrict__ flags, int32_t* __restrict__ idx, float* __restrict__ s_sel, int L, int Lp, int Hkv,
+    int Nc, int topk, float scale_sel) {
+  extern __shared__ __align__(16) unsigned char ex_smem[];
+  float* stage_all = reinterpret_cast<float*>(ex_smem);                    // [warps][32 rows][D]
+  float* qsh = stage_all + kExactWarps * 32 * D;                             // [D]
+  unsigned long long* lists = reinterpret_cast<unsigned long long*>(qsh + D);  // [warps][32]
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  const uint32_t stage = smem_u32(stage_all + wib * 32 * D);
   const unsigned n = *nflag;
-  for (unsigned f = blockIdx.x * 8u + wib; f < n; f += gridDim.x * 8u) {
+  for (unsigned f = blockIdx.x; f < n; f += gridDim.x) {
     const long long p = flags[f];
     const int g = (int)(p % Hkv);
     const long long bt = p / Hkv;
@@ -574,29 +618,27 @@ __global__ void __launch_bounds__(256) sel_exact_rows_kernel(const float* __rest
     const long long b = bt / L;
     const int vis = min(t / kChunk, Nc);
     const float* qcol = qh32t + (b * Hkv + g) * D * Lp + t;
-    __syncwarp();
-    for (int e = lane; e < D; e += 32) qs[wib][e] = qcol[(long long)e * Lp];
-    __syncwarp();
+    for (int e = threadIdx.x; e < D; e += kExactWarps * 32) qsh[e] = qcol[(long long)e * Lp];
+    __syncthreads();
+    float qr[D];
+#pragma unroll
+    for (int e = 0; e < D; ++e) qr[e] = qsh[e];
+    const float* kb = kbar32 + (b * Nc * Hkv + g) * D;
     unsigned long long lst = 0ull;
-    for (int c0 = 0; c0 < vis; c0 += 32) {
-      const int c = c0 + lane;
-      unsigned long long key = 0ull;
-      if (c < vis) {
-        const float4* k4 = reinterpret_cast<const float4*>(kbar32 + ((b * Nc + c) * Hkv + g) * D);
-        float acc = 0.f;
-#pragma unroll 8
-        for (int e4 = 0; e4 < D / 4; ++e4) {
-          const float4 kv = __ldg(k4 + e4);
-          acc = fmaf(qs[wib][4 * e4], kv.x, acc);
-          acc = fmaf(qs[wib][4 * e4 + 1], kv.y, acc);
-          acc = fmaf(qs[wib][4 * e4 + 2], kv.z, acc);
-          acc = fmaf(qs[wib][4 * e4 + 3], kv.w, acc);
-        }
-        key = rank_key(acc * scale_sel, (uint32_t)c);
-      }
+    for (int c0 = wib * 32; c0 < vis; c0 += kExactWarps * 32) {
+      const int c = c0 + lane < vis ? c0 + lane : -1;
+      stage_kbar_rows<D>(stage, kb, (long long)Hkv * D, c, lane);
+      const unsigned long long key = c >= 0 ? rank_key(staged_dot<D>(qr, stage, lane) * scale_sel, (uint32_t)c) : 0ull;
+      __syncwarp();
       warp_topk_offer(lst, key, topk, lane);
     }
-    warp_emit_selection(lst, topk, lane, idx + p * topk, s_sel + p * topk);
+    lists[wib * 32 + lane] = lane < topk ? lst : 0ull;
+    __syncthreads();
+    if (wib == 0) {
+      for (int w = 1; w < kExactWarps; ++w) warp_topk_offer(lst, lists[w * 32 + lane], topk, lane);
+      warp_emit_selection(lst, topk, lane, idx + p * topk, s_sel + p * topk);
+    }
+    __syncthreads();
   }
 }
 
@@ -899,8 +941,12 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   sel_tc_kernel<DD, KT, false><<<(unsigned)blocks, kThreads, smem, st>>>(a, tq, tk, tq32t);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  sel_exact_rows_kernel<DD><<<2 * 152, 256, 0, st>>>(qh32, kbar32, nflag, flags, idx, s_sel, Dm.L, Lp, Dm.Hkv,
-                                                     Dm.Nc, Dm.topk, Dm.scale_sel);
+  const size_t ex_smem = ((size_t)kExactWarps * 32 * DD + DD) * 4 + (size_t)kExactWarps * 32 * 8;
+  if ((e = cudaFuncSetAttribute(sel_exact_rows_kernel<DD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)ex_smem)) != cudaSuccess)
+    return e;
+  sel_exact_rows_kernel<DD><<<152, kExactWarps * 32, ex_smem, st>>>(qh32, kbar32, nflag, flags, idx, s_sel, Dm.L, Lp,
+                                                                    Dm.Hkv, Dm.Nc, Dm.topk, Dm.scale_sel);
   note_launches(1);
   return cudaGetLastError();
 }

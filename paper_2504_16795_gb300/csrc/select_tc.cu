@@ -108,6 +108,7 @@ struct SelTcArgs {
   int32_t* cand_c; //                          chunk indices
   int32_t* cand_n; // [Hkv, Bq, n_split] entry count
   float* cand_d;   // [Hkv, Bq, n_split] largest upper bound the row's buffer dropped (-inf: none)
+  float4* cand_s;  // [Hkv, Bq, n_split] (lambda of the range, largest exported lower bound, largest upper bound)
 };
 
 // x[c] for a run-time c in [0, 32): a five-level select tree.
@@ -400,17 +401,22 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       if (row_ok && !*abort_flag) {
         const long long crow = ((long long)g * a.Bq + t) * a.n_split + split;
         int ne = 0;
+        float lmax = -INFINITY, umax = -INFINITY;
         for (int j = 0; j < cnt; ++j) {
           const float u = sm.bu[j][r];
           if (u >= lam_keep) {
-            a.cand_l[crow * kBuf + ne] = sm.bl[j][r];
+            const float l = sm.bl[j][r];
+            a.cand_l[crow * kBuf + ne] = l;
             a.cand_u[crow * kBuf + ne] = u;
             a.cand_c[crow * kBuf + ne] = sm.bi[j][r];
+            lmax = fmaxf(lmax, l);
+            umax = fmaxf(umax, u);
             ++ne;
           }
         }
         a.cand_n[crow] = ne;
         a.cand_d[crow] = u_drop;
+        a.cand_s[crow] = make_float4(lam_keep, lmax, umax, 0.f);
       }
     } else {
 
@@ -708,62 +714,99 @@ __device__ __forceinline__ float exact_dot(const float* __restrict__ qs, const f
 
 // Decode merge: one block (8 warps) per (query, group). lambda = the k-th
 // largest lower bound over the entries every scan block exported, at most the
-// true lambda. A block whose buffer dropped an entry with upper bound at or
-// above lambda cannot vouch for its range: those ranges are scored exactly
-// (rare). The candidates (entries with upper bound at or above lambda, and
-// the exactly scored chunks at or above it) are ranked by the exact chain,
-// (score desc, chunk index asc). Each warp keeps a top-k list over its share;
-// warp 0 combines the eight.
+// true lambda. Every range exported its own lambda and the largest lower and
+// upper bounds among its entries. lambda is at least the largest range lambda
+// (that range alone holds k chunks whose lower bounds reach it) and at least
+// the k-th largest of the ranges' largest lower bounds (k ranges hold one such
+// chunk each), so only the ranges whose bounds reach that value are read. A block whose
+// buffer dropped an entry with upper bound at or above lambda cannot vouch for
+// its range: those ranges are scored exactly (rare). The candidates (entries
+// with upper bound at or above lambda, and the exactly scored chunks at or
+// above it) are ranked by the exact chain, their K̄ rows staged in shared
+// memory 32 at a time per warp.
+constexpr int kMergeWarps = 8;
+constexpr int kMergeCand = 1024;  // listed candidates; any beyond are scored in place
+constexpr int kMaxSplit = 320;    // ranges per row (the layout keeps n_split at most 2 * 152)
 template <int D>
-__global__ void __launch_bounds__(256) dtc_merge_kernel(const float* __restrict__ cand_l,
-                                                        const float* __restrict__ cand_u,
-                                                        const int32_t* __restrict__ cand_c,
-                                                        const int32_t* __restrict__ cand_n,
-                                                        const float* __restrict__ cand_d, int kbuf,
-                                                        const float* __restrict__ qh32,
-                                                        const float* __restrict__ kbar32, int32_t* __restrict__ idx,
-                                                        float* __restrict__ s_sel, float* __restrict__ w, int Bq,
-                                                        int Hkv, int Nc, int n_split, int range, int topk,
-                                                        float scale_sel) {
-  __shared__ float qs[D];
-  __shared__ unsigned long long lists[8][32];
+__global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
+    const float* __restrict__ cand_l, const float* __restrict__ cand_u, const int32_t* __restrict__ cand_c,
+    const int32_t* __restrict__ cand_n, const float* __restrict__ cand_d, const float4* __restrict__ cand_s, int kbuf,
+    const float* __restrict__ qh32, const float* __restrict__ kbar32, int32_t* __restrict__ idx,
+    float* __restrict__ s_sel, float* __restrict__ w, int Bq, int Hkv, int Nc, int n_split, int range, int topk,
+    float scale_sel) {
+  extern __shared__ __align__(16) unsigned char mg_smem[];
+  float* stage_all = reinterpret_cast<float*>(mg_smem);  // [warps][32 rows][D]
+  float* qs = stage_all + kMergeWarps * 32 * D;           // [D]
+  int* cands = reinterpret_cast<int*>(qs + D);            // [kMergeCand]
+  __shared__ unsigned long long lists[kMergeWarps][32];
+  __shared__ float4 rs[kMaxSplit];  // per range: (lambda, largest lower bound, largest upper bound, dropped bound)
+  __shared__ int rn[kMaxSplit];     // per range: exported entries
+  __shared__ float red[kMergeWarps];
   __shared__ float lam_s;
-  __shared__ int any_unsure;
+  __shared__ int any_unsure, n_cand;
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const int row = blockIdx.x;  // b * Hkv + g
   const int b = row / Hkv, g = row % Hkv;
   const long long cbase = ((long long)g * Bq + b) * n_split;
-  if (threadIdx.x == 0) any_unsure = 0;
-  for (int e = threadIdx.x; e < D; e += 256) qs[e] = qh32[(long long)row * D + e];
+  const uint32_t stage = smem_u32(stage_all + wib * 32 * D);
+  if (threadIdx.x == 0) any_unsure = 0, n_cand = 0;
+  for (int e = threadIdx.x; e < D; e += kMergeWarps * 32) qs[e] = qh32[(long long)row * D + e];
+  // the ranges' summaries into shared memory, and the largest range lambda
+  float ls = -INFINITY;
+  for (int sp = threadIdx.x; sp < n_split; sp += kMergeWarps * 32) {
+    float4 v = cand_s[cbase + sp];
+    v.w = cand_d[cbase + sp];
+    rs[sp] = v;
+    rn[sp] = cand_n[cbase + sp];
+    ls = fmaxf(ls, v.x);
+  }
+  ls = warp_max(ls);
+  if (lane == 0) red[wib] = ls;
   __syncthreads();
-  const long long total = (long long)n_split * kbuf;  // entry slots of the row
+  if (wib == 0) {  // the k-th largest of the ranges' largest lower bounds
+    unsigned long long top = 0ull;
+    for (int sp0 = 0; sp0 < n_split; sp0 += 32) {
+      const int sp = sp0 + lane;
+      const unsigned long long key =
+          sp < n_split && rs[sp].y > -INFINITY ? ((unsigned long long)order_bits(rs[sp].y) << 32) | (uint32_t)sp : 0ull;
+      warp_topk_offer(top, key, topk, lane);
+    }
+    const unsigned long long kth = __shfl_sync(0xFFFFFFFFu, top, topk - 1);
+    if (lane == 0) lam_s = kth != 0ull ? order_bits_to_float((uint32_t)(kth >> 32)) : -INFINITY;
+  }
+  __syncthreads();
+  float lam_star = lam_s;
+#pragma unroll
+  for (int k = 0; k < kMergeWarps; ++k) lam_star = fmaxf(lam_star, red[k]);
+  __syncthreads();  // lam_s is written again below
   auto krow = [&](int c) { return kbar32 + ((long long)c * Hkv + g) * D; };
-  auto combine = [&](unsigned long long mine) {  // top-k of the eight warp lists, in warp 0
+  auto combine = [&](unsigned long long mine) {  // top-k of the warp lists, in warp 0
     lists[wib][lane] = mine;
     __syncthreads();
     unsigned long long all = 0ull;
     if (wib == 0)
-      for (int k = 0; k < 8; ++k) warp_topk_offer(all, lane < topk ? lists[k][lane] : 0ull, topk, lane);
+      for (int k = 0; k < kMergeWarps; ++k) warp_topk_offer(all, lane < topk ? lists[k][lane] : 0ull, topk, lane);
     __syncthreads();
     return all;
   };
-  // ---- lambda: every warp walks slots wib*32 + lane, step 256, four batches
-  // at a time (loads first, then the list updates)
+  // ---- lambda over the entries (at or above lam_star) of the ranges that can
+  // hold them: lanes test 32 ranges at once, then the warp walks the hits
   unsigned long long lst = 0ull;
-  for (long long base = (long long)wib * 32; base < total; base += 4 * 256) {
-    float lv[4];
-    bool ok[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const long long slot = base + u * 256 + lane;
-      ok[u] = slot < total && cand_n[cbase + slot / kbuf] > (int)(slot % kbuf);
-      lv[u] = ok[u] ? cand_l[cbase * kbuf + slot] : 0.f;
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const long long slot = base + u * 256 + lane;
-      const unsigned long long key = ok[u] ? ((unsigned long long)order_bits(lv[u]) << 32) | (uint32_t)slot : 0ull;
-      warp_topk_offer(lst, key, topk, lane);
+  for (int sp0 = wib * 32; sp0 < n_split; sp0 += kMergeWarps * 32) {
+    unsigned hits = __ballot_sync(0xFFFFFFFFu, sp0 + lane < n_split && rs[sp0 + lane].y >= lam_star);
+    while (hits) {
+      const int sp = sp0 + __ffs(hits) - 1;
+      hits &= hits - 1;
+      const int n = rn[sp];
+      for (int j0 = 0; j0 < n; j0 += 32) {
+        const int j = j0 + lane;
+        unsigned long long key = 0ull;
+        if (j < n) {
+          const float l = cand_l[(cbase + sp) * kbuf + j];
+          if (l >= lam_star) key = ((unsigned long long)order_bits(l) << 32) | (uint32_t)(sp * kbuf + j);
+        }
+        warp_topk_offer(lst, key, topk, lane);
+      }
     }
   }
   {
@@ -775,39 +818,56 @@ __global__ void __launch_bounds__(256) dtc_merge_kernel(const float* __restrict_
     __syncthreads();
   }
   const float lam = lam_s;
-  for (int sp = threadIdx.x; sp < n_split; sp += 256)
-    if (cand_d[cbase + sp] >= lam) any_unsure = 1;
+  for (int sp = threadIdx.x; sp < n_split; sp += kMergeWarps * 32)
+    if (rs[sp].w >= lam) any_unsure = 1;
+  // ---- the candidates: entries with upper bound at or above lambda, listed
+  // (past the list's capacity they are scored here, one per lane)
+  unsigned long long fin = 0ull;
+  for (int sp0 = wib * 32; sp0 < n_split; sp0 += kMergeWarps * 32) {
+    unsigned hits = __ballot_sync(0xFFFFFFFFu, sp0 + lane < n_split && rs[sp0 + lane].z >= lam);
+    while (hits) {
+      const int sp = sp0 + __ffs(hits) - 1;
+      hits &= hits - 1;
+      const int n = rn[sp];
+      for (int j0 = 0; j0 < n; j0 += 32) {
+        const int j = j0 + lane;
+        unsigned long long key = 0ull;
+        if (j < n && cand_u[(cbase + sp) * kbuf + j] >= lam) {
+          const int c = cand_c[(cbase + sp) * kbuf + j];
+          const int pos = atomicAdd(&n_cand, 1);
+          if (pos < kMergeCand)
+            cands[pos] = c;
+          else
+            key = rank_key(exact_dot<D>(qs, krow(c)) * scale_sel, (uint32_t)c);
+        }
+        warp_topk_offer(fin, key, topk, lane);
+      }
+    }
+  }
   __syncthreads();
   const bool unsure = any_unsure != 0;
-  // ---- the candidates, exactly
-  unsigned long long fin = 0ull;
-  for (long long base = (long long)wib * 32; base < total; base += 4 * 256) {
-    float uv[4];
-    bool ok[4];
+  {
+    float qr[D];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const long long slot = base + u * 256 + lane;
-      ok[u] = slot < total && cand_n[cbase + slot / kbuf] > (int)(slot % kbuf);
-      uv[u] = ok[u] ? cand_u[cbase * kbuf + slot] : -INFINITY;
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const long long slot = base + u * 256 + lane;
-      unsigned long long key = 0ull;
-      if (ok[u] && uv[u] >= lam) {
-        const int c = cand_c[cbase * kbuf + slot];
-        key = rank_key(exact_dot<D>(qs, krow(c)) * scale_sel, (uint32_t)c);
-      }
+    for (int e = 0; e < D; ++e) qr[e] = qs[e];
+    const int nlist = min(n_cand, kMergeCand);
+    for (int base = wib * 32; base < nlist; base += kMergeWarps * 32) {
+      const int i = base + lane;
+      const int c = i < nlist ? cands[i] : -1;
+      stage_kbar_rows<D>(stage, kbar32 + (long long)g * D, (long long)Hkv * D, c, lane);
+      const unsigned long long key =
+          c >= 0 ? rank_key(staged_dot<D>(qr, stage, lane) * scale_sel, (uint32_t)c) : 0ull;
+      __syncwarp();
       warp_topk_offer(fin, key, topk, lane);
     }
   }
   for (int sp = 0; unsure && sp < n_split; ++sp) {
-    if (!(cand_d[cbase + sp] >= lam)) continue;  // uniform across the block
+    if (!(rs[sp].w >= lam)) continue;  // uniform across the block
     // this range's exported entries are scored again below the whole range:
     // skip them there to keep every chunk once
     const int cb = sp * range, ce = min(cb + range, Nc);
-    const int n = cand_n[cbase + sp];
-    for (int c0 = cb + wib * 32; c0 < ce; c0 += 256) {
+    const int n = rn[sp];
+    for (int c0 = cb + wib * 32; c0 < ce; c0 += kMergeWarps * 32) {
       const int c = c0 + lane;
       unsigned long long key = 0ull;
       if (c < ce) {
@@ -976,7 +1036,7 @@ DecIndexLayout dec_index_layout(const DecodeDims& D) {
 }
 
 struct DecTcLayout {
-  size_t qh32, qh16, qn, cl, cu, cc, cn, cd, opart, total;
+  size_t qh32, qh16, qn, cl, cu, cc, cn, cd, cs, opart, total;
   int n_qt, n_split, range;
 };
 
@@ -1008,6 +1068,8 @@ DecTcLayout dec_tc_layout(const DecodeDims& D) {
   o = align256(o + rows * lo.n_split * 4);
   lo.cd = o;
   o = align256(o + rows * lo.n_split * 4);
+  lo.cs = o;
+  o = align256(o + rows * lo.n_split * 16);
   lo.opart = o;
   o = align256(o + rows * D.topk * D.G * D.d * 4);
   lo.total = o;
@@ -1060,6 +1122,7 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
   a.cand_c = (int32_t*)(base + lo.cc);
   a.cand_n = (int32_t*)(base + lo.cn);
   a.cand_d = (float*)(base + lo.cd);
+  a.cand_s = (float4*)(base + lo.cs);
   const size_t smem = sizeof(SelTcSmem<DD, KT>) + 1024;
   if ((e = cudaFuncSetAttribute(sel_tc_kernel<DD, KT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)smem)) != cudaSuccess)
@@ -1069,9 +1132,14 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int rows = Dm.Bq * Dm.Hkv;
-  dtc_merge_kernel<DD><<<(unsigned)rows, 256, 0, st>>>(
-      a.cand_l, a.cand_u, a.cand_c, a.cand_n, a.cand_d, SelCfg<KT>::kBuf, qh32, kbar32, idx, s_sel, w, Dm.Bq, Dm.Hkv,
-      (int)Dm.Nc, lo.n_split, lo.range, Dm.topk, Dm.scale_sel);
+  if (lo.n_split > kMaxSplit) return cudaErrorNotSupported;
+  const size_t mg_smem = ((size_t)kMergeWarps * 32 * DD + DD) * 4 + (size_t)kMergeCand * 4;
+  if ((e = cudaFuncSetAttribute(dtc_merge_kernel<DD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mg_smem)) !=
+      cudaSuccess)
+    return e;
+  dtc_merge_kernel<DD><<<(unsigned)rows, kMergeWarps * 32, mg_smem, st>>>(
+      a.cand_l, a.cand_u, a.cand_c, a.cand_n, a.cand_d, a.cand_s, SelCfg<KT>::kBuf, qh32, kbar32, idx, s_sel, w, Dm.Bq,
+      Dm.Hkv, (int)Dm.Nc, lo.n_split, lo.range, Dm.topk, Dm.scale_sel);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return launch_decode_attend(Dm, q, K, V, idx, w, O, (float*)(base + lo.opart), st);

@@ -54,8 +54,8 @@ def select_workload(number, batch):
 # has changed).
 NCU_TRAFFIC = {
     # bwd_delta + bwd_chunk + bwd_dq_merge at the long-context workload (B=2, L=32768), one launch each
-    "hsa_backward": {"bytes_per_launch": 15407138304, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
-                     "sha256": "dff8a9b920f1c01b0fc423ea3badf2353e8992233ffdb569294e1bf13cd389a0"},
+    "hsa_backward": {"bytes_per_launch": 15013581312, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
+                     "sha256": "2c3d71e8d977963d053f3e0150d90f65125d0f52d7c359209112566d526e61ee"},
 }
 
 

@@ -33,8 +33,8 @@
 //                                       row-major tiles read MN-major)
 //   dq' = dSk K                        (K read as an MN-major operand)
 // The dK/dV products come first, so the Q/dO stage is released before the
-// dq product runs. Warps 0-3 (one thread per row) turn S, dP' into P and
-// dSk; warps 4-7 store dq' and finally dK, dV; warps 8, 10 and 11 gather the
+// dq product runs. Warps 0-3 and 12-15 (two threads per row) turn S, dP'
+// into P and dSk; warps 4-7 store dq' and finally dK, dV; warps 8, 10 and 11 gather the
 // Q and dO rows of the next tiles; one thread of warp 9 issues the MMAs.
 #include <cstring>
 
@@ -44,7 +44,7 @@ namespace hsa {
 namespace {
 
 constexpr int kRows = 128;     // query rows per step (tensor-core M)
-constexpr int kThreads = 384;  // warps 0-3 softmax/gradients, 4-7 epilogue, 8, 10, 11 loaders, 9 MMA
+constexpr int kThreads = 512;  // warps 0-3 and 12-15 softmax/gradients, 4-7 epilogue, 8, 10, 11 loaders, 9 MMA
 constexpr int kLoaders = 3;
 constexpr int kTmemCols = 512;
 
@@ -64,6 +64,7 @@ struct BwdSmem {
   float slot_w[2][kRows];
   float slot_delta[2][kRows];
   int row_p[3][kRows];            // softmax -> epilogue: the row's slot id (-1: none)
+  float xch[3][2][kRows];         // softmax halves: row maximum, sum and D of each half
   uint64_t bar[16];
   uint32_t tmem_base;
   int abort_flag;
@@ -76,8 +77,8 @@ enum {
   BAR_QD_FULL = 0,   // 2: Q and dO tiles landed
   BAR_QD_EMPTY = 2,  // 2: every MMA reading the tiles finished (commit)
   BAR_S_FULL = 4,    // 2: S and dP' ready (commit)
-  BAR_S_EMPTY = 6,   // 2: S and dP' read (128 arrivals)
-  BAR_P_FULL = 8,    // P, dSq, dSk written (128 arrivals)
+  BAR_S_EMPTY = 6,   // 2: S and dP' read (256 arrivals)
+  BAR_P_FULL = 8,    // P, dSk written (256 arrivals)
   BAR_P_EMPTY = 9,   // P, dSq, dSk consumed (commit)
   BAR_DQ_FULL = 10,  // dq accumulator ready (commit)
   BAR_DQ_EMPTY = 11, // dq read (128 arrivals)
@@ -147,10 +148,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(bar(BAR_QD_FULL + i), a.use_tma ? kLoaders : 32);
       tc::mbar_init(bar(BAR_QD_EMPTY + i), 1);
       tc::mbar_init(bar(BAR_S_FULL + i), 1);
-      tc::mbar_init(bar(BAR_S_EMPTY + i), 128);
+      tc::mbar_init(bar(BAR_S_EMPTY + i), 256);
     }
     for (int i = 0; i < 3; ++i) tc::mbar_init(bar(BAR_DS_FULL + i), 128);
-    tc::mbar_init(bar(BAR_P_FULL), 128);
+    tc::mbar_init(bar(BAR_P_FULL), 256);
     tc::mbar_init(bar(BAR_P_EMPTY), 1);
     tc::mbar_init(bar(BAR_DQ_FULL), 1);
     tc::mbar_init(bar(BAR_DQ_EMPTY), 128);
@@ -175,7 +176,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::fence_after_sync();
   const uint32_t tmem = sm.tmem_base;
 
-  if (warp == 8 || warp >= 10) {
+  if (warp == 8 || warp == 10 || warp == 11) {
     // ---------------------------------------------------------------- loader warps
     // TMA path: a tile's 2 * epi gathers (item s < epi: the q rows of slot s;
     // item epi + s: the dO rows of slot s) are spread over warps 8, 10 and 11,
@@ -381,20 +382,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mma_commit(bar(BAR_ACC_DONE));
     }
     __syncwarp();
-  } else if (warp < 4) {
-    // ---------------------------------------------------------------- softmax / gradient rows (thread = row)
-    const int r = tid;
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  } else if (warp < 4 || warp >= 12) {
+    // ---------------------------------------------------------------- softmax / gradient rows
+    // Two threads per row: warps 0-3 take chunk positions 0-31 and warps
+    // 12-15 positions 32-63 of the same rows (tensor-memory lanes); the row
+    // maximum, sum and D are combined through shared memory, each pair of
+    // warps meeting at its own named barrier.
+    const int hf = warp >= 12 ? 1 : 0;
+    const int r = (warp & 3) * 32 + lane;
+    const int c0 = hf * 32;
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
     const float inv_S = 1.f / (float)kChunk;
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + (warp & 3)) : "memory"); };
     for (int i = 0; i < niter; ++i) {
       const int sb = i & 1, st = i & 1;
       tc::mbar_wait(bar(BAR_S_FULL + sb), (i >> 1) & 1, abort_flag, status);
       tc::fence_after_sync();
-      float x[64], y[64];
-      tc::tmem_ld32(tmem + lane_base + Cols<D>::S + sb * kChunk, *reinterpret_cast<float(*)[32]>(&x[0]));
-      tc::tmem_ld32(tmem + lane_base + Cols<D>::S + sb * kChunk + 32, *reinterpret_cast<float(*)[32]>(&x[32]));
-      tc::tmem_ld32(tmem + lane_base + Cols<D>::dP + sb * kChunk, *reinterpret_cast<float(*)[32]>(&y[0]));
-      tc::tmem_ld32(tmem + lane_base + Cols<D>::dP + sb * kChunk + 32, *reinterpret_cast<float(*)[32]>(&y[32]));
+      float x[32], y[32];
+      tc::tmem_ld32(tmem + lane_base + Cols<D>::S + sb * kChunk + c0, x);
+      tc::tmem_ld32(tmem + lane_base + Cols<D>::dP + sb * kChunk + c0, y);
       tc::tmem_wait_ld();
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_S_EMPTY + sb));
@@ -408,40 +414,48 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int u = 0; u < 8; ++u) mx[u] = x[u];
 #pragma unroll
-      for (int k = 8; k < 64; ++k) mx[k & 7] = fmaxf(mx[k & 7], x[k]);
-      const float m = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
-      const float ms = m * a.scale_log2;
+      for (int k = 8; k < 32; ++k) mx[k & 7] = fmaxf(mx[k & 7], x[k]);
+      sm.xch[0][hf][r] =
+          fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+      pair_sync();
+      const float ms = fmaxf(sm.xch[0][0][r], sm.xch[0][1][r]) * a.scale_log2;
 #pragma unroll
       for (int u = 0; u < 8; ++u) zz[u] = 0.f;
 #pragma unroll
-      for (int k = 0; k < 64; ++k) {
+      for (int k = 0; k < 32; ++k) {
         x[k] = exp2f(fmaf(x[k], a.scale_log2, -ms));
         zz[k & 7] += x[k];
       }
-      const float inv = 1.f / (((zz[0] + zz[1]) + (zz[2] + zz[3])) + ((zz[4] + zz[5]) + (zz[6] + zz[7])));
+      sm.xch[1][hf][r] = ((zz[0] + zz[1]) + (zz[2] + zz[3])) + ((zz[4] + zz[5]) + (zz[6] + zz[7]));
+      pair_sync();
+      const float inv = 1.f / (sm.xch[1][0][r] + sm.xch[1][1][r]);
 #pragma unroll
       for (int u = 0; u < 8; ++u) dd[u] = 0.f;
 #pragma unroll
-      for (int k = 0; k < 64; ++k) {
+      for (int k = 0; k < 32; ++k) {
         x[k] *= inv;
         dd[k & 7] = fmaf(x[k], y[k], dd[k & 7]);
       }
-      const float Drow = ((dd[0] + dd[1]) + (dd[2] + dd[3])) + ((dd[4] + dd[5]) + (dd[6] + dd[7]));
+      sm.xch[2][hf][r] = ((dd[0] + dd[1]) + (dd[2] + dd[3])) + ((dd[4] + dd[5]) + (dd[6] + dd[7]));
+      pair_sync();
+      const float Drow = sm.xch[2][0][r] + sm.xch[2][1][r];
       float dw = Drow;  // sum over the G rows of the slot (consecutive lanes)
       for (int o = 1; o < a.G; o <<= 1) dw += __shfl_xor_sync(0xFFFFFFFFu, dw, o);
       const float dsv = wv * (dw - dl);
       // hand the slot id to the epilogue warps (three buffers: step i+3 runs
-      // after S of step i+3, which the MMA thread issues only after the dK/dV
-      // products of step i+1, which wait for the epilogue of step i to have
+      // after S of step i+3, which the MMA thread issues only after the dq
+      // product of step i+1, which waits for the epilogue of step i to have
       // read the dq accumulator, and so its slot ids)
-      sm.row_p[i % 3][r] = pv;
-      tc::mbar_arrive(bar(BAR_DS_FULL + i % 3));
+      if (hf == 0) {
+        sm.row_p[i % 3][r] = pv;
+        tc::mbar_arrive(bar(BAR_DS_FULL + i % 3));
+      }
       const float ca = a.scale_attn * wv, pool = a.scale_sel * dsv * inv_S;
       tc::mbar_wait(bar(BAR_P_EMPTY), (i & 1) ^ 1, abort_flag, status);
       const uint32_t prow = smem_u32(sm.P), krow = smem_u32(sm.dSk);
 #pragma unroll
-      for (int c16 = 0; c16 < 8; ++c16) {
-        const uint32_t o = tc::sw128_offset(kRows, r, c16 * 8);
+      for (int c16 = 0; c16 < 4; ++c16) {
+        const uint32_t o = tc::sw128_offset(kRows, r, c0 + c16 * 8);
         uint32_t pp[4], gk[4];
 #pragma unroll
         for (int h = 0; h < 4; ++h) {
@@ -468,26 +482,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_wait(bar(BAR_DQ_FULL), j & 1, abort_flag, status);
       tc::fence_after_sync();
       uint16_t* dst = (!a.use_tma && pj >= 0) ? a.dqpart + ((long long)pj * a.G + (r & (a.G - 1))) * D : nullptr;
-      float v[D];
+      // dq' in 64-column halves: each is read from tensor memory, written to the
+      // staging atoms (one 1 KB atom per 8 rows, 128-byte swizzle) and stored by
+      // the first lane of every 8-row group with one TMA box; the accumulator
+      // is released once the last half has been read
+      const uint32_t atom = smem_u32(sm.dqstage) + (warp & 3) * 4096 + (lane >> 3) * 1024;
+      const uint32_t row = atom + (lane & 7) * 128, swz = lane & 7;
+      const bool issuer = (lane & 7) == 0 && pj >= 0;
 #pragma unroll
-      for (int h = 0; h < D / 32; ++h) tc::tmem_ld32(tmem + lane_base + Cols<D>::dq + h * 32, *reinterpret_cast<float(*)[32]>(&v[h * 32]));
-      tc::tmem_wait_ld();
-      tc::fence_before_sync();
-      tc::mbar_arrive(bar(BAR_DQ_EMPTY));
-      if (a.use_tma) {
-        // 64 columns at a time through the warp's staging atoms (one 1 KB
-        // atom per 8 rows, 128-byte swizzle); the first lane of every 8-row
-        // group stores the group with one TMA box
-        const uint32_t atom = smem_u32(sm.dqstage) + (warp & 3) * 4096 + (lane >> 3) * 1024;
-        const uint32_t row = atom + (lane & 7) * 128, swz = lane & 7;
-        const bool issuer = (lane & 7) == 0 && pj >= 0;
-#pragma unroll
-        for (int h = 0; h < D / 64; ++h) {
+      for (int h = 0; h < D / 64; ++h) {
+        float v[64];
+        tc::tmem_ld32(tmem + lane_base + Cols<D>::dq + h * 64, *reinterpret_cast<float(*)[32]>(&v[0]));
+        tc::tmem_ld32(tmem + lane_base + Cols<D>::dq + h * 64 + 32, *reinterpret_cast<float(*)[32]>(&v[32]));
+        tc::tmem_wait_ld();
+        if (h == D / 64 - 1) {
+          tc::fence_before_sync();
+          tc::mbar_arrive(bar(BAR_DQ_EMPTY));
+        }
+        if (a.use_tma) {
           if ((lane & 7) == 0) tc::bulk_wait_read();  // the previous round's boxes have left the atoms
           __syncwarp();
 #pragma unroll
           for (int c8 = 0; c8 < 8; ++c8) {
-            const float* o = &v[h * 64 + 8 * c8];
+            const float* o = &v[8 * c8];
             asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};\n" ::"r"(row + ((c8 ^ swz) << 4)),
                          "r"(pack_bf16x2(o[0], o[1])), "r"(pack_bf16x2(o[2], o[3])), "r"(pack_bf16x2(o[4], o[5])),
                          "r"(pack_bf16x2(o[6], o[7])));
@@ -498,14 +515,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::tma_store_2d_hint(&tmap_dq, h * 64, pj * a.G + (r & (a.G - 1)), atom, stream);
             tc::bulk_commit();
           }
-        }
-      } else if (dst) {
-        uint4* d4 = reinterpret_cast<uint4*>(dst);
+        } else if (dst) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + h * 64);
 #pragma unroll
-        for (int q8 = 0; q8 < D / 8; ++q8) {
-          const float* o = &v[8 * q8];
-          d4[q8] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
-                              pack_bf16x2(o[6], o[7]));
+          for (int q8 = 0; q8 < 8; ++q8) {
+            const float* o = &v[8 * q8];
+            d4[q8] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]),
+                                pack_bf16x2(o[6], o[7]));
+          }
         }
       }
     }

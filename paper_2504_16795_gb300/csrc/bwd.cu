@@ -160,7 +160,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_mbar_init();
   }
   if (warp == 9) tc::tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
-  if (warp < 8) {  // chunk K, V (rows s) and K̄, once per block
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = sm.tmem_base;
+  // chunk K and V (rows s), once per block, by warps 0-7 while the loaders
+  // already gather the first tiles; the MMA warp meets them at named barrier
+  // 5 before its first product
+  if (warp < 8) {
     for (int u = tid; u < kChunk * D8; u += 256) {
       const int srow = u / D8, ch = u % D8;
       const long long src = (row0 + (long long)srow * a.Hkv) * D + ch * 8;
@@ -170,11 +177,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     cp_async_commit();
     cp_async_wait<0>();
     tc::fence_proxy_async_smem();
+    asm volatile("bar.arrive 5, 288;" ::: "memory");
   }
-  tc::fence_before_sync();
-  __syncthreads();
-  tc::fence_after_sync();
-  const uint32_t tmem = sm.tmem_base;
 
   if (warp == 8 || warp == 10 || warp == 11) {
     // ---------------------------------------------------------------- loader warps
@@ -300,6 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 9) {
     // ---------------------------------------------------------------- MMA issue (one thread)
+    asm volatile("bar.sync 5, 288;" ::: "memory");  // K and V staged (the whole warp takes part)
     if (lane == 0) {
       constexpr uint32_t idSP = tc::idesc_bf16(kRows, kChunk);                // S, dP': Q K^T, dO V^T
       constexpr uint32_t idDQ = tc::idesc_bf16(kRows, D, false, true);        // dq = dSq K   (K as MN-major B)
@@ -312,6 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t kMnK = (uint32_t)kChunk * 128;
       const uint32_t kbase = smem_u32(sm.K), vbase = smem_u32(sm.V);
       const uint32_t pbase = smem_u32(sm.P), dsk = smem_u32(sm.dSk);
+      tc::fence_after_sync();
       auto issue_SdP = [&](int i) {
         const int st = i & 1, sb = i & 1;
         tc::fence_after_sync();

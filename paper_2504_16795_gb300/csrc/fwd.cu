@@ -31,7 +31,7 @@ template <int D>
 struct FwdSmem {
   uint16_t Q[kQStages][kRows * D];  // gathered query rows, grouped K-major SW128 (tc::grp_offset)
   uint16_t K[kChunk * D];           // chunk keys [s][d]
-  uint16_t Vt[D * kChunk];          // chunk values transposed [d][s]
+  uint16_t V[kChunk * D];           // chunk values [s][d] (read MN-major by the second product)
   uint16_t Ostage[2][kRows * D];    // TMA path: a step's O' rows (grouped layout) on their way out, two steps
   int slot_row[kQStages][kRows];    // cp.async path: first q row of each slot (-1: past the list)
   uint64_t bar[16];
@@ -102,28 +102,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_mbar_init();
   }
   if (warp == 9) tc::tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
-  if (warp < 8) {  // chunk K (K-major rows s) and V^T (rows d), once per block
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = sm.tmem_base;
+  // chunk K and V ([s][d], 128-byte swizzle), once per block, by warps 0-7
+  // while the loaders already gather the first query tiles; the MMA warp
+  // meets them at named barrier 1 before its first product
+  if (warp < 8) {
     const long long row0 = ((long long)b * a.L + (long long)c * kChunk) * a.Hkv + g;
     for (int u = tid; u < kChunk * D8; u += 256) {
       const int srow = u / D8, ch = u % D8;
       const long long src = (row0 + (long long)srow * a.Hkv) * D + ch * 8;
       cp_async16(smem_u32(sm.K) + tc::sw128_offset(kChunk, srow, ch * 8), a.K + src);
-      const uint4 v = __ldg(reinterpret_cast<const uint4*>(a.V + src));
-      const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const uint16_t h = (uint16_t)(i & 1 ? (w4[i >> 1] >> 16) : (w4[i >> 1] & 0xFFFFu));
-        *reinterpret_cast<uint16_t*>(reinterpret_cast<char*>(sm.Vt) + tc::sw128_offset(D, ch * 8 + i, srow)) = h;
-      }
+      cp_async16(smem_u32(sm.V) + tc::sw128_offset(kChunk, srow, ch * 8), a.V + src);
     }
     cp_async_commit();
     cp_async_wait<0>();
     tc::fence_proxy_async_smem();
+    asm volatile("bar.arrive 1, 288;" ::: "memory");
   }
-  tc::fence_before_sync();
-  __syncthreads();
-  tc::fence_after_sync();
-  const uint32_t tmem = sm.tmem_base;
 
   if (warp == 8 || warp >= 10) {
     // ---------------------------------------------------------------- loader warps
@@ -199,10 +197,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 9) {
     // ---------------------------------------------------------------- MMA issue (one thread)
+    asm volatile("bar.sync 1, 288;" ::: "memory");  // K and V staged (the whole warp takes part)
     if (lane == 0) {
       constexpr uint32_t idS = tc::idesc_bf16(kRows, kChunk);
-      constexpr uint32_t idO = tc::idesc_bf16(kRows, D);
-      const uint32_t kbase = smem_u32(sm.K), vbase = smem_u32(sm.Vt);
+      constexpr uint32_t idO = tc::idesc_bf16(kRows, D, false, true);  // V as the MN-major B operand
+      constexpr uint32_t kMnV = (uint32_t)kChunk * 128;                  // 64-column blocks of V
+      const uint32_t kbase = smem_u32(sm.K), vbase = smem_u32(sm.V);
+      tc::fence_after_sync();
       auto issue_S = [&](int i) {
         const int st = i % kQStages, sb = i & 1;
         tc::fence_after_sync();
@@ -222,7 +223,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < kChunk / 16; ++kk)
           tc::mma_bf16_ts(tmem + 2 * kChunk + pb * D, tmem + kColP + pb * (kChunk / 2) + kk * 8,
-                          tc::sdesc_sw128(vbase + kk * 32), idO, kk > 0);
+                          tc::sdesc_sw128_mn(vbase + kk * 2048, kMnV), idO, kk > 0);
         tc::mma_commit(bar(BAR_O_FULL + pb));
       };
       // Event loop: issue S of step nS (tile landed, S buffer read) or O of step

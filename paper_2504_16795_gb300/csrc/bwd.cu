@@ -122,8 +122,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int key = blockIdx.x;
-  const int c = key % a.Nc, bg = key / a.Nc;
+  int c, bg;
+  block_key(a.Nc, (int)(gridDim.x / (unsigned)a.Nc), c, bg);
+  const int key = bg * a.Nc + c;
   const int b = bg / a.Hkv, g = bg % a.Hkv;
   const int off = a.offsets[key];
   const int cnt = a.offsets[key + 1] - off;

@@ -10,6 +10,26 @@
 namespace hsa {
 
 constexpr int kChunk = 64;  // S: the only chunk size the kernels are built for
+
+// Block order of the chunk kernels. A chunk's list holds the slots of every
+// later token that chose it, so early chunks carry the longest lists. The
+// first kHeadChunks chunks of every (b, g) run first, chunk-major across the
+// pairs, so that no long list starts near the end of the grid; the rest run
+// pair by pair in chunk order, so that the blocks in flight gather query rows
+// of one (b, g) and share them in L2.
+constexpr int kHeadChunks = 16;
+__device__ __forceinline__ void block_key(int Nc, int n_bg, int& c, int& bg) {
+  const int head = min(kHeadChunks, Nc);
+  const int b = (int)blockIdx.x;
+  if (b < head * n_bg) {
+    c = b / n_bg;
+    bg = b % n_bg;
+  } else {
+    const int r = b - head * n_bg, rest = Nc - head;
+    bg = r / rest;
+    c = head + r % rest;
+  }
+}
 constexpr int kWarp = 32;
 
 // Resolved shape shared by host launchers.

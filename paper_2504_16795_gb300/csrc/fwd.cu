@@ -73,8 +73,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int D8 = D / 8;
   constexpr uint32_t kColP = 2 * kChunk + 2 * D;  // tensor memory: S x2 | O' x2 | P x2 (32 columns each)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int key = blockIdx.x;
-  const int c = key % a.Nc, bg = key / a.Nc;
+  int c, bg;
+  block_key(a.Nc, (int)(gridDim.x / (unsigned)a.Nc), c, bg);
+  const int key = bg * a.Nc + c;
   const int b = bg / a.Hkv, g = bg % a.Hkv;
   const int off = a.offsets[key];
   const int cnt = a.offsets[key + 1] - off;

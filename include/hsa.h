@@ -101,6 +101,13 @@ unsigned long long hsa_kernel_launches(void);
  * Synchronising: not for use inside a timed region. */
 hsa_status_t hsa_device_check(void);
 
+/* Self-test of that bound: launches one block that waits on a barrier nothing
+ * ever completes, for at most limit_ns (1 ns to 1 s). The wait gives up, the
+ * block returns, and the next hsa_device_check reports HSA_ERR_TIMEOUT once;
+ * the context stays usable. No device fault and no hang is involved.
+ * Asynchronous on `stream`; HSA_ERR_INVALID_ARG for a limit outside the range. */
+hsa_status_t hsa_selftest_wait_timeout(unsigned long long limit_ns, cudaStream_t stream);
+
 /* Workspace bytes that `op` needs for `shape` (0 when it needs none). Returns
  * 0 too for an invalid shape; the call itself then reports the error. */
 size_t hsa_workspace_size(int op, const hsa_shape_t* shape);

@@ -23,6 +23,7 @@ from .binding import (  # noqa: F401
     decode_noalloc,
     decode_workspace_size,
     device_check,
+    selftest_wait_timeout,
     forward,
     hsa_backward_path,
     hsa_forward_path,

@@ -104,6 +104,8 @@ def load():
     L.hsa_kernel_launches.argtypes = []
     L.hsa_device_check.restype = i
     L.hsa_device_check.argtypes = []
+    L.hsa_selftest_wait_timeout.restype = i
+    L.hsa_selftest_wait_timeout.argtypes = [ctypes.c_ulonglong, vp]
     L.hsa_workspace_size.restype = sz
     L.hsa_workspace_size.argtypes = [i, sp]
     L.hsa_decode_workspace_size.restype = sz
@@ -136,6 +138,12 @@ def kernel_launches() -> int:
 def device_check() -> None:
     """Synchronise and raise if a device-side wait gave up since the last check."""
     _check(load().hsa_device_check(), "hsa_device_check")
+
+
+def selftest_wait_timeout(limit_ns: int, device=None) -> None:
+    """Launch the bounded-wait self-test (a wait nothing completes, given up after limit_ns)."""
+    dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+    _check(load().hsa_selftest_wait_timeout(int(limit_ns), _stream(dev)), "hsa_selftest_wait_timeout")
 
 
 def status_string(status: int) -> str:

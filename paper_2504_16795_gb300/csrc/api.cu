@@ -86,9 +86,14 @@ unsigned long long hsa_kernel_launches(void) { return hsa::g_launches.load(std::
 hsa_status_t hsa_device_check(void) {
   if (cudaDeviceSynchronize() != cudaSuccess) return HSA_ERR_CUDA;
   const unsigned s1 = hsa::forward_take_status(), s2 = hsa::backward_take_status(),
-                 s3 = hsa::select_take_status();
-  if (s1 == ~0u || s2 == ~0u || s3 == ~0u) return HSA_ERR_CUDA;
-  return (s1 | s2 | s3) ? HSA_ERR_TIMEOUT : HSA_OK;
+                 s3 = hsa::select_take_status(), s4 = hsa::selftest_take_status();
+  if (s1 == ~0u || s2 == ~0u || s3 == ~0u || s4 == ~0u) return HSA_ERR_CUDA;
+  return (s1 | s2 | s3 | s4) ? HSA_ERR_TIMEOUT : HSA_OK;
+}
+
+hsa_status_t hsa_selftest_wait_timeout(unsigned long long limit_ns, cudaStream_t stream) {
+  if (limit_ns == 0 || limit_ns > 1000000000ull) return HSA_ERR_INVALID_ARG;
+  return hsa::launch_selftest_wait(limit_ns, stream) == cudaSuccess ? HSA_OK : HSA_ERR_CUDA;
 }
 
 size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {

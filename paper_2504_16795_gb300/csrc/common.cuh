@@ -204,6 +204,9 @@ cudaError_t launch_forward(const Dims& D, const void* q, const void* K, const vo
                            void* ws, cudaStream_t st);
 size_t backward_workspace(const Dims& D);
 unsigned backward_take_status();
+// Self-test of the bounded waits: one block waits on a barrier nothing arrives at.
+cudaError_t launch_selftest_wait(unsigned long long limit_ns, cudaStream_t st);
+unsigned selftest_take_status();
 cudaError_t launch_backward(const Dims& D, const void* q, const void* K, const void* V, const float* kbar32,
                             const int32_t* idx, const float* w, const void* O, const void* dO,
                             const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,

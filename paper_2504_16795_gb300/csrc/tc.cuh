@@ -59,11 +59,12 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Wait for the phase with the given parity to complete. Bounded (see above);
-// the clock is first read after 256 unsuccessful polls, so a wait that ends
-// soon pays nothing for the bound.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          unsigned* status) {
+// Wait for the phase with the given parity to complete, for at most
+// `limit_ns`: on giving up it sets the block's abort flag and the status word
+// and returns false. The clock is first read after 256 unsuccessful polls, so
+// a wait that ends soon pays nothing for the bound.
+__device__ __forceinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, unsigned long long limit_ns,
+                                              volatile int* abort_flag, unsigned* status) {
   unsigned long long t0 = 0;
   for (unsigned it = 0;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -72,13 +73,18 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
       const unsigned long long now = globaltimer();
       if (it == 255u) {
         t0 = now;
-      } else if (now - t0 > kWaitLimitNs) {
+      } else if (now - t0 > limit_ns) {
         *abort_flag = 1;
         if (status) atomicOr(status, kStatusTimeout);
         return false;
       }
     }
   }
+}
+// The pipelines' wait: bounded by kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          unsigned* status) {
+  return mbar_wait_for(bar, parity, kWaitLimitNs, abort_flag, status);
 }
 
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {

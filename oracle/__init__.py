@@ -42,11 +42,11 @@ def lib():
         i64 = ctypes.c_int64
         L.hsa_oracle_pool.argtypes = [vp, ci, ci, ci, ci, ci, ci, vp]
         L.hsa_oracle_select.argtypes = [vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, ci, vp, vp, vp, vp]
-        L.hsa_oracle_forward.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, vp, vp, vp]
-        L.hsa_oracle_backward.argtypes = [vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, cd,
+        L.hsa_oracle_forward.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, ci, ci, vp, vp, vp]
+        L.hsa_oracle_backward.argtypes = [vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, cd, ci, ci,
                                           vp, vp, vp, vp, vp, vp]
         L.hsa_oracle_decode_select.argtypes = [vp, vp, i64, ci, ci, ci, ci, ci, cd, ci, vp, vp, vp]
-        L.hsa_oracle_decode_attend.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, cd, vp, vp]
+        L.hsa_oracle_decode_attend.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, cd, ci, ci, vp, vp]
         for f in (L.hsa_oracle_pool, L.hsa_oracle_select, L.hsa_oracle_forward, L.hsa_oracle_backward,
                   L.hsa_oracle_decode_select, L.hsa_oracle_decode_attend):
             f.restype = None
@@ -107,8 +107,16 @@ def select(q, kbar, S, topk, scale_sel=None, f32=False, token_mask=None):
     return idx, s_sel, gap
 
 
-def forward(q, K, V, idx, s_sel, S, scale_attn=None, token_mask=None):
-    """-> O [B, L, Hq, d], w [B, L, Hkv, k] (rows outside token_mask stay 0)."""
+def _variant(inner, weights):
+    assert inner in ("softmax", "softmax1") and weights in ("softmax", "stick")
+    return int(inner == "softmax1"), int(weights == "stick")
+
+
+def forward(q, K, V, idx, s_sel, S, scale_attn=None, token_mask=None, inner="softmax", weights="softmax"):
+    """-> O [B, L, Hq, d], w [B, L, Hkv, k] (rows outside token_mask stay 0).
+
+    inner: "softmax" or "softmax1" (softmax-off-by-one inside a chunk); weights:
+    "softmax" or "stick" (stick-breaking chunk weights over I')."""
     q, K, V, s_sel = _f64(q), _f64(K), _f64(V), _f64(s_sel)
     idx = np.ascontiguousarray(idx, dtype=np.int32)
     B, L, Hq, d = q.shape
@@ -120,12 +128,13 @@ def forward(q, K, V, idx, s_sel, S, scale_attn=None, token_mask=None):
     w = np.zeros((B, L, Hkv, topk))
     m = _mask(token_mask, B, L)
     lib().hsa_oracle_forward(_p(q), _p(K), _p(V), _p(idx), _p(s_sel), B, L, Hq, Hkv, d, S, topk, float(scale_attn),
-                             _p(m), _p(O), _p(w))
+                             *_variant(inner, weights), _p(m), _p(O), _p(w))
     return O, w
 
 
-def backward(q, K, V, kbar, idx, s_sel, dO, S, scale_sel=None, scale_attn=None, token_mask=None):
-    """-> dict(dq, dK, dV, dkbar, ds); with token_mask only those tokens contribute."""
+def backward(q, K, V, kbar, idx, s_sel, dO, S, scale_sel=None, scale_attn=None, token_mask=None, inner="softmax",
+             weights="softmax"):
+    """-> dict(dq, dK, dV, dkbar, ds); with token_mask only those tokens contribute (variants as in forward)."""
     q, K, V, kbar, s_sel, dO = map(_f64, (q, K, V, kbar, s_sel, dO))
     idx = np.ascontiguousarray(idx, dtype=np.int32)
     B, L, Hq, d = q.shape
@@ -139,7 +148,8 @@ def backward(q, K, V, kbar, idx, s_sel, dO, S, scale_sel=None, scale_attn=None, 
     ds = np.zeros((B, L, Hkv, topk))
     m = _mask(token_mask, B, L)
     lib().hsa_oracle_backward(_p(q), _p(K), _p(V), _p(kbar), _p(idx), _p(s_sel), _p(dO), B, L, Hq, Hkv, d, S, topk,
-                              float(scale_sel), float(scale_attn), _p(m), _p(dq), _p(dK), _p(dV), _p(dkbar), _p(ds))
+                              float(scale_sel), float(scale_attn), *_variant(inner, weights), _p(m), _p(dq), _p(dK),
+                              _p(dV), _p(dkbar), _p(ds))
     return dict(dq=dq, dK=dK, dV=dV, dkbar=dkbar, ds=ds)
 
 
@@ -158,7 +168,7 @@ def decode_select(q, kbar, topk, scale_sel=None, f32=False):
     return idx, s_sel, gap
 
 
-def decode_attend(q, Ksel, Vsel, idx, s_sel, scale_attn=None):
+def decode_attend(q, Ksel, Vsel, idx, s_sel, scale_attn=None, inner="softmax", weights="softmax"):
     """Ksel, Vsel [Bq, Hkv, k, S, d] rows of the selected chunks -> w [Bq, Hkv, k], O [Bq, Hq, d]."""
     q, Ksel, Vsel, s_sel = map(_f64, (q, Ksel, Vsel, s_sel))
     idx = np.ascontiguousarray(idx, dtype=np.int32)
@@ -169,7 +179,7 @@ def decode_attend(q, Ksel, Vsel, idx, s_sel, scale_attn=None):
     w = np.zeros((Bq, Hkv, topk))
     O = np.zeros_like(q)
     lib().hsa_oracle_decode_attend(_p(q), _p(Ksel), _p(Vsel), _p(idx), _p(s_sel), Bq, Hq, Hkv, d, S, topk,
-                                   float(scale_attn), _p(w), _p(O))
+                                   float(scale_attn), *_variant(inner, weights), _p(w), _p(O))
     return w, O
 
 
@@ -187,8 +197,10 @@ def gather_chunks(mem, idx, S):
     return out
 
 
-def decode(q, Kmem, Vmem, kbar, S, topk, scale_sel=None, scale_attn=None, f32=False):
+def decode(q, Kmem, Vmem, kbar, S, topk, scale_sel=None, scale_attn=None, f32=False, inner="softmax",
+           weights="softmax"):
     """Whole decode step for small memories (full K, V given)."""
     idx, s_sel, gap = decode_select(q, kbar, topk, scale_sel, f32)
-    w, O = decode_attend(q, gather_chunks(Kmem, idx, S), gather_chunks(Vmem, idx, S), idx, s_sel, scale_attn)
+    w, O = decode_attend(q, gather_chunks(Kmem, idx, S), gather_chunks(Vmem, idx, S), idx, s_sel, scale_attn, inner,
+                         weights)
     return dict(idx=idx, s_sel=s_sel, gap=gap, w=w, O=O)

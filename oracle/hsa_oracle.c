@@ -14,10 +14,14 @@
  *     top-k by rank                                            (§3.1 "Chunk Selection")
  *   - selected indices ordered by decreasing chunk index (I')  (§3.1.1 "Chunk Weights")
  *   - chunk weights w = softmax over the selected scores        (§4.1 "Ablation
- *     Studies", the "w/o s.b." variant: softmax instead of stick-breaking)
+ *     Studies", the "w/o s.b." variant: softmax instead of stick-breaking),
+ *     or, with `stick`, the paper's default stick-breaking weights over I'
+ *     (§3.1.1 "Chunk Weights"): w_k = sigmoid(s_k) * prod_{i<k} (1 - sigmoid(s_i))
  *   - token-level attention inside every selected chunk and the weighted sum
  *     over chunks                                              (§3.1.1 "Hierarchical
- *     Attention"; Algorithm 1)
+ *     Attention"; Algorithm 1); plain softmax inside a chunk, or with
+ *     `softmax1` the softmax-off-by-one of §3.1.2 "Kernel Design" (a zero logit
+ *     joins the denominator, so a token may give a chunk little weight)
  *   - gradients into q, K, V (Algorithms 2 and 3) and, through w, into the
  *     selection scores, K̄ and K (Appendix A: the scores receive gradients
  *     because w takes part in the forward pass)
@@ -191,17 +195,35 @@ static int count_selected(const int32_t* I, int topk) {
     return k;
 }
 
-/* chunk weights: softmax over the k_eff selected scores */
-static void chunk_weights(const double* s, int keff, int topk, double* w) {
+static double sigmoid(double x) { return 1.0 / (1.0 + exp(-x)); }
+
+/* chunk weights over the k_eff selected scores, slots in I' order (decreasing
+ * chunk index): softmax, or (stick) stick-breaking — slot k takes the fraction
+ * sigmoid(s_k) of what the slots before it left of a unit stick */
+static void chunk_weights(const double* s, int keff, int topk, int stick, double* w) {
+    if (stick) {
+        double rest = 1.0;
+        for (int j = 0; j < topk; ++j) {
+            if (j < keff) {
+                const double beta = sigmoid(s[j]);
+                w[j] = beta * rest;
+                rest *= 1.0 - beta;
+            } else {
+                w[j] = 0.0;
+            }
+        }
+        return;
+    }
     double m = -INFINITY, z = 0.0;
     for (int j = 0; j < keff; ++j) m = s[j] > m ? s[j] : m;
     for (int j = 0; j < keff; ++j) z += exp(s[j] - m);
     for (int j = 0; j < topk; ++j) w[j] = j < keff ? exp(s[j] - m) / z : 0.0;
 }
 
-/* token-level attention of one query head over one chunk: P (S) and O_j (d) */
+/* token-level attention of one query head over one chunk: P (S) and O_j (d);
+ * softmax1: the denominator also holds exp(0) (softmax-off-by-one) */
 static void chunk_attention(const double* qh, const double* Kc, const double* Vc, int64_t row_stride, int d, int S,
-                            double scale_attn, double* P, double* Oj) {
+                            double scale_attn, int softmax1, double* P, double* Oj) {
     double m = -INFINITY, z = 0.0;
     for (int s = 0; s < S; ++s) {
         double a = 0.0;
@@ -213,6 +235,7 @@ static void chunk_attention(const double* qh, const double* Kc, const double* Vc
         P[s] = exp(P[s] - m);
         z += P[s];
     }
+    if (softmax1) z += exp(-m);
     for (int s = 0; s < S; ++s) P[s] /= z;
     for (int e = 0; e < d; ++e) {
         double acc = 0.0;
@@ -227,7 +250,7 @@ static void chunk_attention(const double* qh, const double* Kc, const double* Vc
  */
 void hsa_oracle_forward(const double* q, const double* K, const double* V, const int32_t* idx,
                         const double* s_sel, int B, int L, int Hq, int Hkv, int d, int S, int topk,
-                        double scale_attn, const uint8_t* token_mask, double* O, double* w) {
+                        double scale_attn, int softmax1, int stick, const uint8_t* token_mask, double* O, double* w) {
     const int G = Hq / Hkv;
 #pragma omp parallel
     {
@@ -240,7 +263,7 @@ void hsa_oracle_forward(const double* q, const double* K, const double* V, const
                     if (token_mask && !token_mask[(int64_t)b * L + t]) continue;
                     const int64_t o = at4(b, t, g, 0, L, Hkv, topk);
                     const int keff = count_selected(idx + o, topk);
-                    chunk_weights(s_sel + o, keff, topk, w + o);
+                    chunk_weights(s_sel + o, keff, topk, stick, w + o);
                     for (int hh = 0; hh < G; ++hh) {
                         const int h = g * G + hh;
                         const double* qh = q + at4(b, t, h, 0, L, Hq, d);
@@ -250,7 +273,7 @@ void hsa_oracle_forward(const double* q, const double* K, const double* V, const
                             const int64_t i = idx[o + j];
                             const double* Kc = K + at4(b, i * S, g, 0, L, Hkv, d);
                             const double* Vc = V + at4(b, i * S, g, 0, L, Hkv, d);
-                            chunk_attention(qh, Kc, Vc, (int64_t)Hkv * d, d, S, scale_attn, P, Oj);
+                            chunk_attention(qh, Kc, Vc, (int64_t)Hkv * d, d, S, scale_attn, softmax1, P, Oj);
                             for (int e = 0; e < d; ++e) Oh[e] += w[o + j] * Oj[e];
                         }
                     }
@@ -272,6 +295,8 @@ void hsa_oracle_forward(const double* q, const double* K, const double* V, const
  *   da_s     = P_s (dP_s - w_j D_{h,j})               (Algorithm 2/3: ∇S = wP∘(∇P - D'))
  *   dq_h    += c_att sum_s da_s K_s ; dK_s += c_att da_s q_h ; dV_s += w_j P_s dO_h
  *   ds_j     = w_j (dw_j - sum_j' w_j' dw_j')        (softmax over the selected scores)
+ *   ds_j     = (1 - b_j) w_j dw_j - b_j sum_{k>j} w_k dw_k,  b = sigmoid(s)
+ *                                                     (stick-breaking: w_k = b_k prod_{i<k} (1 - b_i))
  *   dq_h    += c_sel sum_j ds_j K̄_{I_j} (every head of the group) ; dK̄_{I_j} += c_sel ds_j q̂
  *   dK_{iS+s} += dK̄_i / S                             (mean pool)
  * token_mask (optional, [B, L]): only those tokens are processed, so dq rows
@@ -281,8 +306,9 @@ void hsa_oracle_forward(const double* q, const double* K, const double* V, const
  */
 void hsa_oracle_backward(const double* q, const double* K, const double* V, const double* kbar,
                          const int32_t* idx, const double* s_sel, const double* dO, int B, int L, int Hq,
-                         int Hkv, int d, int S, int topk, double scale_sel, double scale_attn,
-                         const uint8_t* token_mask, double* dq, double* dK, double* dV, double* dkbar, double* ds) {
+                         int Hkv, int d, int S, int topk, double scale_sel, double scale_attn, int softmax1,
+                         int stick, const uint8_t* token_mask, double* dq, double* dK, double* dV, double* dkbar,
+                         double* ds) {
     const int G = Hq / Hkv, Nc = L / S;
 #pragma omp parallel for collapse(2) schedule(dynamic, 1)
     for (int b = 0; b < B; ++b)
@@ -310,7 +336,7 @@ void hsa_oracle_backward(const double* q, const double* K, const double* V, cons
                 if (ds)
                     for (int j = 0; j < topk; ++j) ds[o + j] = 0.0;
                 if (keff == 0) continue;
-                chunk_weights(s_sel + o, keff, topk, w);
+                chunk_weights(s_sel + o, keff, topk, stick, w);
                 /* recompute the forward quantities of Algorithm 1 */
                 for (int j = 0; j < keff; ++j) dw[j] = 0.0;
                 for (int hh = 0; hh < G; ++hh) {
@@ -321,16 +347,25 @@ void hsa_oracle_backward(const double* q, const double* K, const double* V, cons
                         double* Pj = P + ((size_t)hh * topk + j) * S;
                         double* Ojh = Oj + ((size_t)hh * topk + j) * d;
                         chunk_attention(qh, K + at4(b, i * S, g, 0, L, Hkv, d), V + at4(b, i * S, g, 0, L, Hkv, d),
-                                        (int64_t)Hkv * d, d, S, scale_attn, Pj, Ojh);
+                                        (int64_t)Hkv * d, d, S, scale_attn, softmax1, Pj, Ojh);
                         double acc = 0.0;
                         for (int e = 0; e < d; ++e) acc += dOh[e] * Ojh[e];
                         D[hh * topk + j] = acc;
                         dw[j] += acc;
                     }
                 }
-                double wdw = 0.0;
-                for (int j = 0; j < keff; ++j) wdw += w[j] * dw[j];
-                for (int j = 0; j < keff; ++j) dsl[j] = w[j] * (dw[j] - wdw);
+                if (stick) {
+                    double later = 0.0; /* sum_{k>j} w_k dw_k */
+                    for (int j = keff - 1; j >= 0; --j) {
+                        const double beta = sigmoid(s_sel[o + j]);
+                        dsl[j] = (1.0 - beta) * w[j] * dw[j] - beta * later;
+                        later += w[j] * dw[j];
+                    }
+                } else {
+                    double wdw = 0.0;
+                    for (int j = 0; j < keff; ++j) wdw += w[j] * dw[j];
+                    for (int j = 0; j < keff; ++j) dsl[j] = w[j] * (dw[j] - wdw);
+                }
                 group_query(q + at4(b, t, 0, 0, L, Hq, d), G, g, d, 0, qhat);
                 for (int hh = 0; hh < G; ++hh) {
                     const int h = g * G + hh;
@@ -411,7 +446,7 @@ void hsa_oracle_decode_select(const double* q, const double* kbar, int64_t Nc, i
  * content where idx = -1). -> w [Bq, Hkv, topk], O [Bq, Hq, d]. */
 void hsa_oracle_decode_attend(const double* q, const double* Ksel, const double* Vsel, const int32_t* idx,
                               const double* s_sel, int Bq, int Hq, int Hkv, int d, int S, int topk,
-                              double scale_attn, double* w, double* O) {
+                              double scale_attn, int softmax1, int stick, double* w, double* O) {
     const int G = Hq / Hkv;
 #pragma omp parallel
     {
@@ -422,7 +457,7 @@ void hsa_oracle_decode_attend(const double* q, const double* Ksel, const double*
             for (int g = 0; g < Hkv; ++g) {
                 const int64_t o = ((int64_t)b * Hkv + g) * topk;
                 const int keff = count_selected(idx + o, topk);
-                chunk_weights(s_sel + o, keff, topk, w + o);
+                chunk_weights(s_sel + o, keff, topk, stick, w + o);
                 for (int hh = 0; hh < G; ++hh) {
                     const int h = g * G + hh;
                     const double* qh = q + ((int64_t)b * Hq + h) * d;
@@ -430,7 +465,7 @@ void hsa_oracle_decode_attend(const double* q, const double* Ksel, const double*
                     for (int e = 0; e < d; ++e) Oh[e] = 0.0;
                     for (int j = 0; j < keff; ++j) {
                         const int64_t base = ((o + j) * S) * (int64_t)d;
-                        chunk_attention(qh, Ksel + base, Vsel + base, d, d, S, scale_attn, P, Oj);
+                        chunk_attention(qh, Ksel + base, Vsel + base, d, d, S, scale_attn, softmax1, P, Oj);
                         for (int e = 0; e < d; ++e) Oh[e] += w[o + j] * Oj[e];
                     }
                 }

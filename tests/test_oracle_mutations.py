@@ -34,6 +34,12 @@ MUTATIONS = {
                                   "for (int hh = 0; hh < 1; ++hh) acc += q_row[(int64_t)(g * G + hh) * d + e];"),
     "chunk-summary gradient without q": ("dkb[(size_t)i * d + e] += scale_sel * dsl[j] * qhat[e];",
                                          "dkb[(size_t)i * d + e] += scale_sel * dsl[j];"),
+    "off-by-one term dropped": ("if (softmax1) z += exp(-m);", "if (softmax1) z += 0.0;"),
+    "stick-breaking remainder not shrunk": ("rest *= 1.0 - beta;", "rest *= 1.0;"),
+    "stick-breaking gradient without later slots": ("dsl[j] = (1.0 - beta) * w[j] * dw[j] - beta * later;",
+                                                     "dsl[j] = (1.0 - beta) * w[j] * dw[j];"),
+    "stick-breaking gradient over earlier slots": ("for (int j = keff - 1; j >= 0; --j) {",
+                                                   "for (int j = 0; j < keff; ++j) {"),
 }
 
 

@@ -345,6 +345,117 @@ def test_backward_invariants():
     assert (g["dq"][:, :S] == 0).all()
 
 
+# ----------------------------------------------------------------------------- variants: stick-breaking weights
+# (§3.1.1 "Chunk Weights") and softmax-off-by-one inside a chunk (§3.1.2 "Kernel Design")
+
+def sigmoid(x):
+    return 0.5 * (1.0 + np.tanh(0.5 * x))
+
+
+def test_stick_breaking_leaves_the_product_of_the_refusals():
+    # the slots share a unit stick: what they take together is 1 - prod(1 - sigmoid(s))
+    rng = np.random.default_rng(21)
+    B, L, S, Hq, Hkv, d, k = 1, 96, 8, 2, 1, 4, 4
+    q, K = rng.standard_normal((B, L, Hq, d)), rng.standard_normal((B, L, Hkv, d))
+    V = np.ones((B, L, Hkv, d))
+    kbar = oracle.pool(K, S)
+    idx, s_sel, _ = oracle.select(q, kbar, S, k)
+    O, w = oracle.forward(q, K, V, idx, s_sel, S, weights="stick")
+    keff = (idx >= 0).sum(-1)
+    for t in range(L):
+        n = keff[0, t, 0]
+        left = np.prod([1.0 - sigmoid(x) for x in s_sel[0, t, 0, :n]]) if n else 1.0
+        np.testing.assert_allclose(w[0, t, 0].sum(), 1.0 - left, atol=1e-14)
+        np.testing.assert_allclose(O[0, t], 1.0 - left, atol=1e-13)  # constant values: O = taken share
+        assert (w[0, t, 0, n:] == 0).all()
+
+
+def test_stick_breaking_with_equal_scores_is_geometric_from_the_latest_chunk():
+    # equal selection scores (identical chunk means): slot j (j-th latest chunk)
+    # takes b (1 - b)^j with b = sigmoid(s)
+    B, S, Nc, Hq, Hkv, d, k = 1, 4, 8, 1, 1, 3, 5
+    L = S * Nc
+    m = np.array([0.3, -0.2, 0.5])
+    r = RNG.standard_normal((Nc, S // 2, d))
+    K = (m[None, None] + np.concatenate([r, -r], axis=1)).reshape(1, L, 1, d)
+    q, V = RNG.standard_normal((B, L, Hq, d)), RNG.standard_normal((B, L, Hkv, d))
+    kbar = oracle.pool(K, S)
+    idx, s_sel, _ = oracle.select(q, kbar, S, k)
+    _, w = oracle.forward(q, K, V, idx, s_sel, S, weights="stick")
+    for t in range(S, L):
+        n = min(k, t // S)
+        b = sigmoid(s_sel[0, t, 0, 0])
+        np.testing.assert_allclose(w[0, t, 0, :n], b * (1.0 - b) ** np.arange(n), rtol=1e-12)
+        assert (np.diff(idx[0, t, 0, :n]) < 0).all()  # slot order: the latest chunk first
+
+
+def test_softmax_off_by_one_on_single_token_chunks_is_a_sigmoid_gate():
+    # S = 1: each chunk is one token, the inner softmax-off-by-one is sigmoid(c_att q·k)
+    rng = np.random.default_rng(5)
+    B, L, Hq, Hkv, d = 1, 20, 2, 1, 5
+    q, K, V = rng.standard_normal((B, L, Hq, d)), rng.standard_normal((B, L, Hkv, d)), rng.standard_normal((B, L, Hkv, d))
+    ca = 0.6
+    kbar = oracle.pool(K, 1)
+    idx, s_sel, _ = oracle.select(q, kbar, 1, L)
+    O, w = oracle.forward(q, K, V, idx, s_sel, 1, scale_attn=ca, inner="softmax1")
+    for t in range(1, L):
+        for h in range(Hq):
+            acc = np.zeros(d)
+            for j, c in enumerate(idx[0, t, 0]):
+                if c < 0:
+                    break
+                acc += w[0, t, 0, j] * sigmoid(ca * q[0, t, h] @ K[0, c, 0]) * V[0, c, 0]
+            np.testing.assert_allclose(O[0, t, h], acc, rtol=1e-12, atol=1e-14)
+
+
+def test_softmax_off_by_one_with_constant_values_keeps_z_over_one_plus_z():
+    rng = np.random.default_rng(9)
+    B, L, S, Hq, Hkv, d, k = 1, 48, 8, 2, 1, 4, 3
+    q, K = rng.standard_normal((B, L, Hq, d)), 2.0 * rng.standard_normal((B, L, Hkv, d))
+    V = np.ones((B, L, Hkv, d))
+    ca = 0.9
+    kbar = oracle.pool(K, S)
+    idx, s_sel, _ = oracle.select(q, kbar, S, k)
+    O, w = oracle.forward(q, K, V, idx, s_sel, S, scale_attn=ca, inner="softmax1")
+    for t in range(S, L):
+        for h in range(Hq):
+            want = 0.0
+            for j, c in enumerate(idx[0, t, 0]):
+                if c < 0:
+                    break
+                z = np.exp(ca * K[0, c * S:(c + 1) * S, 0] @ q[0, t, h]).sum()
+                want += w[0, t, 0, j] * z / (1.0 + z)
+            np.testing.assert_allclose(O[0, t, h], want, rtol=1e-12)
+
+
+@pytest.mark.parametrize("inner,weights,topk", [("softmax1", "softmax", 2), ("softmax", "stick", 3),
+                                                ("softmax1", "stick", 2), ("softmax", "stick", 1)])
+def test_variant_backward_matches_central_finite_differences(inner, weights, topk):
+    rng = np.random.default_rng(11 + topk)
+    B, L, S, Hq, Hkv, d = 1, 192, 16, 2, 1, 8
+    q, K, V, dO = (rng.standard_normal(s) for s in [(B, L, Hq, d), (B, L, Hkv, d), (B, L, Hkv, d), (B, L, Hq, d)])
+    kbar = oracle.pool(K, S)
+    idx0, s0, _ = oracle.select(q, kbar, S, topk)
+    g = oracle.backward(q, K, V, kbar, idx0, s0, dO, S, inner=inner, weights=weights)
+    if weights == "stick":
+        assert np.abs(g["ds"]).max() > 1e-3  # even one chunk: w = sigmoid(s) depends on its score
+
+    for name, arr in (("q", q), ("K", K), ("V", V)):
+        flat = arr.reshape(-1)
+
+        def setter(p, v, flat=flat):
+            flat[p] = v
+            return None
+
+        def f(_):
+            kb = oracle.pool(K, S)
+            idx, s_sel, _ = oracle.select(q, kb, S, topk)
+            O, _w = oracle.forward(q, K, V, idx, s_sel, S, inner=inner, weights=weights)
+            return float((O * dO).sum()), idx
+
+        fd_check(name, arr, setter, f, g["d" + name], 50, rng)
+
+
 # ----------------------------------------------------------------------------- decode (Section 3.2, Inference)
 
 def test_decode_equals_the_forward_row_after_the_memory():

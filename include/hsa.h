@@ -62,10 +62,22 @@ typedef enum {
     HSA_ERR_TIMEOUT = 5
 } hsa_status_t;
 
+/* Variant flags (hsa_shape_t.flags, hsa_decode_shape_t.flags); 0 selects the
+ * defaults: plain softmax inside a chunk, softmax chunk weights.
+ *   HSA_FLAG_SOFTMAX1        softmax-off-by-one inside a chunk (§3.1.2 "Kernel
+ *                            Design"): a zero logit joins every denominator.
+ *   HSA_FLAG_STICK_BREAKING  stick-breaking chunk weights over I' (§3.1.1 "Chunk
+ *                            Weights"): slot k (k-th latest selected chunk) gets
+ *                            sigmoid(s_k) * prod_{i<k} (1 - sigmoid(s_i)).
+ * Any other bit: HSA_ERR_UNSUPPORTED. */
+#define HSA_FLAG_SOFTMAX1 1
+#define HSA_FLAG_STICK_BREAKING 2
+
 typedef struct {
     int B, L, Hq, Hkv, d, S, topk;
     float scale_sel;  /* c_sel; <= 0 selects 1/sqrt((Hq/Hkv) * d) */
     float scale_attn; /* c_att; <= 0 selects 1/sqrt(d) */
+    int flags;        /* HSA_FLAG_*; 0: defaults */
 } hsa_shape_t;
 
 typedef struct {
@@ -73,6 +85,7 @@ typedef struct {
     long long n_chunks; /* complete chunks in the memory: the memory holds n_chunks * S tokens */
     float scale_sel;    /* <= 0 selects 1/sqrt((Hq/Hkv) * d) */
     float scale_attn;   /* <= 0 selects 1/sqrt(d) */
+    int flags;          /* HSA_FLAG_*; 0: defaults */
 } hsa_decode_shape_t;
 
 typedef enum {
@@ -183,7 +196,14 @@ hsa_status_t hsa_forward(const hsa_shape_t* shape, const void* q, const void* K,
  *   dq [B,L,Hq,d], dK, dV [B,L,Hkv,d] fp32, outputs (fully written).
  * Deterministic: every dK/dV row is owned by one thread block that walks its
  * chunk's entries in index order; no floating-point atomics.
- * Needs workspace HSA_OP_BACKWARD.
+ * Variants (shape->flags): softmax-off-by-one recomputes P with the zero
+ * logit; with stick-breaking weights the score gradient of a slot depends on
+ * the later slots' dw (ds_j = (1 - b_j) w_j dw_j - b_j sum_{k>j} w_k dw_k,
+ * b = sigmoid(s)), so the chunk pass writes dw per slot and three more passes
+ * add the selection terms (ds from w and dw; c_sel ds K̄ into dq; the mean-pool
+ * share of dK̄ into dK, per chunk in index order). b is recovered from w
+ * (b_j = w_j / (1 - sum_{i<j} w_i)), so s_sel is not an input.
+ * Needs workspace HSA_OP_BACKWARD (larger with stick-breaking weights).
  */
 hsa_status_t hsa_backward(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
                           const float* kbar32, const int32_t* idx, const float* w, const void* O, const void* dO,

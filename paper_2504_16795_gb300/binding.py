@@ -28,13 +28,19 @@ class HsaError(RuntimeError):
 class _Shape(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("L", ctypes.c_int), ("Hq", ctypes.c_int), ("Hkv", ctypes.c_int),
                 ("d", ctypes.c_int), ("S", ctypes.c_int), ("topk", ctypes.c_int),
-                ("scale_sel", ctypes.c_float), ("scale_attn", ctypes.c_float)]
+                ("scale_sel", ctypes.c_float), ("scale_attn", ctypes.c_float), ("flags", ctypes.c_int)]
 
 
 class _DecodeShape(ctypes.Structure):
     _fields_ = [("Bq", ctypes.c_int), ("Hq", ctypes.c_int), ("Hkv", ctypes.c_int), ("d", ctypes.c_int),
                 ("S", ctypes.c_int), ("topk", ctypes.c_int), ("n_chunks", ctypes.c_longlong),
-                ("scale_sel", ctypes.c_float), ("scale_attn", ctypes.c_float)]
+                ("scale_sel", ctypes.c_float), ("scale_attn", ctypes.c_float), ("flags", ctypes.c_int)]
+
+
+def _flags(inner: str, weights: str) -> int:
+    if inner not in ("softmax", "softmax1") or weights not in ("softmax", "stick"):
+        raise ValueError(f"unknown variant: inner={inner!r}, weights={weights!r}")
+    return (1 if inner == "softmax1" else 0) | (2 if weights == "stick" else 0)
 
 
 @dataclass(frozen=True)
@@ -49,6 +55,12 @@ class Shape:
     topk: int = 8
     scale_sel: float = 0.0   # <= 0: 1/sqrt(G*d)
     scale_attn: float = 0.0  # <= 0: 1/sqrt(d)
+    inner: str = "softmax"    # or "softmax1": softmax-off-by-one inside a chunk
+    weights: str = "softmax"  # or "stick": stick-breaking chunk weights
+
+    @property
+    def flags(self) -> int:
+        return _flags(self.inner, self.weights)
 
     @property
     def G(self) -> int:
@@ -59,7 +71,8 @@ class Shape:
         return self.L // self.S
 
     def c(self) -> _Shape:
-        return _Shape(self.B, self.L, self.Hq, self.Hkv, self.d, self.S, self.topk, self.scale_sel, self.scale_attn)
+        return _Shape(self.B, self.L, self.Hq, self.Hkv, self.d, self.S, self.topk, self.scale_sel, self.scale_attn,
+                      self.flags)
 
 
 @dataclass(frozen=True)
@@ -73,10 +86,12 @@ class DecodeShape:
     topk: int = 8
     scale_sel: float = 0.0
     scale_attn: float = 0.0
+    inner: str = "softmax"
+    weights: str = "softmax"
 
     def c(self) -> _DecodeShape:
         return _DecodeShape(self.Bq, self.Hq, self.Hkv, self.d, self.S, self.topk, self.n_chunks, self.scale_sel,
-                            self.scale_attn)
+                            self.scale_attn, _flags(self.inner, self.weights))
 
 
 _lib = None

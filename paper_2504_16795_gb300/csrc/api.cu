@@ -34,6 +34,7 @@ hsa_status_t resolve(const hsa_shape_t* s, Dims* out) {
   if (s->d != 64 && s->d != 128) return HSA_ERR_UNSUPPORTED;
   if (s->S != hsa::kChunk) return HSA_ERR_UNSUPPORTED;
   if (s->topk > 32) return HSA_ERR_UNSUPPORTED;
+  if (s->flags & ~(HSA_FLAG_SOFTMAX1 | HSA_FLAG_STICK_BREAKING)) return HSA_ERR_UNSUPPORTED;
   const long long slots = (long long)s->B * s->L * s->Hkv * s->topk;
   if (slots >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
   const long long rows = (long long)s->B * s->L * s->Hq;  // query rows are indexed in int32
@@ -50,6 +51,8 @@ hsa_status_t resolve(const hsa_shape_t* s, Dims* out) {
   D.Nc = s->L / s->S;
   D.scale_sel = s->scale_sel > 0.f ? s->scale_sel : (float)(1.0 / std::sqrt((double)G * s->d));
   D.scale_attn = s->scale_attn > 0.f ? s->scale_attn : (float)(1.0 / std::sqrt((double)s->d));
+  D.softmax1 = (s->flags & HSA_FLAG_SOFTMAX1) != 0;
+  D.stick = (s->flags & HSA_FLAG_STICK_BREAKING) != 0;
   *out = D;
   return HSA_OK;
 }
@@ -216,6 +219,7 @@ hsa_status_t resolve_decode(const hsa_decode_shape_t* s, hsa::DecodeDims* out) {
   if (s->S != hsa::kChunk) return HSA_ERR_UNSUPPORTED;
   if (s->topk > 32) return HSA_ERR_UNSUPPORTED;
   if (s->n_chunks >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
+  if (s->flags & ~(HSA_FLAG_SOFTMAX1 | HSA_FLAG_STICK_BREAKING)) return HSA_ERR_UNSUPPORTED;
   if ((long long)s->Bq * s->Hkv * s->topk >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
   hsa::DecodeDims D;
   D.Bq = s->Bq;
@@ -228,6 +232,8 @@ hsa_status_t resolve_decode(const hsa_decode_shape_t* s, hsa::DecodeDims* out) {
   D.Nc = s->n_chunks;
   D.scale_sel = s->scale_sel > 0.f ? s->scale_sel : (float)(1.0 / std::sqrt((double)G * s->d));
   D.scale_attn = s->scale_attn > 0.f ? s->scale_attn : (float)(1.0 / std::sqrt((double)s->d));
+  D.softmax1 = (s->flags & HSA_FLAG_SOFTMAX1) != 0;
+  D.stick = (s->flags & HSA_FLAG_STICK_BREAKING) != 0;
   *out = D;
   return HSA_OK;
 }

@@ -102,6 +102,9 @@ struct BwdArgs {
   int n_rows;   // B * L * Hq (a row index past it reads zeros)
   int use_tma;  // G >= 8: each slot's G rows arrive as one swizzled TMA box
   float scale_log2, scale_attn, scale_sel;
+  int softmax1;   // softmax-off-by-one inside the chunk
+  int stick;      // stick-breaking chunk weights: write dw per slot, no selection term here
+  float* dw_out;  // [slots] (stick-breaking only)
 };
 
 // TMEM columns
@@ -435,7 +438,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       sm.xch[1][hf][r] = ((zz[0] + zz[1]) + (zz[2] + zz[3])) + ((zz[4] + zz[5]) + (zz[6] + zz[7]));
       pair_sync();
-      const float inv = 1.f / (sm.xch[1][0][r] + sm.xch[1][1][r]);
+      const float inv = 1.f / ((sm.xch[1][0][r] + sm.xch[1][1][r]) + (a.softmax1 ? exp2f(-ms) : 0.f));
 #pragma unroll
       for (int u = 0; u < 8; ++u) dd[u] = 0.f;
 #pragma unroll
@@ -448,7 +451,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float Drow = sm.xch[2][0][r] + sm.xch[2][1][r];
       float dw = Drow;  // sum over the G rows of the slot (consecutive lanes)
       for (int o = 1; o < a.G; o <<= 1) dw += __shfl_xor_sync(0xFFFFFFFFu, dw, o);
-      const float dsv = wv * (dw - dl);
+      // softmax weights: ds = w (dw - Δ), folded in here; stick-breaking weights
+      // need every slot's dw first, so the slot's dw goes out and a later pass
+      // adds the selection terms
+      const float dsv = a.stick ? 0.f : wv * (dw - dl);
+      if (a.stick && hf == 0 && (r & (a.G - 1)) == 0 && pv >= 0) a.dw_out[pv] = dw;
       // hand the slot id to the epilogue warps (three buffers: step i+3 runs
       // after S of step i+3, which the MMA thread issues only after the dq
       // product of step i+1, which waits for the epilogue of step i to have
@@ -583,11 +590,120 @@ __global__ void __launch_bounds__(256) bwd_delta_kernel(const uint16_t* __restri
   if (lane == 0) delta[row] = acc;
 }
 
-// dq_t = sum_j dq'_{t,j} in slot order (one warp per (b, t, g)).
+// Stick-breaking weights (§3.1.1): w_j = b_j R_j with R_j = prod_{i<j} (1 - b_i)
+// = 1 - sum_{i<j} w_i, so b_j = w_j / R_j and
+//   ds_j = (1 - b_j) w_j dw_j - b_j sum_{k>j} w_k dw_k = (w_j / R_j) (R_{j+1} dw_j - U_j),
+// U_j = sum_{k>j} w_k dw_k. One thread per (b, t, g) row; R in double (a
+// slot that finds almost no stick left has almost no weight, and its ds stays
+// small whatever R's rounding).
+__global__ void __launch_bounds__(256) bwd_stick_ds_kernel(const int32_t* __restrict__ idx, const float* __restrict__ w,
+                                                           const float* __restrict__ dw, float* __restrict__ ds,
+                                                           long long n_rows, int topk, int Nc) {
+  const long long row = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (row >= n_rows) return;
+  const long long p0 = row * topk;
+  int keff = 0;
+  while (keff < topk) {
+    const int c = idx[p0 + keff];
+    if (c < 0 || c >= Nc) break;
+    ++keff;
+  }
+  double R[32];
+  double rest = 1.0;
+  for (int j = 0; j < keff; ++j) {
+    R[j] = rest;
+    rest -= (double)w[p0 + j];
+  }
+  double U = 0.0;
+  for (int j = topk - 1; j >= keff; --j) ds[p0 + j] = 0.f;
+  for (int j = keff - 1; j >= 0; --j) {
+    const double wj = w[p0 + j], dwj = dw[p0 + j];
+    ds[p0 + j] = R[j] > 0.0 ? (float)((wj / R[j]) * ((R[j] - wj) * dwj - U)) : 0.f;
+    U += wj * dwj;
+  }
+}
+
+// q̂ rows for the chunk-summary gradient: [b, t, g][e] = fp32 head-order sum of
+// the group's query rows (the selection's group query).
+template <int D>
+__global__ void __launch_bounds__(256) bwd_qhat_kernel(const uint16_t* __restrict__ q, float* __restrict__ qhat,
+                                                       long long n_rows, int G) {
+  constexpr int D8 = D / 8;
+  const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (u >= n_rows * D8) return;
+  const long long row = u / D8;
+  const int e8 = (int)(u % D8);
+  const uint4* src = reinterpret_cast<const uint4*>(q) + row * G * D8 + e8;
+  float acc[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+  for (int h = 0; h < G; ++h) {
+    const uint4 v = src[(long long)h * D8];
+    acc[0] += bf16_lo(v.x);
+    acc[1] += bf16_hi(v.x);
+    acc[2] += bf16_lo(v.y);
+    acc[3] += bf16_hi(v.y);
+    acc[4] += bf16_lo(v.z);
+    acc[5] += bf16_hi(v.z);
+    acc[6] += bf16_lo(v.w);
+    acc[7] += bf16_hi(v.w);
+  }
+  float4* dst = reinterpret_cast<float4*>(qhat) + row * (D / 4) + e8 * 2;
+  dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+}
+
+// Stick-breaking: the chunk-summary gradient dK̄_i = c_sel sum over the slots
+// that chose chunk i (in token order, from the inverse index) of ds * q̂_t,
+// spread over the chunk's S key rows (mean pool): dK_{iS+s} += dK̄_i / S. Block
+// per (b, g, chunk), thread per dimension.
+template <int D>
+__global__ void __launch_bounds__(D) bwd_stick_dkbar_kernel(const int32_t* __restrict__ offsets,
+                                                            const int32_t* __restrict__ entries,
+                                                            const float* __restrict__ ds,
+                                                            const float* __restrict__ qhat, float* __restrict__ dK,
+                                                            int L, int Hkv, int topk, int Nc, float scale_sel) {
+  const int key = blockIdx.x;
+  const int c = key % Nc, bg = key / Nc;
+  const int b = bg / Hkv, g = bg % Hkv;
+  const int off = offsets[key], cnt = offsets[key + 1] - off;
+  if (cnt <= 0) return;
+  const int e = threadIdx.x;
+  const int slot_div = Hkv * topk;
+  float acc = 0.f;
+  int n = 0;
+  for (; n + 4 <= cnt; n += 4) {  // four slots' loads in flight
+    int p[4];
+    float dv[4], qv[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) p[u] = entries[off + n + u];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      dv[u] = ds[p[u]];
+      qv[u] = qhat[((long long)(p[u] / slot_div) * Hkv + g) * D + e];
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) acc = fmaf(dv[u], qv[u], acc);
+  }
+  for (; n < cnt; ++n) {
+    const int p = entries[off + n];
+    acc = fmaf(ds[p], qhat[((long long)(p / slot_div) * Hkv + g) * D + e], acc);
+  }
+  const float add = scale_sel * acc / (float)kChunk;
+  const long long row0 = ((long long)b * L + (long long)c * kChunk) * Hkv + g;
+  for (int s = 0; s < kChunk; ++s) dK[(row0 + (long long)s * Hkv) * D + e] += add;
+}
+
+// dq_t = sum_j dq'_{t,j} in slot order (one warp per (b, t, g)); with
+// stick-breaking weights also the selection term c_sel sum_j ds_j K̄_{I_j}
+// for every head of the group.
 template <int D>
 __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __restrict__ idx,
                                                            const uint16_t* __restrict__ dqpart, float* __restrict__ dq,
-                                                           long long n_rows, int G, int topk, int Nc) {
+                                                           long long n_rows, int G, int topk, int Nc,
+                                                           const float* __restrict__ ds,
+                                                           const float* __restrict__ kbar32, int L, int Hkv,
+                                                           float scale_sel) {
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -616,6 +732,25 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
       acc[6] += bf16_lo(v.w);
       acc[7] += bf16_hi(v.w);
     }
+    if (ds != nullptr) {  // stick-breaking: c_sel sum_j ds_j K̄_{I_j}, dims [8 e8, 8 e8 + 8) of this head
+      const int e8 = ch % (D / 8);
+      const long long b = row / ((long long)L * Hkv);
+      const int g = (int)(row % Hkv);
+      for (int j = 0; j < keff; ++j) {
+        const float sj = scale_sel * ds[p0 + j];
+        const float4* kb =
+            reinterpret_cast<const float4*>(kbar32 + ((b * Nc + idx[p0 + j]) * Hkv + g) * D) + e8 * 2;
+        const float4 k0 = kb[0], k1 = kb[1];
+        acc[0] = fmaf(sj, k0.x, acc[0]);
+        acc[1] = fmaf(sj, k0.y, acc[1]);
+        acc[2] = fmaf(sj, k0.z, acc[2]);
+        acc[3] = fmaf(sj, k0.w, acc[3]);
+        acc[4] = fmaf(sj, k1.x, acc[4]);
+        acc[5] = fmaf(sj, k1.y, acc[5]);
+        acc[6] = fmaf(sj, k1.z, acc[6]);
+        acc[7] = fmaf(sj, k1.w, acc[7]);
+      }
+    }
     dst[2 * ch] = make_float4(acc[0], acc[1], acc[2], acc[3]);
     dst[2 * ch + 1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
   }
@@ -637,16 +772,50 @@ __global__ void zero_tail_kernel(float* __restrict__ dK, float* __restrict__ dV,
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+// Workspace: bf16 dq partials [slots, G, d]; Δ [rows]; with stick-breaking
+// weights also dw, ds [slots] and q̂ [rows, d] (fp32).
+struct BwdLayout {
+  size_t dqpart, delta, dw, ds, qhat, total;
+};
+BwdLayout bwd_layout(const Dims& D) {
+  const size_t rows = (size_t)D.B * D.L * D.Hkv;
+  BwdLayout lo{};
+  size_t o = 0;
+  lo.dqpart = o;
+  o = align256(o + (size_t)D.slots() * D.G * D.d * sizeof(uint16_t));
+  lo.delta = o;
+  o = align256(o + rows * sizeof(float));
+  if (D.stick) {
+    lo.dw = o;
+    o = align256(o + (size_t)D.slots() * sizeof(float));
+    lo.ds = o;
+    o = align256(o + (size_t)D.slots() * sizeof(float));
+    lo.qhat = o;
+    o = align256(o + rows * D.d * sizeof(float));
+  }
+  lo.total = o;
+  return lo;
+}
+
 template <int D>
 cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, const float* kbar32, const int32_t* idx,
                 const float* w, const void* O, const void* dO, const int32_t* offsets, const int32_t* entries,
                 float* dq, float* dK, float* dV, void* ws, cudaStream_t st) {
   const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
-  uint16_t* dqpart = (uint16_t*)ws;
-  float* delta = (float*)((char*)ws + align256((size_t)Dm.slots() * Dm.G * D * sizeof(uint16_t)));
+  const BwdLayout lo = bwd_layout(Dm);
+  uint16_t* dqpart = (uint16_t*)((char*)ws + lo.dqpart);
+  float* delta = (float*)((char*)ws + lo.delta);
+  float* dwb = Dm.stick ? (float*)((char*)ws + lo.dw) : nullptr;
+  float* dsb = Dm.stick ? (float*)((char*)ws + lo.ds) : nullptr;
+  float* qhat = Dm.stick ? (float*)((char*)ws + lo.qhat) : nullptr;
   cudaError_t e;
-  bwd_delta_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>((const uint16_t*)O, (const uint16_t*)dO, delta,
-                                                                  rows, Dm.G);
+  if (!Dm.stick) {  // Δ_t = sum_j w_j dw_j = dO · O feeds the softmax weights' ds inside the chunk kernel
+    bwd_delta_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>((const uint16_t*)O, (const uint16_t*)dO, delta,
+                                                                    rows, Dm.G);
+  } else {
+    bwd_qhat_kernel<D><<<(unsigned)((rows * (D / 8) + 255) / 256), 256, 0, st>>>((const uint16_t*)q, qhat, rows,
+                                                                                  Dm.G);
+  }
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const long long keys = Dm.keys();
@@ -673,6 +842,9 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.scale_log2 = Dm.scale_attn * 1.4426950408889634f;
     a.scale_attn = Dm.scale_attn;
     a.scale_sel = Dm.scale_sel;
+    a.softmax1 = Dm.softmax1 ? 1 : 0;
+    a.stick = Dm.stick ? 1 : 0;
+    a.dw_out = dwb;
     const size_t smem = sizeof(BwdSmem<D>) + 1024;
     if ((e = cudaFuncSetAttribute(bwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
         cudaSuccess)
@@ -691,7 +863,19 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  bwd_dq_merge_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(idx, dqpart, dq, rows, Dm.G, Dm.topk, Dm.Nc);
+  if (Dm.stick) {
+    bwd_stick_ds_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(idx, w, dwb, dsb, rows, Dm.topk, Dm.Nc);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (keys > 0) {
+      bwd_stick_dkbar_kernel<D><<<(unsigned)keys, D, 0, st>>>(offsets, entries, dsb, qhat, dK, Dm.L, Dm.Hkv, Dm.topk,
+                                                              Dm.Nc, Dm.scale_sel);
+      note_launches(1);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+  }
+  bwd_dq_merge_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(idx, dqpart, dq, rows, Dm.G, Dm.topk, Dm.Nc,
+                                                                      dsb, kbar32, Dm.L, Dm.Hkv, Dm.scale_sel);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int tail0 = Dm.Nc * kChunk;
@@ -714,10 +898,7 @@ unsigned backward_take_status() {
   return v;
 }
 
-size_t backward_workspace(const Dims& D) {
-  return align256((size_t)D.slots() * D.G * D.d * sizeof(uint16_t)) +
-         align256((size_t)D.B * D.L * D.Hkv * sizeof(float));
-}
+size_t backward_workspace(const Dims& D) { return bwd_layout(D).total; }
 
 cudaError_t launch_backward(const Dims& D, const void* q, const void* K, const void* V, const float* kbar32,
                             const int32_t* idx, const float* w, const void* O, const void* dO,

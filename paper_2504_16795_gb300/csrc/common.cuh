@@ -36,9 +36,40 @@ constexpr int kWarp = 32;
 struct Dims {
   int B, L, Hq, Hkv, d, S, topk, G, Nc;
   float scale_sel, scale_attn;
+  bool softmax1, stick;  // variants: softmax-off-by-one inside chunks, stick-breaking chunk weights
   long long slots() const { return (long long)B * L * Hkv * topk; }
   long long keys() const { return (long long)B * Hkv * Nc; }
 };
+
+// Chunk weights of one selection row held by a warp, lane j = slot j (the
+// first keff slots valid, in I' order: latest chunk first): softmax over the
+// scores, or stick-breaking (§3.1.1 "Chunk Weights") — slot j takes
+// sigmoid(s_j) of what the earlier slots left, w_j = b_j prod_{i<j} (1 - b_i).
+// Lanes past keff get 0.
+__device__ __forceinline__ float warp_chunk_weight(float s, bool valid, bool stick) {
+  if (stick) {
+    // 1 - sigmoid(s) = sigmoid(-s), exact for large scores
+    const float b = valid ? 1.f / (1.f + expf(-s)) : 0.f;
+    const float keep = valid ? 1.f / (1.f + expf(s)) : 1.f;
+    const int lane = threadIdx.x & 31;
+    float r = __shfl_up_sync(0xFFFFFFFFu, keep, 1);  // exclusive product: prod over earlier lanes
+    if (lane == 0) r = 1.f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float v = __shfl_up_sync(0xFFFFFFFFu, r, o);
+      if (lane >= o) r *= v;
+    }
+    return valid ? b * r : 0.f;
+  }
+  float m = s;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+  const float ex = valid ? expf(s - m) : 0.f;
+  float z = ex;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
+  return valid ? ex / z : 0.f;
+}
 
 // ------------------------------------------------------------------ bf16
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
@@ -215,6 +246,7 @@ struct DecodeDims {
   int Bq, Hq, Hkv, d, S, topk, G;
   long long Nc;
   float scale_sel, scale_attn;
+  bool softmax1, stick;  // variants as in Dims
 };
 size_t decode_workspace(const DecodeDims& D);
 cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,

@@ -106,9 +106,11 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
 }
 
-// Final top-k per (query, group) and the softmax chunk weights. One warp each.
+// Final top-k per (query, group) and the chunk weights (softmax or
+// stick-breaking). One warp each.
 __global__ void dec_merge_kernel(const unsigned long long* __restrict__ cand, int32_t* __restrict__ idx,
-                                 float* __restrict__ s_sel, float* __restrict__ w, int rows, int nx, int topk) {
+                                 float* __restrict__ s_sel, float* __restrict__ w, int rows, int nx, int topk,
+                                 int stick) {
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
   if (row >= rows) return;
@@ -128,10 +130,8 @@ __global__ void dec_merge_kernel(const unsigned long long* __restrict__ cand, in
     valid = idx[o + lane] >= 0;
     if (valid) s = s_sel[o + lane];
   }
-  const float m = warp_max(s);
-  const float ex = valid ? expf(s - m) : 0.f;
-  const float z = warp_sum(ex);
-  if (lane < topk) w[o + lane] = valid ? ex / z : 0.f;
+  const float wj = warp_chunk_weight(s, valid, stick != 0);
+  if (lane < topk) w[o + lane] = wj;
 }
 
 template <int D>
@@ -148,7 +148,8 @@ __global__ void __launch_bounds__(kThreads) dec_attend_kernel(const uint16_t* __
                                                               const uint16_t* __restrict__ Kmem,
                                                               const uint16_t* __restrict__ Vmem,
                                                               const int32_t* __restrict__ idx, float* __restrict__ Opart,
-                                                              int Hq, int Hkv, int G, int topk, float scale_attn) {
+                                                              int Hq, int Hkv, int G, int topk, float scale_attn,
+                                                              int softmax1) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   AttSmem<D>& sm = *reinterpret_cast<AttSmem<D>*>(smem_raw);
   auto& Ks = sm.K;
@@ -187,7 +188,7 @@ __global__ void __launch_bounds__(kThreads) dec_attend_kernel(const uint16_t* __
     const float x0 = P[hh][lane], x1 = P[hh][lane + 32];
     const float m = warp_max(fmaxf(x0, x1));
     const float e0 = expf(x0 - m), e1 = expf(x1 - m);
-    const float z = warp_sum(e0 + e1);
+    const float z = warp_sum(e0 + e1) + (softmax1 ? expf(-m) : 0.f);  // softmax-off-by-one: the zero logit
     P[hh][lane] = e0 / z;
     P[hh][lane + 32] = e1 / z;
   }
@@ -259,7 +260,7 @@ cudaError_t run(const DecodeDims& D, const void* q, const void* K, const void* V
         cudaSuccess)
       return e;
   }
-  dec_merge_kernel<<<(rows + 7) / 8, 256, 0, st>>>(cand, idx, s_sel, w, rows, lo.nx, D.topk);
+  dec_merge_kernel<<<(rows + 7) / 8, 256, 0, st>>>(cand, idx, s_sel, w, rows, lo.nx, D.topk, D.stick ? 1 : 0);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const size_t att_smem = sizeof(AttSmem<DD>);
@@ -268,7 +269,7 @@ cudaError_t run(const DecodeDims& D, const void* q, const void* K, const void* V
     return e;
   dec_attend_kernel<DD><<<rows * D.topk, kThreads, att_smem, st>>>((const uint16_t*)q, (const uint16_t*)K,
                                                            (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk,
-                                                           D.scale_attn);
+                                                           D.scale_attn, D.softmax1 ? 1 : 0);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   dec_out_kernel<DD><<<rows, 256, 0, st>>>(opart, w, (uint16_t*)O, D.G, D.topk);
@@ -289,7 +290,8 @@ cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void*
                                   (int)sizeof(AttSmem<64>))) != cudaSuccess)
       return e;
     dec_attend_kernel<64><<<rows * D.topk, kThreads, sizeof(AttSmem<64>), st>>>(
-        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk, D.scale_attn);
+        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk, D.scale_attn,
+        D.softmax1 ? 1 : 0);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     dec_out_kernel<64><<<rows, 256, 0, st>>>(opart, w, (uint16_t*)O, D.G, D.topk);
@@ -298,7 +300,8 @@ cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void*
                                   (int)sizeof(AttSmem<128>))) != cudaSuccess)
       return e;
     dec_attend_kernel<128><<<rows * D.topk, kThreads, sizeof(AttSmem<128>), st>>>(
-        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk, D.scale_attn);
+        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk, D.scale_attn,
+        D.softmax1 ? 1 : 0);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     dec_out_kernel<128><<<rows, 256, 0, st>>>(opart, w, (uint16_t*)O, D.G, D.topk);

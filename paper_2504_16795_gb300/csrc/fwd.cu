@@ -11,7 +11,10 @@
 // operand of the second product (no shared-memory round trip). Each chunk is complete, so its softmax needs no online
 // rescaling. The normalised per-slot result O' (bf16) goes to a workspace
 // and a second kernel forms O_t = sum_j w_j O'_{t,j} with the chunk weights
-// w = softmax_j(s_sel) (the "w/o s.b." variant of §4.1), slots in order j.
+// w = softmax_j(s_sel) (the "w/o s.b." variant of §4.1) or, with the
+// stick-breaking flag, the paper's stick-breaking weights over I' (§3.1.1),
+// slots in order j. The softmax-off-by-one flag (§3.1.2) adds the zero logit
+// to every chunk-local softmax.
 #include <cstring>
 
 #include "tc.cuh"
@@ -63,6 +66,7 @@ struct FwdArgs {
   int n_rows;   // B * L * Hq (query rows; a row index past it reads zeros)
   int use_tma;  // G >= 8: each slot's G rows arrive as one swizzled TMA box
   float scale_log2;  // c_att * log2(e)
+  int softmax1;      // softmax-off-by-one inside the chunk
 };
 
 template <int D>
@@ -280,7 +284,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         x[k] = exp2f(fmaf(x[k], a.scale_log2, -ms));
         zz[k & 7] += x[k];
       }
-      const float inv = 1.f / (((zz[0] + zz[1]) + (zz[2] + zz[3])) + ((zz[4] + zz[5]) + (zz[6] + zz[7])));
+      // softmax-off-by-one: the zero logit adds exp(0 - max) to the denominator
+      const float inv = 1.f / ((((zz[0] + zz[1]) + (zz[2] + zz[3])) + ((zz[4] + zz[5]) + (zz[6] + zz[7]))) +
+                               (a.softmax1 ? exp2f(-ms) : 0.f));
       // P into tensor memory: the row's 64 probabilities as 32 bf16 pairs
       uint32_t pk[kChunk / 2];
 #pragma unroll
@@ -355,13 +361,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// O_t = sum_j w_j O'_{t,j}; w = softmax over the selected scores. One warp per (b, t, g).
+// O_t = sum_j w_j O'_{t,j}; w = softmax over the selected scores or stick-breaking. One warp per (b, t, g).
 template <int D>
 __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict__ s_sel,
                                                         const int32_t* __restrict__ idx,
                                                         const uint16_t* __restrict__ Opart, uint16_t* __restrict__ O,
                                                         float* __restrict__ w, long long n_rows, int Hkv, int G,
-                                                        int topk, int Nc) {
+                                                        int topk, int Nc, int stick) {
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -373,10 +379,7 @@ __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict_
     valid = c >= 0 && c < Nc;
     if (valid) s = s_sel[p0 + lane];
   }
-  const float m = warp_max(s);
-  const float ex = valid ? expf(s - m) : 0.f;
-  const float z = warp_sum(ex);
-  const float wj = valid ? ex / z : 0.f;
+  const float wj = warp_chunk_weight(s, valid, stick != 0);
   if (lane < topk) w[p0 + lane] = wj;
   const int keff = __popc(__ballot_sync(0xFFFFFFFFu, valid));
   const int GD8 = G * (D / 8);
@@ -434,6 +437,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.topk = Dm.topk;
     a.Nc = Dm.Nc;
     a.scale_log2 = Dm.scale_attn * 1.4426950408889634f;
+    a.softmax1 = Dm.softmax1 ? 1 : 0;
     const size_t smem = sizeof(FwdSmem<D>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(fwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -451,7 +455,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
   }
   const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
   fwd_merge_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(s_sel, idx, Opart, (uint16_t*)O, w, rows, Dm.Hkv,
-                                                                  Dm.G, Dm.topk, Dm.Nc);
+                                                                  Dm.G, Dm.topk, Dm.Nc, Dm.stick ? 1 : 0);
   note_launches(1);
   return cudaGetLastError();
 }

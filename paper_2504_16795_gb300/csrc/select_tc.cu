@@ -733,7 +733,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
     const int32_t* __restrict__ cand_n, const float* __restrict__ cand_d, const float4* __restrict__ cand_s, int kbuf,
     const float* __restrict__ qh32, const float* __restrict__ kbar32, int32_t* __restrict__ idx,
     float* __restrict__ s_sel, float* __restrict__ w, int Bq, int Hkv, int Nc, int n_split, int range, int topk,
-    float scale_sel) {
+    float scale_sel, int stick) {
   extern __shared__ __align__(16) unsigned char mg_smem[];
   float* stage_all = reinterpret_cast<float*>(mg_smem);  // [warps][32 rows][D]
   float* qs = stage_all + kMergeWarps * 32 * D;           // [D]
@@ -890,10 +890,8 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
     valid = idx[o + lane] >= 0;
     if (valid) sv = s_sel[o + lane];
   }
-  const float m = warp_max(sv);
-  const float ex = valid ? expf(sv - m) : 0.f;
-  const float z = warp_sum(ex);
-  if (lane < topk) w[o + lane] = valid ? ex / z : 0.f;
+  const float wj = warp_chunk_weight(sv, valid, stick != 0);
+  if (lane < topk) w[o + lane] = wj;
 }
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -1139,7 +1137,7 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
     return e;
   dtc_merge_kernel<DD><<<(unsigned)rows, kMergeWarps * 32, mg_smem, st>>>(
       a.cand_l, a.cand_u, a.cand_c, a.cand_n, a.cand_d, a.cand_s, SelCfg<KT>::kBuf, qh32, kbar32, idx, s_sel, w, Dm.Bq,
-      Dm.Hkv, (int)Dm.Nc, lo.n_split, lo.range, Dm.topk, Dm.scale_sel);
+      Dm.Hkv, (int)Dm.Nc, lo.n_split, lo.range, Dm.topk, Dm.scale_sel, Dm.stick ? 1 : 0);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return launch_decode_attend(Dm, q, K, V, idx, w, O, (float*)(base + lo.opart), st);

@@ -60,18 +60,19 @@ def host_inputs(w: synth.Workload, with_dO=True):
     return out
 
 
-def oracle_prefill(w: synth.Workload, bits: dict, backward=True, token_mask=None):
-    """Oracle results for a prefill workload from its bf16 inputs."""
+def oracle_prefill(w: synth.Workload, bits: dict, backward=True, token_mask=None, inner="softmax", weights="softmax"):
+    """Oracle results for a prefill workload from its bf16 inputs (variants as in oracle.forward)."""
     q = synth.bf16_to_f64(bits["q"])
     K = synth.bf16_to_f64(bits["K"])
     V = synth.bf16_to_f64(bits["V"])
     S, k = w.S, w.topk
     kbar32 = oracle.pool(K, S, f32=True)
     idx, s_sel, gap = oracle.select(q, kbar32, S, k, f32=True, token_mask=token_mask)
-    O, wts = oracle.forward(q, K, V, idx, s_sel, S, token_mask=token_mask)
+    O, wts = oracle.forward(q, K, V, idx, s_sel, S, token_mask=token_mask, inner=inner, weights=weights)
     res = dict(kbar32=kbar32, idx=idx, s_sel=s_sel, gap=gap, O=O, w=wts)
     if backward:
         dO = synth.bf16_to_f64(bits["dO"])
         kbar64 = oracle.pool(K, S)
-        res.update(oracle.backward(q, K, V, kbar64, idx, s_sel, dO, S, token_mask=token_mask))
+        res.update(oracle.backward(q, K, V, kbar64, idx, s_sel, dO, S, token_mask=token_mask, inner=inner,
+                                   weights=weights))
     return res

@@ -81,6 +81,25 @@ def test_shape_validation(lib, kw, code):
     assert call_forward(lib, shape(**kw), ws_bytes=0) == code
 
 
+def test_unknown_variant_flags_are_unsupported(lib):
+    c = shape().c()
+    c.flags = 4
+    vp = ctypes.c_void_p
+    assert lib.hsa_forward(ctypes.byref(c), *[vp(FAKE)] * 10, 1 << 30, None) == UNSUPPORTED
+    d = hsa.DecodeShape(Bq=4, Hq=8, Hkv=1, d=128, n_chunks=100).c()
+    d.flags = 8
+    assert lib.hsa_decode(ctypes.byref(d), *[vp(FAKE)] * 9, 1 << 30, None) == UNSUPPORTED
+    with pytest.raises(ValueError):
+        shape(weights="uniform").flags
+
+
+def test_stick_breaking_backward_needs_its_extra_workspace(lib):
+    base = hsa.workspace_size(hsa.HSA_OP_BACKWARD, shape())
+    stick = hsa.workspace_size(hsa.HSA_OP_BACKWARD, shape(weights="stick"))
+    s = shape()
+    assert stick == base + 2 * s.B * s.L * s.Hkv * s.topk * 4 + s.B * s.L * s.Hkv * s.d * 4
+
+
 def test_null_and_misaligned_pointers_are_rejected(lib):
     s = shape()
     assert call_forward(lib, s, q=0) == INVALID

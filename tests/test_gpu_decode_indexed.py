@@ -35,17 +35,22 @@ def small_memory(w, bits=None):
     return bits, qd, Kmem, Vmem, kbar32.view(Nc, w.Hkv, d)
 
 
-def check_against_oracle(w, bits=None):
+def check_against_oracle(w, bits=None, inner="softmax", weights="softmax", exact=False):
     bits, qd, Kmem, Vmem, kbar32 = small_memory(w, bits)
-    dshape = hsa.DecodeShape(Bq=w.Bq, Hq=w.Hq, Hkv=w.Hkv, d=w.d, n_chunks=w.Nc, topk=w.topk)
-    index = hsa.decode_index(dshape, kbar32)
-    O, idx, s_sel, wts = hsa.decode_indexed(dshape, qd, Kmem, Vmem, kbar32, index)
+    dshape = hsa.DecodeShape(Bq=w.Bq, Hq=w.Hq, Hkv=w.Hkv, d=w.d, n_chunks=w.Nc, topk=w.topk, inner=inner,
+                             weights=weights)
+    if exact:
+        O, idx, s_sel, wts = hsa.decode(dshape, qd, Kmem, Vmem, kbar32)
+    else:
+        index = hsa.decode_index(dshape, kbar32)
+        O, idx, s_sel, wts = hsa.decode_indexed(dshape, qd, Kmem, Vmem, kbar32, index)
     torch.cuda.synchronize()
     hsa.device_check()
     K = synth.bf16_to_f64(bits["K"])[0]
     V = synth.bf16_to_f64(bits["V"])[0]
     kb = oracle.pool(K[None], w.S, f32=True)[0]
-    ref = oracle.decode(synth.bf16_to_f64(bits["q"])[0], K, V, kb, w.S, w.topk, f32=True)
+    ref = oracle.decode(synth.bf16_to_f64(bits["q"])[0], K, V, kb, w.S, w.topk, f32=True, inner=inner,
+                        weights=weights)
     assert np.array_equal(idx.cpu().numpy(), ref["idx"])
     assert np.array_equal(s_sel.cpu().numpy(), ref["s_sel"].astype(np.float32))
     assert_close("decode w", wts.cpu().numpy(), ref["w"], max_abs=1e-5, rel=1e-5)
@@ -65,6 +70,15 @@ def test_indexed_decode_matches_oracle(name):
     kw = CASES[name]
     w = synth.Workload("dec-ix", 61, B=1, S=64, backward=False, decode=True, needle_chunks=kw["Bq"], **kw)
     check_against_oracle(w)
+
+
+@pytest.mark.parametrize("exact", [False, True])
+@pytest.mark.parametrize("variant", [("softmax1", "softmax"), ("softmax", "stick"), ("softmax1", "stick")])
+def test_decode_variants_match_oracle(variant, exact):
+    # softmax-off-by-one inside chunks (§3.1.2) and stick-breaking chunk weights (§3.1.1)
+    kw = CASES["d64 k8 two groups"]
+    w = synth.Workload("dec-var", 63, B=1, S=64, backward=False, decode=True, needle_chunks=kw["Bq"], **kw)
+    check_against_oracle(w, inner=variant[0], weights=variant[1], exact=exact)
 
 
 def test_indexed_decode_equal_summaries_take_the_exact_path():

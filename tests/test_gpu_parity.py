@@ -29,12 +29,12 @@ def built():
     hsa.load()
 
 
-def shape_of(w):
-    return hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk)
+def shape_of(w, inner="softmax", weights="softmax"):
+    return hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk, inner=inner, weights=weights)
 
 
-def run_gpu(w, bits, backward=True):
-    shape = shape_of(w)
+def run_gpu(w, bits, backward=True, inner="softmax", weights="softmax"):
+    shape = shape_of(w, inner, weights)
     q, K, V = (to_device_bf16(bits[n]) for n in ("q", "K", "V"))
     wss = hsa.Workspaces(shape, q.device)
     fwd = hsa.hsa_forward_path(shape, q, K, V, wss)
@@ -46,10 +46,10 @@ def run_gpu(w, bits, backward=True):
     return out
 
 
-def check_prefill(w, backward=True, bits=None):
+def check_prefill(w, backward=True, bits=None, inner="softmax", weights="softmax"):
     bits = bits or host_inputs(w, with_dO=backward)
-    got = run_gpu(w, bits, backward)
-    ref = oracle_prefill(w, bits, backward)
+    got = run_gpu(w, bits, backward, inner, weights)
+    ref = oracle_prefill(w, bits, backward, inner=inner, weights=weights)
     # chunk summaries: bit-exact fp32 and its bf16 rounding
     kb = got["kbar32"].cpu().numpy()
     assert np.array_equal(kb, ref["kbar32"].astype(np.float32))
@@ -102,6 +102,17 @@ SMALL = {
 @pytest.mark.parametrize("name", list(SMALL))
 def test_prefill_matches_oracle(name):
     check_prefill(SMALL[name])
+
+
+@pytest.mark.parametrize("variant", [("softmax1", "softmax"), ("softmax", "stick"), ("softmax1", "stick")])
+@pytest.mark.parametrize("name", ["tiny (config 1)", "pretrain shape, ragged", "G16 d128 k16"])
+def test_prefill_variants_match_oracle(name, variant):
+    # softmax-off-by-one inside chunks (§3.1.2) and stick-breaking chunk weights (§3.1.1)
+    inner, weights = variant
+    got, ref = check_prefill(SMALL[name], inner=inner, weights=weights)
+    keff = (ref["idx"] >= 0).sum(-1)
+    if weights == "stick":  # the slots take less than the whole stick
+        assert (ref["w"].sum(-1)[keff > 0] < 1.0).all()
 
 
 @pytest.mark.parametrize("L", [50, 64, 65, 128])

@@ -45,9 +45,11 @@ def lib():
         L.hsa_oracle_forward.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, ci, ci, vp, vp, vp]
         L.hsa_oracle_backward.argtypes = [vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, cd, ci, ci,
                                           vp, vp, vp, vp, vp, vp]
+        L.hsa_oracle_select_backward.argtypes = [vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, ci, cd, vp, vp, vp]
         L.hsa_oracle_decode_select.argtypes = [vp, vp, i64, ci, ci, ci, ci, ci, cd, ci, vp, vp, vp]
         L.hsa_oracle_decode_attend.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, ci, cd, ci, ci, vp, vp]
         for f in (L.hsa_oracle_pool, L.hsa_oracle_select, L.hsa_oracle_forward, L.hsa_oracle_backward,
+                  L.hsa_oracle_select_backward,
                   L.hsa_oracle_decode_select, L.hsa_oracle_decode_attend):
             f.restype = None
         L.hsa_oracle_threads.restype = ci
@@ -151,6 +153,23 @@ def backward(q, K, V, kbar, idx, s_sel, dO, S, scale_sel=None, scale_attn=None, 
                               float(scale_sel), float(scale_attn), *_variant(inner, weights), _p(m), _p(dq), _p(dK),
                               _p(dV), _p(dkbar), _p(ds))
     return dict(dq=dq, dK=dK, dV=dV, dkbar=dkbar, ds=ds)
+
+
+def select_backward(q, kbar, idx, ds, S, scale_sel=None):
+    """The selection chain for a given score gradient ds [B,L,Hkv,k] -> dict(dq, dK, dkbar)."""
+    q, kbar, ds = _f64(q), _f64(kbar), _f64(ds)
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    B, L, Hq, d = q.shape
+    Hkv = kbar.shape[2]
+    topk = idx.shape[-1]
+    if scale_sel is None:
+        scale_sel = default_scales(Hq // Hkv, d)[0]
+    dq = np.zeros_like(q)
+    dK = np.zeros((B, L, Hkv, d))
+    dkbar = np.zeros_like(kbar)
+    lib().hsa_oracle_select_backward(_p(q), _p(kbar), _p(idx), _p(ds), B, L, Hq, Hkv, d, S, topk, float(scale_sel),
+                                     _p(dq), _p(dK), _p(dkbar))
+    return dict(dq=dq, dK=dK, dkbar=dkbar)
 
 
 def decode_select(q, kbar, topk, scale_sel=None, f32=False):

@@ -415,6 +415,46 @@ void hsa_oracle_backward(const double* q, const double* K, const double* V, cons
         }
 }
 
+/* ------------------------------------------------------------------ selection backward
+ * The selection chain alone, for a given score gradient ds [B,L,Hkv,topk]
+ * (Appendix A: the scores s = c_sel q̂·K̄ receive gradient through the chunk
+ * weights; several layers sharing one selection add their ds first):
+ *   dq_h    = c_sel sum_j ds_j K̄_{I_j}         (every head h of the group)
+ *   dK̄_i    = c_sel sum_{(t,j): I_j = i} ds_j q̂_t
+ *   dK_{iS+s} = dK̄_i / S                       (mean pool); other rows 0
+ */
+void hsa_oracle_select_backward(const double* q, const double* kbar, const int32_t* idx, const double* ds, int B,
+                                int L, int Hq, int Hkv, int d, int S, int topk, double scale_sel, double* dq,
+                                double* dK, double* dkbar) {
+    const int G = Hq / Hkv, Nc = L / S;
+    for (int64_t u = 0; u < (int64_t)B * L * Hq * d; ++u) dq[u] = 0.0;
+    for (int64_t u = 0; u < (int64_t)B * L * Hkv * d; ++u) dK[u] = 0.0;
+    for (int64_t u = 0; u < (int64_t)B * Nc * Hkv * d; ++u) dkbar[u] = 0.0;
+    double* qhat = (double*)malloc(sizeof(double) * (size_t)d);
+    for (int b = 0; b < B; ++b)
+        for (int t = 0; t < L; ++t)
+            for (int g = 0; g < Hkv; ++g) {
+                const int64_t o = at4(b, t, g, 0, L, Hkv, topk);
+                const int keff = count_selected(idx + o, topk);
+                if (keff == 0) continue;
+                group_query(q + at4(b, t, 0, 0, L, Hq, d), G, g, d, 0, qhat);
+                for (int j = 0; j < keff; ++j) {
+                    const int64_t i = idx[o + j];
+                    for (int hh = 0; hh < G; ++hh)
+                        for (int e = 0; e < d; ++e)
+                            dq[at4(b, t, g * G + hh, e, L, Hq, d)] += scale_sel * ds[o + j] * kbar[at4(b, i, g, e, Nc, Hkv, d)];
+                    for (int e = 0; e < d; ++e) dkbar[at4(b, i, g, e, Nc, Hkv, d)] += scale_sel * ds[o + j] * qhat[e];
+                }
+            }
+    for (int b = 0; b < B; ++b)
+        for (int i = 0; i < Nc; ++i)
+            for (int g = 0; g < Hkv; ++g)
+                for (int e = 0; e < d; ++e)
+                    for (int s = 0; s < S; ++s)
+                        dK[at4(b, (int64_t)i * S + s, g, e, L, Hkv, d)] = dkbar[at4(b, i, g, e, Nc, Hkv, d)] / (double)S;
+    free(qhat);
+}
+
 /* ------------------------------------------------------------------ decode
  * One query token per batch row sitting right after a memory of Nc complete
  * chunks (§3.2 "Inference": only the chunk summaries are scanned, then the k

@@ -40,6 +40,9 @@ MUTATIONS = {
                                                      "dsl[j] = (1.0 - beta) * w[j] * dw[j];"),
     "stick-breaking gradient over earlier slots": ("for (int j = keff - 1; j >= 0; --j) {",
                                                    "for (int j = 0; j < keff; ++j) {"),
+    "selection-chain pool share not divided by S": (
+        "dK[at4(b, (int64_t)i * S + s, g, e, L, Hkv, d)] = dkbar[at4(b, i, g, e, Nc, Hkv, d)] / (double)S;",
+        "dK[at4(b, (int64_t)i * S + s, g, e, L, Hkv, d)] = dkbar[at4(b, i, g, e, Nc, Hkv, d)];"),
 }
 
 

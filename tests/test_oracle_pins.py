@@ -456,6 +456,49 @@ def test_variant_backward_matches_central_finite_differences(inner, weights, top
         fd_check(name, arr, setter, f, g["d" + name], 50, rng)
 
 
+# ----------------------------------------------------------------------------- the selection chain on its own
+# (layers that share one selection add their score gradients, then the chain runs once)
+
+def test_selection_backward_is_the_gradient_of_the_scores_against_fixed_weights():
+    # loss = sum ds * s_sel(q, K) with ds fixed: its gradient is exactly the selection chain
+    rng = np.random.default_rng(17)
+    B, L, S, Hq, Hkv, d, k = 1, 160, 16, 4, 2, 6, 3
+    q, K = rng.standard_normal((B, L, Hq, d)), rng.standard_normal((B, L, Hkv, d))
+    kbar = oracle.pool(K, S)
+    idx0, _, _ = oracle.select(q, kbar, S, k)
+    ds = rng.standard_normal(idx0.shape) * (idx0 >= 0)
+    g = oracle.select_backward(q, kbar, idx0, ds, S)
+
+    for name, arr in (("q", q), ("K", K)):
+        flat = arr.reshape(-1)
+
+        def setter(p, v, flat=flat):
+            flat[p] = v
+            return None
+
+        def f(_):
+            kb = oracle.pool(K, S)
+            idx, s_sel, _ = oracle.select(q, kb, S, k)
+            return float((np.where(idx >= 0, s_sel, 0.0) * ds).sum()), idx
+
+        fd_check(name, arr, setter, f, g["d" + name], 60, rng)
+
+
+def test_full_backward_is_attention_part_plus_selection_chain():
+    rng = np.random.default_rng(19)
+    B, L, S, Hq, Hkv, d, k = 2, 130, 8, 4, 2, 6, 3
+    q, K, V, dO = (rng.standard_normal(s) for s in [(B, L, Hq, d), (B, L, Hkv, d), (B, L, Hkv, d), (B, L, Hq, d)])
+    kbar = oracle.pool(K, S)
+    idx, s_sel, _ = oracle.select(q, kbar, S, k)
+    full = oracle.backward(q, K, V, kbar, idx, s_sel, dO, S)
+    att = oracle.backward(q, K, V, kbar, idx, s_sel, dO, S, scale_sel=1e-300)  # selection terms vanish
+    sel = oracle.select_backward(q, kbar, idx, full["ds"], S)
+    np.testing.assert_allclose(att["ds"], full["ds"], atol=1e-14)
+    np.testing.assert_allclose(att["dq"] + sel["dq"], full["dq"], atol=1e-12)
+    np.testing.assert_allclose(att["dK"] + sel["dK"], full["dK"], atol=1e-12)
+    np.testing.assert_allclose(sel["dkbar"], full["dkbar"], atol=1e-12)
+
+
 # ----------------------------------------------------------------------------- decode (Section 3.2, Inference)
 
 def test_decode_equals_the_forward_row_after_the_memory():

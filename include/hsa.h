@@ -92,7 +92,9 @@ typedef enum {
     HSA_OP_SELECT = 1,
     HSA_OP_INDEX = 2,
     HSA_OP_FORWARD = 3,
-    HSA_OP_BACKWARD = 4
+    HSA_OP_BACKWARD = 4,
+    HSA_OP_BACKWARD_ATTENTION = 5,
+    HSA_OP_SELECT_BACKWARD = 6
 } hsa_op_t;
 
 /* Human-readable name of a status code (static storage). */
@@ -209,6 +211,47 @@ hsa_status_t hsa_backward(const hsa_shape_t* shape, const void* q, const void* K
                           const float* kbar32, const int32_t* idx, const float* w, const void* O, const void* dO,
                           const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,
                           void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/*
+ * Layers that share one selection (the paper shares K, V and the retrieved
+ * chunks across its HSA layers, §3.1, and may select with its own q_sel and
+ * K^slc): each layer's backward is hsa_backward_attention, which adds that
+ * layer's score gradient into ds_accum; the selection chain then runs once,
+ * hsa_select_backward, on the summed ds. hsa_backward equals
+ * hsa_backward_attention followed by hsa_select_backward with q_sel = q and
+ * K^slc = K (outputs added).
+ *
+ * hsa_backward_attention (Algorithms 2 and 3 without the selection chain):
+ *   Inputs as in hsa_backward, without kbar32 and O.
+ *   dq [B,L,Hq,d], dK, dV [B,L,Hkv,d] fp32: the attention's gradients (fully written).
+ *   ds_accum [B,L,Hkv,topk] fp32, in/out: ds of every slot is added (padding
+ *     slots add 0); ds_j = w_j (dw_j - sum_k w_k dw_k) for softmax weights, the
+ *     stick-breaking form for HSA_FLAG_STICK_BREAKING (see hsa_backward).
+ *   Needs workspace HSA_OP_BACKWARD_ATTENTION.
+ */
+hsa_status_t hsa_backward_attention(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
+                                    const int32_t* idx, const float* w, const void* dO, const int32_t* offsets,
+                                    const int32_t* entries, float* dq, float* dK, float* dV, float* ds_accum,
+                                    void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/*
+ * hsa_select_backward (Appendix A: the selection scores s = c_sel q̂_sel·K̄_sel
+ * receive gradient through the chunk weights):
+ *   shape    the selection problem: B, L, S, topk, Hkv, Hq and d of q_sel
+ *            (d_sel in {64, 128}), scale_sel; flags and scale_attn unused.
+ *   q_sel    [B,L,Hq,d] bf16; kbar_sel [B,L/S,Hkv,d] fp32 (hsa_chunk_pool of K^slc);
+ *   idx, offsets, entries: the shared selection and its inverse index;
+ *   ds       [B,L,Hkv,topk] fp32 (summed over the layers).
+ *   dq_sel   [B,L,Hq,d] fp32 = c_sel sum_j ds_j K̄_sel[I_j] for every head of the
+ *            group (fully written).
+ *   dK_sel   [B,L,Hkv,d] fp32: dK̄_sel / S on the S rows of every complete
+ *            chunk, dK̄_sel[i] = c_sel sum over the slots that chose i of ds q̂_sel
+ *            (in index order); 0 elsewhere (fully written).
+ *   Needs workspace HSA_OP_SELECT_BACKWARD.
+ */
+hsa_status_t hsa_select_backward(const hsa_shape_t* shape, const void* q_sel, const float* kbar_sel,
+                                 const int32_t* idx, const float* ds, const int32_t* offsets, const int32_t* entries,
+                                 float* dq_sel, float* dK_sel, void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /*
  * Decode against a resident memory (§3.2 "Inference": only the chunk

@@ -7,6 +7,8 @@ its calls.
 from .binding import (  # noqa: F401
     CHUNK,
     HSA_OP_BACKWARD,
+    HSA_OP_BACKWARD_ATTENTION,
+    HSA_OP_SELECT_BACKWARD,
     HSA_OP_FORWARD,
     HSA_OP_INDEX,
     HSA_OP_SELECT,
@@ -15,6 +17,8 @@ from .binding import (  # noqa: F401
     Shape,
     Workspaces,
     backward,
+    backward_attention,
+    select_backward,
     build_index,
     chunk_pool,
     decode,

@@ -16,6 +16,7 @@ import torch
 from . import build as _build
 
 HSA_OP_SELECT, HSA_OP_INDEX, HSA_OP_FORWARD, HSA_OP_BACKWARD = 1, 2, 3, 4
+HSA_OP_BACKWARD_ATTENTION, HSA_OP_SELECT_BACKWARD = 5, 6
 CHUNK = 64
 
 
@@ -130,6 +131,8 @@ def load():
     L.hsa_build_index.argtypes = [sp, vp, vp, vp, vp, sz, vp]
     L.hsa_forward.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     L.hsa_backward.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    L.hsa_backward_attention.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    L.hsa_select_backward.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     L.hsa_decode.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     L.hsa_decode_noalloc.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
     L.hsa_decode_index_size.restype = sz
@@ -279,6 +282,41 @@ def backward(shape: Shape, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq=
                                _ptr(dO), _ptr(offsets), _ptr(entries), _ptr(dq), _ptr(dK), _ptr(dV), _ptr(wsp), nb,
                                _stream(dev)), "hsa_backward")
     return dq, dK, dV
+
+
+def backward_attention(shape: Shape, q, K, V, idx, w, dO, offsets, entries, ds_accum=None, dq=None, dK=None, dV=None,
+                       ws=None):
+    """The attention's gradients of one layer; its score gradient is added into ds_accum (zeros if None)."""
+    _need(dO, "dO", torch.bfloat16, (shape.B, shape.L, shape.Hq, shape.d))
+    dev = q.device
+    dq = torch.empty(q.shape, dtype=torch.float32, device=dev) if dq is None else dq
+    dK = torch.empty(K.shape, dtype=torch.float32, device=dev) if dK is None else dK
+    dV = torch.empty(V.shape, dtype=torch.float32, device=dev) if dV is None else dV
+    if ds_accum is None:
+        ds_accum = torch.zeros((shape.B, shape.L, shape.Hkv, shape.topk), dtype=torch.float32, device=dev)
+    nb = workspace_size(HSA_OP_BACKWARD_ATTENTION, shape)
+    wsp = _workspace(nb, dev, ws)
+    s = shape.c()
+    _check(load().hsa_backward_attention(ctypes.byref(s), _ptr(q), _ptr(K), _ptr(V), _ptr(idx), _ptr(w), _ptr(dO),
+                                         _ptr(offsets), _ptr(entries), _ptr(dq), _ptr(dK), _ptr(dV), _ptr(ds_accum),
+                                         _ptr(wsp), nb, _stream(dev)), "hsa_backward_attention")
+    return dq, dK, dV, ds_accum
+
+
+def select_backward(shape: Shape, q_sel, kbar_sel, idx, ds, offsets, entries, dq_sel=None, dK_sel=None, ws=None):
+    """The selection chain once for the summed score gradient: (dq_sel, dK_sel)."""
+    _need(q_sel, "q_sel", torch.bfloat16, (shape.B, shape.L, shape.Hq, shape.d))
+    dev = q_sel.device
+    dq_sel = torch.empty(q_sel.shape, dtype=torch.float32, device=dev) if dq_sel is None else dq_sel
+    if dK_sel is None:
+        dK_sel = torch.empty((shape.B, shape.L, shape.Hkv, shape.d), dtype=torch.float32, device=dev)
+    nb = workspace_size(HSA_OP_SELECT_BACKWARD, shape)
+    wsp = _workspace(nb, dev, ws)
+    s = shape.c()
+    _check(load().hsa_select_backward(ctypes.byref(s), _ptr(q_sel), _ptr(kbar_sel), _ptr(idx), _ptr(ds), _ptr(offsets),
+                                      _ptr(entries), _ptr(dq_sel), _ptr(dK_sel), _ptr(wsp), nb, _stream(dev)),
+           "hsa_select_backward")
+    return dq_sel, dK_sel
 
 
 def decode(shape: DecodeShape, q, K_mem, V_mem, kbar32, O=None, idx=None, s_sel=None, w=None, ws=None):

@@ -108,6 +108,8 @@ size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {
     case HSA_OP_INDEX: return hsa::index_workspace(D);
     case HSA_OP_FORWARD: return hsa::forward_workspace(D);
     case HSA_OP_BACKWARD: return hsa::backward_workspace(D);
+    case HSA_OP_BACKWARD_ATTENTION: return hsa::backward_attention_workspace(D);
+    case HSA_OP_SELECT_BACKWARD: return hsa::select_backward_workspace(D);
   }
   return 0;
 }
@@ -202,6 +204,53 @@ hsa_status_t hsa_backward(const hsa_shape_t* shape, const void* q, const void* K
   if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
   return cuda_status(
       hsa::launch_backward(D, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq, dK, dV, ws, stream));
+}
+
+hsa_status_t hsa_backward_attention(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
+                                    const int32_t* idx, const float* w, const void* dO, const int32_t* offsets,
+                                    const int32_t* entries, float* dq, float* dK, float* dV, float* ds_accum,
+                                    void* ws, size_t ws_bytes, cudaStream_t stream) {
+  Dims D;
+  hsa_status_t st = resolve(shape, &D);
+  if (st != HSA_OK) return st;
+  if (empty(D)) return HSA_OK;
+  HSA_REQUIRE_PTR(q);
+  HSA_REQUIRE_PTR(K);
+  HSA_REQUIRE_PTR(V);
+  HSA_REQUIRE_PTR(idx);
+  HSA_REQUIRE_PTR(w);
+  HSA_REQUIRE_PTR(dO);
+  HSA_REQUIRE_PTR(offsets);
+  HSA_REQUIRE_PTR(entries);
+  HSA_REQUIRE_PTR(dq);
+  HSA_REQUIRE_PTR(dK);
+  HSA_REQUIRE_PTR(dV);
+  HSA_REQUIRE_PTR(ds_accum);
+  const size_t need = hsa::backward_attention_workspace(D);
+  if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
+  return cuda_status(hsa::launch_backward_attention(D, q, K, V, idx, w, dO, offsets, entries, dq, dK, dV, ds_accum,
+                                                    ws, stream));
+}
+
+hsa_status_t hsa_select_backward(const hsa_shape_t* shape, const void* q_sel, const float* kbar_sel,
+                                 const int32_t* idx, const float* ds, const int32_t* offsets, const int32_t* entries,
+                                 float* dq_sel, float* dK_sel, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  Dims D;
+  hsa_status_t st = resolve(shape, &D);
+  if (st != HSA_OK) return st;
+  if (empty(D)) return HSA_OK;
+  HSA_REQUIRE_PTR(q_sel);
+  if (D.Nc > 0) HSA_REQUIRE_PTR(kbar_sel);
+  HSA_REQUIRE_PTR(idx);
+  HSA_REQUIRE_PTR(ds);
+  HSA_REQUIRE_PTR(offsets);
+  HSA_REQUIRE_PTR(entries);
+  HSA_REQUIRE_PTR(dq_sel);
+  HSA_REQUIRE_PTR(dK_sel);
+  const size_t need = hsa::select_backward_workspace(D);
+  if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+  return cuda_status(
+      hsa::launch_select_backward(D, q_sel, kbar_sel, idx, ds, offsets, entries, dq_sel, dK_sel, ws, stream));
 }
 
 namespace {

@@ -103,8 +103,9 @@ struct BwdArgs {
   int use_tma;  // G >= 8: each slot's G rows arrive as one swizzled TMA box
   float scale_log2, scale_attn, scale_sel;
   int softmax1;   // softmax-off-by-one inside the chunk
-  int stick;      // stick-breaking chunk weights: write dw per slot, no selection term here
-  float* dw_out;  // [slots] (stick-breaking only)
+  int dw_mode;    // write dw per slot and leave the selection terms to later passes
+                  // (stick-breaking weights, or the attention-only backward)
+  float* dw_out;  // [slots] (dw_mode only)
 };
 
 // TMEM columns
@@ -454,8 +455,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       // softmax weights: ds = w (dw - Δ), folded in here; stick-breaking weights
       // need every slot's dw first, so the slot's dw goes out and a later pass
       // adds the selection terms
-      const float dsv = a.stick ? 0.f : wv * (dw - dl);
-      if (a.stick && hf == 0 && (r & (a.G - 1)) == 0 && pv >= 0) a.dw_out[pv] = dw;
+      const float dsv = a.dw_mode ? 0.f : wv * (dw - dl);
+      if (a.dw_mode && hf == 0 && (r & (a.G - 1)) == 0 && pv >= 0) a.dw_out[pv] = dw;
       // hand the slot id to the epilogue warps (three buffers: step i+3 runs
       // after S of step i+3, which the MMA thread issues only after the dq
       // product of step i+1, which waits for the epilogue of step i to have
@@ -596,9 +597,12 @@ __global__ void __launch_bounds__(256) bwd_delta_kernel(const uint16_t* __restri
 // U_j = sum_{k>j} w_k dw_k. One thread per (b, t, g) row; R in double (a
 // slot that finds almost no stick left has almost no weight, and its ds stays
 // small whatever R's rounding).
-__global__ void __launch_bounds__(256) bwd_stick_ds_kernel(const int32_t* __restrict__ idx, const float* __restrict__ w,
-                                                           const float* __restrict__ dw, float* __restrict__ ds,
-                                                           long long n_rows, int topk, int Nc) {
+//
+// Softmax weights (the attention-only backward): ds_j = w_j (dw_j - sum_k w_k dw_k).
+// accumulate: ds += (layers sharing one selection add their score gradients).
+__global__ void __launch_bounds__(256) bwd_ds_kernel(const int32_t* __restrict__ idx, const float* __restrict__ w,
+                                                     const float* __restrict__ dw, float* __restrict__ ds,
+                                                     long long n_rows, int topk, int Nc, int stick, int accumulate) {
   const long long row = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (row >= n_rows) return;
   const long long p0 = row * topk;
@@ -608,6 +612,14 @@ __global__ void __launch_bounds__(256) bwd_stick_ds_kernel(const int32_t* __rest
     if (c < 0 || c >= Nc) break;
     ++keff;
   }
+  auto put = [&](int j, float v) { ds[p0 + j] = accumulate ? ds[p0 + j] + v : v; };
+  for (int j = topk - 1; j >= keff; --j) put(j, 0.f);
+  if (!stick) {
+    double wdw = 0.0;
+    for (int j = 0; j < keff; ++j) wdw += (double)w[p0 + j] * dw[p0 + j];
+    for (int j = 0; j < keff; ++j) put(j, (float)(w[p0 + j] * (dw[p0 + j] - wdw)));
+    return;
+  }
   double R[32];
   double rest = 1.0;
   for (int j = 0; j < keff; ++j) {
@@ -615,11 +627,53 @@ __global__ void __launch_bounds__(256) bwd_stick_ds_kernel(const int32_t* __rest
     rest -= (double)w[p0 + j];
   }
   double U = 0.0;
-  for (int j = topk - 1; j >= keff; --j) ds[p0 + j] = 0.f;
   for (int j = keff - 1; j >= 0; --j) {
     const double wj = w[p0 + j], dwj = dw[p0 + j];
-    ds[p0 + j] = R[j] > 0.0 ? (float)((wj / R[j]) * ((R[j] - wj) * dwj - U)) : 0.f;
+    put(j, R[j] > 0.0 ? (float)((wj / R[j]) * ((R[j] - wj) * dwj - U)) : 0.f);
     U += wj * dwj;
+  }
+}
+
+// Selection chain into the group query: dq_sel[t, h] = c_sel sum_j ds_j K̄_{I_j}
+// for every head h of the group (one warp per (b, t, g); every element written).
+template <int D>
+__global__ void __launch_bounds__(256) sel_dq_kernel(const int32_t* __restrict__ idx, const float* __restrict__ ds,
+                                                     const float* __restrict__ kbar32, float* __restrict__ dq,
+                                                     long long n_rows, int G, int topk, int Nc, int L, int Hkv,
+                                                     float scale_sel) {
+  const int lane = threadIdx.x & 31;
+  const long long row = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (row >= n_rows) return;
+  const long long p0 = row * topk;
+  bool valid = false;
+  if (lane < topk) {
+    const int c = idx[p0 + lane];
+    valid = c >= 0 && c < Nc;
+  }
+  const int keff = __popc(__ballot_sync(0xFFFFFFFFu, valid));
+  const long long b = row / ((long long)L * Hkv);
+  const int g = (int)(row % Hkv);
+  float4* dst = reinterpret_cast<float4*>(dq) + row * G * (D / 4);
+  for (int ch = lane; ch < G * (D / 8); ch += 32) {
+    const int e8 = ch % (D / 8);
+    float acc[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+    for (int j = 0; j < keff; ++j) {
+      const float sj = scale_sel * ds[p0 + j];
+      const float4* kb = reinterpret_cast<const float4*>(kbar32 + ((b * Nc + idx[p0 + j]) * Hkv + g) * D) + e8 * 2;
+      const float4 k0 = kb[0], k1 = kb[1];
+      acc[0] = fmaf(sj, k0.x, acc[0]);
+      acc[1] = fmaf(sj, k0.y, acc[1]);
+      acc[2] = fmaf(sj, k0.z, acc[2]);
+      acc[3] = fmaf(sj, k0.w, acc[3]);
+      acc[4] = fmaf(sj, k1.x, acc[4]);
+      acc[5] = fmaf(sj, k1.y, acc[5]);
+      acc[6] = fmaf(sj, k1.z, acc[6]);
+      acc[7] = fmaf(sj, k1.w, acc[7]);
+    }
+    dst[2 * ch] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    dst[2 * ch + 1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
   }
 }
 
@@ -772,22 +826,30 @@ __global__ void zero_tail_kernel(float* __restrict__ dK, float* __restrict__ dV,
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// Workspace: bf16 dq partials [slots, G, d]; Δ [rows]; with stick-breaking
-// weights also dw, ds [slots] and q̂ [rows, d] (fp32).
+// Workspace of a backward call: bf16 dq partials [slots, G, d]; the full
+// backward with softmax weights Δ [rows]; whenever the chunk pass writes dw
+// (stick-breaking weights, attention-only backward) dw [slots]; the full
+// backward with stick-breaking weights also ds [slots] and q̂ [rows, d] fp32.
+enum class BwdMode { kFull, kAttention };
 struct BwdLayout {
   size_t dqpart, delta, dw, ds, qhat, total;
 };
-BwdLayout bwd_layout(const Dims& D) {
+BwdLayout bwd_layout(const Dims& D, BwdMode mode) {
   const size_t rows = (size_t)D.B * D.L * D.Hkv;
+  const bool full = mode == BwdMode::kFull;
   BwdLayout lo{};
   size_t o = 0;
   lo.dqpart = o;
   o = align256(o + (size_t)D.slots() * D.G * D.d * sizeof(uint16_t));
-  lo.delta = o;
-  o = align256(o + rows * sizeof(float));
-  if (D.stick) {
+  if (full && !D.stick) {
+    lo.delta = o;
+    o = align256(o + rows * sizeof(float));
+  }
+  if (!full || D.stick) {
     lo.dw = o;
     o = align256(o + (size_t)D.slots() * sizeof(float));
+  }
+  if (full && D.stick) {
     lo.ds = o;
     o = align256(o + (size_t)D.slots() * sizeof(float));
     lo.qhat = o;
@@ -798,26 +860,46 @@ BwdLayout bwd_layout(const Dims& D) {
 }
 
 template <int D>
-cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, const float* kbar32, const int32_t* idx,
-                const float* w, const void* O, const void* dO, const int32_t* offsets, const int32_t* entries,
-                float* dq, float* dK, float* dV, void* ws, cudaStream_t st) {
+cudaError_t launch_dkbar(const Dims& Dm, const void* q, const int32_t* offsets, const int32_t* entries, const float* ds,
+                         float* qhat, float* dK, cudaStream_t st) {
   const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
-  const BwdLayout lo = bwd_layout(Dm);
-  uint16_t* dqpart = (uint16_t*)((char*)ws + lo.dqpart);
-  float* delta = (float*)((char*)ws + lo.delta);
-  float* dwb = Dm.stick ? (float*)((char*)ws + lo.dw) : nullptr;
-  float* dsb = Dm.stick ? (float*)((char*)ws + lo.ds) : nullptr;
-  float* qhat = Dm.stick ? (float*)((char*)ws + lo.qhat) : nullptr;
   cudaError_t e;
-  if (!Dm.stick) {  // Δ_t = sum_j w_j dw_j = dO · O feeds the softmax weights' ds inside the chunk kernel
-    bwd_delta_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>((const uint16_t*)O, (const uint16_t*)dO, delta,
-                                                                    rows, Dm.G);
-  } else {
-    bwd_qhat_kernel<D><<<(unsigned)((rows * (D / 8) + 255) / 256), 256, 0, st>>>((const uint16_t*)q, qhat, rows,
-                                                                                  Dm.G);
-  }
+  bwd_qhat_kernel<D><<<(unsigned)((rows * (D / 8) + 255) / 256), 256, 0, st>>>((const uint16_t*)q, qhat, rows, Dm.G);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const long long keys = Dm.keys();
+  if (keys > 0) {
+    bwd_stick_dkbar_kernel<D><<<(unsigned)keys, D, 0, st>>>(offsets, entries, ds, qhat, dK, Dm.L, Dm.Hkv, Dm.topk,
+                                                            Dm.Nc, Dm.scale_sel);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+// kFull: dq, dK, dV including the selection chain (q and K are also the
+// selection's inputs). kAttention: dq, dK, dV of the attention alone, and the
+// slots' score gradients added into ds_acc.
+template <int D>
+cudaError_t run(const Dims& Dm, BwdMode mode, const void* q, const void* K, const void* V, const float* kbar32,
+                const int32_t* idx, const float* w, const void* O, const void* dO, const int32_t* offsets,
+                const int32_t* entries, float* dq, float* dK, float* dV, float* ds_acc, void* ws, cudaStream_t st) {
+  const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
+  const bool full = mode == BwdMode::kFull;
+  const bool dw_mode = !full || Dm.stick;
+  const BwdLayout lo = bwd_layout(Dm, mode);
+  uint16_t* dqpart = (uint16_t*)((char*)ws + lo.dqpart);
+  float* delta = full && !Dm.stick ? (float*)((char*)ws + lo.delta) : nullptr;
+  float* dwb = dw_mode ? (float*)((char*)ws + lo.dw) : nullptr;
+  float* dsb = full && Dm.stick ? (float*)((char*)ws + lo.ds) : ds_acc;
+  float* qhat = full && Dm.stick ? (float*)((char*)ws + lo.qhat) : nullptr;
+  cudaError_t e;
+  if (delta != nullptr) {  // Δ_t = sum_j w_j dw_j = dO · O feeds the softmax weights' ds inside the chunk kernel
+    bwd_delta_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>((const uint16_t*)O, (const uint16_t*)dO, delta,
+                                                                    rows, Dm.G);
+    note_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   const long long keys = Dm.keys();
   if (keys > 0) {
     BwdArgs a;
@@ -826,7 +908,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.V = (const uint16_t*)V;
     a.dO = (const uint16_t*)dO;
     a.w = w;
-    a.delta = delta;
+    a.delta = delta != nullptr ? delta : w;  // read by the loader; unused when dw_mode
     a.offsets = offsets;
     a.entries = entries;
     a.dqpart = dqpart;
@@ -843,7 +925,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.scale_attn = Dm.scale_attn;
     a.scale_sel = Dm.scale_sel;
     a.softmax1 = Dm.softmax1 ? 1 : 0;
-    a.stick = Dm.stick ? 1 : 0;
+    a.dw_mode = dw_mode ? 1 : 0;
     a.dw_out = dwb;
     const size_t smem = sizeof(BwdSmem<D>) + 1024;
     if ((e = cudaFuncSetAttribute(bwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
@@ -863,19 +945,17 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  if (Dm.stick) {
-    bwd_stick_ds_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(idx, w, dwb, dsb, rows, Dm.topk, Dm.Nc);
+  if (dw_mode) {
+    bwd_ds_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(idx, w, dwb, dsb, rows, Dm.topk, Dm.Nc,
+                                                                   Dm.stick ? 1 : 0, full ? 0 : 1);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    if (keys > 0) {
-      bwd_stick_dkbar_kernel<D><<<(unsigned)keys, D, 0, st>>>(offsets, entries, dsb, qhat, dK, Dm.L, Dm.Hkv, Dm.topk,
-                                                              Dm.Nc, Dm.scale_sel);
-      note_launches(1);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
+    if (full && (e = launch_dkbar<D>(Dm, q, offsets, entries, dsb, qhat, dK, st)) != cudaSuccess) return e;
   }
+  const bool sel_term = full && Dm.stick;
   bwd_dq_merge_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(idx, dqpart, dq, rows, Dm.G, Dm.topk, Dm.Nc,
-                                                                      dsb, kbar32, Dm.L, Dm.Hkv, Dm.scale_sel);
+                                                                      sel_term ? dsb : nullptr, kbar32, Dm.L, Dm.Hkv,
+                                                                      Dm.scale_sel);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int tail0 = Dm.Nc * kChunk;
@@ -889,6 +969,22 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
   return cudaSuccess;
 }
 
+// The selection chain for a given score gradient: dq_sel (every element), dK_sel
+// (zeroed, then the mean-pool share of dK̄ on every complete chunk's rows).
+template <int D>
+cudaError_t run_select_backward(const Dims& Dm, const void* q_sel, const float* kbar_sel, const int32_t* idx,
+                                const float* ds, const int32_t* offsets, const int32_t* entries, float* dq_sel,
+                                float* dK_sel, void* ws, cudaStream_t st) {
+  const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
+  cudaError_t e;
+  if ((e = cudaMemsetAsync(dK_sel, 0, (size_t)rows * D * sizeof(float), st)) != cudaSuccess) return e;
+  sel_dq_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(idx, ds, kbar_sel, dq_sel, rows, Dm.G, Dm.topk, Dm.Nc,
+                                                               Dm.L, Dm.Hkv, Dm.scale_sel);
+  note_launches(1);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  return launch_dkbar<D>(Dm, q_sel, offsets, entries, ds, (float*)ws, dK_sel, st);
+}
+
 }  // namespace
 
 unsigned backward_take_status() {
@@ -898,14 +994,35 @@ unsigned backward_take_status() {
   return v;
 }
 
-size_t backward_workspace(const Dims& D) { return bwd_layout(D).total; }
+size_t backward_workspace(const Dims& D) { return bwd_layout(D, BwdMode::kFull).total; }
+size_t backward_attention_workspace(const Dims& D) { return bwd_layout(D, BwdMode::kAttention).total; }
+size_t select_backward_workspace(const Dims& D) { return align256((size_t)D.B * D.L * D.Hkv * D.d * sizeof(float)); }
 
 cudaError_t launch_backward(const Dims& D, const void* q, const void* K, const void* V, const float* kbar32,
                             const int32_t* idx, const float* w, const void* O, const void* dO,
                             const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,
                             void* ws, cudaStream_t st) {
-  return D.d == 64 ? run<64>(D, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq, dK, dV, ws, st)
-                   : run<128>(D, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq, dK, dV, ws, st);
+  return D.d == 64 ? run<64>(D, BwdMode::kFull, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq, dK, dV, nullptr,
+                             ws, st)
+                   : run<128>(D, BwdMode::kFull, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq, dK, dV,
+                              nullptr, ws, st);
+}
+
+cudaError_t launch_backward_attention(const Dims& D, const void* q, const void* K, const void* V, const int32_t* idx,
+                                      const float* w, const void* dO, const int32_t* offsets,
+                                      const int32_t* entries, float* dq, float* dK, float* dV, float* ds_acc,
+                                      void* ws, cudaStream_t st) {
+  return D.d == 64 ? run<64>(D, BwdMode::kAttention, q, K, V, nullptr, idx, w, nullptr, dO, offsets, entries, dq, dK,
+                             dV, ds_acc, ws, st)
+                   : run<128>(D, BwdMode::kAttention, q, K, V, nullptr, idx, w, nullptr, dO, offsets, entries, dq,
+                              dK, dV, ds_acc, ws, st);
+}
+
+cudaError_t launch_select_backward(const Dims& D, const void* q_sel, const float* kbar_sel, const int32_t* idx,
+                                   const float* ds, const int32_t* offsets, const int32_t* entries, float* dq_sel,
+                                   float* dK_sel, void* ws, cudaStream_t st) {
+  return D.d == 64 ? run_select_backward<64>(D, q_sel, kbar_sel, idx, ds, offsets, entries, dq_sel, dK_sel, ws, st)
+                   : run_select_backward<128>(D, q_sel, kbar_sel, idx, ds, offsets, entries, dq_sel, dK_sel, ws, st);
 }
 
 }  // namespace hsa

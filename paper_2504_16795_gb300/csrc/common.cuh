@@ -235,6 +235,15 @@ cudaError_t launch_forward(const Dims& D, const void* q, const void* K, const vo
                            void* ws, cudaStream_t st);
 size_t backward_workspace(const Dims& D);
 unsigned backward_take_status();
+size_t backward_attention_workspace(const Dims& D);
+cudaError_t launch_backward_attention(const Dims& D, const void* q, const void* K, const void* V, const int32_t* idx,
+                                      const float* w, const void* dO, const int32_t* offsets,
+                                      const int32_t* entries, float* dq, float* dK, float* dV, float* ds_acc,
+                                      void* ws, cudaStream_t st);
+size_t select_backward_workspace(const Dims& D);
+cudaError_t launch_select_backward(const Dims& D, const void* q_sel, const float* kbar_sel, const int32_t* idx,
+                                   const float* ds, const int32_t* offsets, const int32_t* entries, float* dq_sel,
+                                   float* dK_sel, void* ws, cudaStream_t st);
 // Self-test of the bounded waits: one block waits on a barrier nothing arrives at.
 cudaError_t launch_selftest_wait(unsigned long long limit_ns, cudaStream_t st);
 unsigned selftest_take_status();

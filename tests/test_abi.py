@@ -97,7 +97,12 @@ def test_stick_breaking_backward_needs_its_extra_workspace(lib):
     base = hsa.workspace_size(hsa.HSA_OP_BACKWARD, shape())
     stick = hsa.workspace_size(hsa.HSA_OP_BACKWARD, shape(weights="stick"))
     s = shape()
-    assert stick == base + 2 * s.B * s.L * s.Hkv * s.topk * 4 + s.B * s.L * s.Hkv * s.d * 4
+    rows, slots = s.B * s.L * s.Hkv, s.B * s.L * s.Hkv * s.topk
+    # stick-breaking: no Δ; dw and ds per slot and the fp32 q̂ rows instead
+    assert stick == base - rows * 4 + 2 * slots * 4 + rows * s.d * 4
+    att = hsa.workspace_size(hsa.HSA_OP_BACKWARD_ATTENTION, s)
+    assert att == base - rows * 4 + slots * 4  # dq partials and dw
+    assert hsa.workspace_size(hsa.HSA_OP_SELECT_BACKWARD, s) == rows * s.d * 4
 
 
 def test_null_and_misaligned_pointers_are_rejected(lib):

@@ -295,6 +295,8 @@ def run_gpu(args, rank, world, local_rank):
     roof.update({"kernel": dom, "traffic": traffic,
                  "peak_source": f"{pk['source']} ({'bf16 sustained' if roof['bound'] == 'tensor' else 'hbm copy'})"})
 
+    variants = None if args.no_variants else run_variants(args, dev, pk, hsa, w, X, Y, barrier, model)
+
     # end to end through host buffers: H2D inputs, the path, D2H outputs, every step
     e2e = None
     if not args.no_e2e:
@@ -334,7 +336,62 @@ def run_gpu(args, rank, world, local_rank):
         decode = run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa)
 
     return dict(value=value, ms_step=ms_step, kernels=kernels, roofline=roof, e2e=e2e, clocks=clocks,
-                launches=launches, decode=decode, wall_ms_step=wall / K * 1e3)
+                launches=launches, decode=decode, wall_ms_step=wall / K * 1e3, variants=variants)
+
+
+def run_variants(args, dev, pk, hsa, w, X, Y, barrier, model):
+    """Forward and backward of the paper-default variants, and the split backward of layers sharing one
+    selection, on the same inputs and selection (outside the headline's timed region)."""
+    import torch
+
+    def timed(fn, n):
+        for _ in range(2):
+            fn()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(n):
+            fn()
+        e1.record()
+        barrier()
+        return e0.elapsed_time(e1) / n
+
+    def frac(call, ms):
+        return round(model[call]["flops"] / (ms / 1e3) / 1e12 / pk["bf16_sus"], 4)
+
+    n = max(args.steps, 5)
+    out = {}
+    for label, inner, weights in (("softmax-off-by-one", "softmax1", "softmax"), ("stick-breaking", "softmax", "stick")):
+        sh = hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk, inner=inner, weights=weights)
+        wsf = torch.empty(hsa.workspace_size(hsa.HSA_OP_FORWARD, sh), dtype=torch.uint8, device=dev)
+        wsb = torch.empty(hsa.workspace_size(hsa.HSA_OP_BACKWARD, sh), dtype=torch.uint8, device=dev)
+
+        def fwd():
+            hsa.forward(sh, X["q"], X["K"], X["V"], Y["idx"], Y["s_sel"], Y["offsets"], Y["entries"], Y["O"], Y["w"],
+                        ws=wsf)
+
+        def bwd():
+            hsa.backward(sh, X["q"], X["K"], X["V"], Y["kbar32"], Y["idx"], Y["w"], Y["O"], X["dO"], Y["offsets"],
+                         Y["entries"], Y["dq"], Y["dK"], Y["dV"], ws=wsb)
+
+        tf, tb = timed(fwd, n), timed(bwd, n)
+        out[label] = {"hsa_forward_ms": round(tf, 4), "hsa_backward_ms": round(tb, 4),
+                      "forward_frac": frac("hsa_forward", tf), "backward_frac": frac("hsa_backward", tb)}
+        del wsf, wsb
+    # layers sharing one selection: per layer the attention-only backward, then the selection chain once
+    sh = hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk)
+    wsa = torch.empty(hsa.workspace_size(hsa.HSA_OP_BACKWARD_ATTENTION, sh), dtype=torch.uint8, device=dev)
+    wss = torch.empty(hsa.workspace_size(hsa.HSA_OP_SELECT_BACKWARD, sh), dtype=torch.uint8, device=dev)
+    ds = torch.zeros(Y["idx"].shape, dtype=torch.float32, device=dev)
+    dq_sel, dK_sel = torch.empty_like(Y["dq"]), torch.empty_like(Y["dK"])
+    ta = timed(lambda: hsa.backward_attention(sh, X["q"], X["K"], X["V"], Y["idx"], Y["w"], X["dO"], Y["offsets"],
+                                              Y["entries"], ds, Y["dq"], Y["dK"], Y["dV"], ws=wsa), n)
+    ts = timed(lambda: hsa.select_backward(sh, X["q"], Y["kbar32"], Y["idx"], ds, Y["offsets"], Y["entries"], dq_sel,
+                                           dK_sel, ws=wss), n)
+    out["shared selection"] = {"hsa_backward_attention_ms": round(ta, 4), "hsa_select_backward_ms": round(ts, 4),
+                               "attention_frac": frac("hsa_backward", ta)}
+    del wsa, wss, ds, dq_sel, dK_sel
+    return out
 
 
 def run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa):
@@ -489,6 +546,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["hsa", "reference"], default="hsa")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-variants", action="store_true", help="skip the variant and shared-selection timings")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", type=int, default=3, help="prefill workload number (3 is the headline)")
@@ -532,7 +590,7 @@ def main():
                 "warmup": args.warmup, "ms_per_step": r["ms_step"], "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_obj(),
                 "roofline": r["roofline"], "cpu_baseline": cpu, "e2e": r["e2e"], "gpu_launches": r["launches"],
-                "clocks": r["clocks"], "kernels": r["kernels"], "decode": r["decode"],
+                "clocks": r["clocks"], "kernels": r["kernels"], "decode": r["decode"], "variants": r["variants"],
                 "wall_ms_per_step": r["wall_ms_step"]}
         print(json.dumps(line), flush=True)
     if world > 1:

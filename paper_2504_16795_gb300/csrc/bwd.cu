@@ -646,22 +646,28 @@ __global__ void __launch_bounds__(256) sel_dq_kernel(const int32_t* __restrict__
   if (row >= n_rows) return;
   const long long p0 = row * topk;
   bool valid = false;
-  if (lane < topk) {
-    const int c = idx[p0 + lane];
-    valid = c >= 0 && c < Nc;
+  int cl = 0;
+  float sl = 0.f;
+  if (lane < topk) {  // lane j holds slot j's chunk and scaled score gradient
+    cl = idx[p0 + lane];
+    valid = cl >= 0 && cl < Nc;
+    sl = valid ? scale_sel * ds[p0 + lane] : 0.f;
   }
   const int keff = __popc(__ballot_sync(0xFFFFFFFFu, valid));
   const long long b = row / ((long long)L * Hkv);
   const int g = (int)(row % Hkv);
   float4* dst = reinterpret_cast<float4*>(dq) + row * G * (D / 4);
-  for (int ch = lane; ch < G * (D / 8); ch += 32) {
+  for (int ch0 = 0; ch0 < G * (D / 8); ch0 += 32) {
+    const int ch = ch0 + lane;
     const int e8 = ch % (D / 8);
     float acc[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i] = 0.f;
     for (int j = 0; j < keff; ++j) {
-      const float sj = scale_sel * ds[p0 + j];
-      const float4* kb = reinterpret_cast<const float4*>(kbar32 + ((b * Nc + idx[p0 + j]) * Hkv + g) * D) + e8 * 2;
+      const float sj = __shfl_sync(0xFFFFFFFFu, sl, j);
+      const int cj = __shfl_sync(0xFFFFFFFFu, cl, j);
+      if (ch >= G * (D / 8)) continue;
+      const float4* kb = reinterpret_cast<const float4*>(kbar32 + ((b * Nc + cj) * Hkv + g) * D) + e8 * 2;
       const float4 k0 = kb[0], k1 = kb[1];
       acc[0] = fmaf(sj, k0.x, acc[0]);
       acc[1] = fmaf(sj, k0.y, acc[1]);
@@ -672,13 +678,14 @@ __global__ void __launch_bounds__(256) sel_dq_kernel(const int32_t* __restrict__
       acc[6] = fmaf(sj, k1.z, acc[6]);
       acc[7] = fmaf(sj, k1.w, acc[7]);
     }
+    if (ch >= G * (D / 8)) continue;
     dst[2 * ch] = make_float4(acc[0], acc[1], acc[2], acc[3]);
     dst[2 * ch + 1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
   }
 }
 
-// q̂ rows for the chunk-summary gradient: [b, t, g][e] = fp32 head-order sum of
-// the group's query rows (the selection's group query).
+// q̂ rows for the chunk-summary gradient: [b, t, g][e] = head-order fp32 sum
+// of the group's query rows (the selection's group query).
 template <int D>
 __global__ void __launch_bounds__(256) bwd_qhat_kernel(const uint16_t* __restrict__ q, float* __restrict__ qhat,
                                                        long long n_rows, int G) {
@@ -707,43 +714,57 @@ __global__ void __launch_bounds__(256) bwd_qhat_kernel(const uint16_t* __restric
   dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
 }
 
-// Stick-breaking: the chunk-summary gradient dK̄_i = c_sel sum over the slots
-// that chose chunk i (in token order, from the inverse index) of ds * q̂_t,
-// spread over the chunk's S key rows (mean pool): dK_{iS+s} += dK̄_i / S. Block
-// per (b, g, chunk), thread per dimension.
+// The chunk-summary gradient dK̄_i = c_sel sum over the slots that chose chunk
+// i (from the inverse index) of ds * q̂_t, spread over the chunk's S key rows
+// (mean pool): dK_{iS+s} += dK̄_i / S. Block per (b, g, chunk), in the chunk
+// kernels' order (long lists first): kDkbarGroups groups of D threads (thread =
+// dimension) take the entries n = group, group + kDkbarGroups, ... with eight
+// loads in flight each, and the group sums are added in group order
+// (deterministic).
+constexpr int kDkbarGroups = 4;
 template <int D>
-__global__ void __launch_bounds__(D) bwd_stick_dkbar_kernel(const int32_t* __restrict__ offsets,
-                                                            const int32_t* __restrict__ entries,
-                                                            const float* __restrict__ ds,
-                                                            const float* __restrict__ qhat, float* __restrict__ dK,
-                                                            int L, int Hkv, int topk, int Nc, float scale_sel) {
-  const int key = blockIdx.x;
-  const int c = key % Nc, bg = key / Nc;
+__global__ void __launch_bounds__(D * kDkbarGroups, 2) bwd_stick_dkbar_kernel(const int32_t* __restrict__ offsets,
+                                                                           const int32_t* __restrict__ entries,
+                                                                           const float* __restrict__ ds,
+                                                                           const float* __restrict__ qhat,
+                                                                           float* __restrict__ dK, int L, int Hkv,
+                                                                           int topk, int Nc, float scale_sel) {
+  __shared__ float part[kDkbarGroups][D];
+  int c, bg;
+  block_key(Nc, (int)(gridDim.x / (unsigned)Nc), c, bg);
+  const int key = bg * Nc + c;
   const int b = bg / Hkv, g = bg % Hkv;
   const int off = offsets[key], cnt = offsets[key + 1] - off;
   if (cnt <= 0) return;
-  const int e = threadIdx.x;
+  const int e = threadIdx.x % D, grp = threadIdx.x / D;
   const int slot_div = Hkv * topk;
+  constexpr int kStep = kDkbarGroups;
   float acc = 0.f;
-  int n = 0;
-  for (; n + 4 <= cnt; n += 4) {  // four slots' loads in flight
-    int p[4];
-    float dv[4], qv[4];
+  int n = grp;
+  for (; n + 7 * kStep < cnt; n += 8 * kStep) {  // eight slots' loads in flight
+    int p[8];
+    float dv[8], qv[8];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) p[u] = entries[off + n + u];
+    for (int u = 0; u < 8; ++u) p[u] = entries[off + n + u * kStep];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < 8; ++u) {
       dv[u] = ds[p[u]];
       qv[u] = qhat[((long long)(p[u] / slot_div) * Hkv + g) * D + e];
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) acc = fmaf(dv[u], qv[u], acc);
+    for (int u = 0; u < 8; ++u) acc = fmaf(dv[u], qv[u], acc);
   }
-  for (; n < cnt; ++n) {
+  for (; n < cnt; n += kStep) {
     const int p = entries[off + n];
     acc = fmaf(ds[p], qhat[((long long)(p / slot_div) * Hkv + g) * D + e], acc);
   }
-  const float add = scale_sel * acc / (float)kChunk;
+  part[grp][e] = acc;
+  __syncthreads();
+  if (grp != 0) return;
+  float sum = part[0][e];
+#pragma unroll
+  for (int k = 1; k < kDkbarGroups; ++k) sum += part[k][e];
+  const float add = scale_sel * sum / (float)kChunk;
   const long long row0 = ((long long)b * L + (long long)c * kChunk) * Hkv + g;
   for (int s = 0; s < kChunk; ++s) dK[(row0 + (long long)s * Hkv) * D + e] += add;
 }
@@ -763,19 +784,24 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
   if (row >= n_rows) return;
   const long long p0 = row * topk;
   bool valid = false;
-  if (lane < topk) {
-    const int c = idx[p0 + lane];
-    valid = c >= 0 && c < Nc;
+  int cl = 0;
+  float sl = 0.f;
+  if (lane < topk) {  // lane j holds slot j's chunk (and, for the selection term, scaled ds)
+    cl = idx[p0 + lane];
+    valid = cl >= 0 && cl < Nc;
+    if (ds != nullptr && valid) sl = scale_sel * ds[p0 + lane];
   }
   const int keff = __popc(__ballot_sync(0xFFFFFFFFu, valid));
   const int GD8 = G * (D / 8);
   const uint4* src = reinterpret_cast<const uint4*>(dqpart) + p0 * GD8;
   float4* dst = reinterpret_cast<float4*>(dq) + row * GD8 * 2;
-  for (int ch = lane; ch < GD8; ch += 32) {
+  for (int ch0 = 0; ch0 < GD8; ch0 += 32) {  // every lane runs every round (the slot broadcasts need the warp)
+    const int ch = ch0 + lane;
+    const bool active = ch < GD8;
     float acc[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-    for (int j = 0; j < keff; ++j) {
+    for (int j = 0; j < keff && active; ++j) {
       const uint4 v = src[(long long)j * GD8 + ch];
       acc[0] += bf16_lo(v.x);
       acc[1] += bf16_hi(v.x);
@@ -791,9 +817,10 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
       const long long b = row / ((long long)L * Hkv);
       const int g = (int)(row % Hkv);
       for (int j = 0; j < keff; ++j) {
-        const float sj = scale_sel * ds[p0 + j];
-        const float4* kb =
-            reinterpret_cast<const float4*>(kbar32 + ((b * Nc + idx[p0 + j]) * Hkv + g) * D) + e8 * 2;
+        const float sj = __shfl_sync(0xFFFFFFFFu, sl, j);
+        const int cj = __shfl_sync(0xFFFFFFFFu, cl, j);
+        if (!active) continue;
+        const float4* kb = reinterpret_cast<const float4*>(kbar32 + ((b * Nc + cj) * Hkv + g) * D) + e8 * 2;
         const float4 k0 = kb[0], k1 = kb[1];
         acc[0] = fmaf(sj, k0.x, acc[0]);
         acc[1] = fmaf(sj, k0.y, acc[1]);
@@ -805,6 +832,7 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
         acc[7] = fmaf(sj, k1.w, acc[7]);
       }
     }
+    if (!active) continue;
     dst[2 * ch] = make_float4(acc[0], acc[1], acc[2], acc[3]);
     dst[2 * ch + 1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
   }
@@ -869,8 +897,8 @@ cudaError_t launch_dkbar(const Dims& Dm, const void* q, const int32_t* offsets, 
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const long long keys = Dm.keys();
   if (keys > 0) {
-    bwd_stick_dkbar_kernel<D><<<(unsigned)keys, D, 0, st>>>(offsets, entries, ds, qhat, dK, Dm.L, Dm.Hkv, Dm.topk,
-                                                            Dm.Nc, Dm.scale_sel);
+    bwd_stick_dkbar_kernel<D><<<(unsigned)keys, D * kDkbarGroups, 0, st>>>(offsets, entries, ds, qhat, dK, Dm.L,
+                                                                           Dm.Hkv, Dm.topk, Dm.Nc, Dm.scale_sel);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

@@ -439,6 +439,11 @@ def run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa):
     needles = synth.needle_chunk_ids(w)
     got = idx.cpu().numpy()
     found = int(sum(int(needles[b]) in got[b, 0] for b in range(w.Bq)))
+    host = None
+    if not args.no_host_memory:
+        ref = [t.clone() for t in (O, idx, s_sel, wts)]
+        call = (lambda Kx, Vx: hsa.decode_indexed(dshape, q, Kx, Vx, kb, index, O, idx, s_sel, wts, ws))
+        host = run_decode_host_memory(args, w, Kmem, Vmem, call, ref, ms, barrier, max_over_ranks)
     scan_bytes = Nc * w.Hkv * w.d * 2  # one pass over the bf16 chunk summaries
     gather_bytes = w.Bq * w.Hkv * w.topk * 2 * w.S * w.d * 2
     nbytes = scan_bytes + gather_bytes + 2 * w.Bq * w.Hq * w.d * 2
@@ -449,10 +454,72 @@ def run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa):
     return {"value": world * w.Bq / (ms / 1e3), "unit": "queries/s", "ms_per_call": ms,
             "memory_tokens": T, "chunks": Nc, "queries": w.Bq, "Hq": w.Hq, "Hkv": w.Hkv, "d": w.d, "topk": w.topk,
             "needles_found": f"{found}/{w.Bq}", "pool_ms_once": pool_ms, "index_ms_once": index_ms,
+            "host_memory": host,
             "path": "hsa_decode_indexed (tensor-core scan of the bf16 summaries, exact fp32 rescoring)",
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm"], "unit": "GB/s",
                          "frac": round(achieved / pk["hbm"], 4), "algorithmic_bytes": nbytes,
                          "scan": "bf16 chunk summaries", "flops": flops}}
+
+
+def mem_available_bytes():
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
+
+
+def run_decode_host_memory(args, w, Kmem, Vmem, call, ref, hbm_ms, barrier, max_over_ranks):
+    """The same decode with the token memory K, V in page-locked host memory, read by the
+    kernels over the CPU-GPU link (only the k selected chunks per query cross it); the
+    summaries and the index stay in HBM. Outputs must equal the HBM-resident run's."""
+    import torch
+
+    need = 2 * Kmem.numel() * Kmem.element_size()
+    avail = mem_available_bytes()
+    if avail < 2 * need:
+        return {"skipped": f"host memory available {avail / 2**30:.0f} GiB < twice the {need / 2**30:.0f} GiB memory"}
+    cudart = torch.cuda.cudart()
+    t0 = time.perf_counter()
+    Kh = torch.empty(Kmem.shape, dtype=Kmem.dtype)
+    Vh = torch.empty(Vmem.shape, dtype=Vmem.dtype)
+    registered = []
+    try:
+        for t in (Kh, Vh):
+            rc = int(cudart.cudaHostRegister(t.data_ptr(), t.numel() * t.element_size(), 2))  # mapped
+            if rc != 0:
+                return {"skipped": f"cudaHostRegister failed ({rc})"}
+            registered.append(t)
+        Kh.copy_(Kmem)
+        Vh.copy_(Vmem)
+        torch.cuda.synchronize()
+        setup_s = time.perf_counter() - t0
+        for _ in range(args.warmup):
+            call(Kh, Vh)
+        barrier()
+        steps = max(args.steps, 10)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(steps):
+            call(Kh, Vh)
+        e1.record()
+        barrier()
+        ms = max_over_ranks(e0.elapsed_time(e1)) / steps
+        out = call(Kh, Vh)
+        torch.cuda.synchronize()
+        identical = all(torch.equal(a, b) for a, b in zip(out, ref))
+    finally:
+        for t in registered:
+            cudart.cudaHostUnregister(t.data_ptr())
+    link_bytes = w.Bq * w.Hkv * w.topk * 2 * w.S * w.d * 2  # the selected chunks' K and V rows
+    return {"ms_per_call": ms, "queries_per_s": w.Bq / (ms / 1e3), "vs_hbm_resident": round(hbm_ms / ms, 3),
+            "identical_to_hbm_resident": identical, "memory_bytes_in_host": need,
+            "link_bytes_per_call": link_bytes, "link_gbs": round(link_bytes / (ms / 1e3) / 1e9, 1),
+            "setup_s": round(setup_s, 1),
+            "layout": "K, V in cudaHostRegister-mapped host memory; summaries, index, q, O in HBM"}
 
 
 # ----------------------------------------------------------------------------- CPU oracle (baseline / reference arm)
@@ -546,6 +613,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["hsa", "reference"], default="hsa")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-host-memory", action="store_true",
+                    help="skip the decode over a memory kept in host memory")
     ap.add_argument("--no-variants", action="store_true", help="skip the variant and shared-selection timings")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -257,10 +257,17 @@ hsa_status_t hsa_select_backward(const hsa_shape_t* shape, const void* q_sel, co
  * Decode against a resident memory (§3.2 "Inference": only the chunk
  * summaries are scanned on every step, then the k selected chunks are
  * fetched). One query token per batch row; all n_chunks chunks are visible.
- *   q      [Bq, Hq, d] bf16.
- *   K_mem, V_mem [n_chunks*S, Hkv, d] bf16 (the memory).
- *   kbar32 [n_chunks, Hkv, d] fp32 (hsa_chunk_pool of K_mem with B = 1).
- *   O [Bq, Hq, d] bf16, idx, s_sel, w [Bq, Hkv, topk], outputs.
+ *   K_mem, V_mem [n_chunks*S, Hkv, d] bf16 (the memory). Device memory, or
+ *          page-locked host memory that the device reads at the same address
+ *          (cudaHostAlloc, cudaMallocHost, or cudaHostRegister with
+ *          cudaHostRegisterMapped): a memory larger than HBM then stays in
+ *          host memory and only the k selected chunks per query cross the
+ *          CPU-GPU link, with results identical to a device-resident memory.
+ *          Pageable or unknown memory returns HSA_ERR_INVALID_ARG before any
+ *          launch (checked with cudaPointerGetAttributes on every call).
+ *   kbar32 [n_chunks, Hkv, d] fp32 (hsa_chunk_pool of K_mem with B = 1),
+ *          device memory.
+ *   q, O [Bq, Hq, d] bf16, idx, s_sel, w [Bq, Hkv, topk]: device memory.
  * Needs workspace hsa_decode_workspace_size.
  */
 hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const void* K_mem, const void* V_mem,

@@ -313,6 +313,8 @@ hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const vo
   }
   const size_t need = hsa::decode_workspace(D);
   if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+  if (D.Nc > 0 && !(hsa::memory_device_readable(K_mem) && hsa::memory_device_readable(V_mem)))
+    return HSA_ERR_INVALID_ARG;
   return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, ws, stream));
 }
 
@@ -360,11 +362,14 @@ hsa_status_t hsa_decode_indexed(const hsa_decode_shape_t* shape, const void* q, 
   if (!hsa::decode_tc_applies(D)) {  // k > 16 or an empty memory: the CUDA-core scan of hsa_decode
     const size_t need = hsa::decode_workspace(D);
     if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+    if (D.Nc > 0 && !(hsa::memory_device_readable(K_mem) && hsa::memory_device_readable(V_mem)))
+      return HSA_ERR_INVALID_ARG;
     return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, ws, stream));
   }
   HSA_REQUIRE_PTR(index);
   const size_t need = hsa::decode_tc_workspace(D);
   if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+  if (!(hsa::memory_device_readable(K_mem) && hsa::memory_device_readable(V_mem))) return HSA_ERR_INVALID_ARG;
   return cuda_status(hsa::launch_decode_tc(D, q, K_mem, V_mem, kbar32, index, O, idx, s_sel, w, ws, stream));
 }
 

@@ -258,6 +258,10 @@ struct DecodeDims {
   bool softmax1, stick;  // variants as in Dims
 };
 size_t decode_workspace(const DecodeDims& D);
+// True when a kernel of the current device may read p at that address: device or
+// managed memory, or page-locked host memory mapped at the same address (a decode
+// memory kept in host memory). Pageable or unknown memory gives false.
+bool memory_device_readable(const void* p);
 cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
                           void* O, int32_t* idx, float* s_sel, float* w, void* ws, cudaStream_t st);
 // Token-level attention over the selected chunks and the weighted sum (the last two decode steps).

@@ -166,11 +166,31 @@ __global__ void __launch_bounds__(kThreads) dec_attend_kernel(const uint16_t* __
     for (int u = tid; u < G * D; u += kThreads) out[u] = 0.f;
     return;
   }
-  for (int u = tid; u < kChunk * D; u += kThreads) {
-    const int s = u / D, e = u % D;
-    const long long r = (((long long)c * kChunk + s) * Hkv + g) * D + e;
-    Ks[s][e] = bf16_bits_to_f32(Kmem[r]);
-    Vs[s][e] = bf16_bits_to_f32(Vmem[r]);
+  // the chunk's rows in 16-byte pieces, every piece of a thread requested before
+  // the first is used (the memory may also sit in host memory, read over the
+  // CPU-GPU link, where a round trip costs microseconds)
+  constexpr int kPieces = kChunk * (D / 8) / kThreads;
+  static_assert(kPieces * kThreads == kChunk * (D / 8), "whole pieces per thread");
+  uint4 kv[kPieces], vv[kPieces];
+#pragma unroll
+  for (int i = 0; i < kPieces; ++i) {
+    const int u = tid + i * kThreads;
+    const long long r = (((long long)c * kChunk + u / (D / 8)) * Hkv + g) * D + (u % (D / 8)) * 8;
+    kv[i] = *reinterpret_cast<const uint4*>(Kmem + r);
+    vv[i] = *reinterpret_cast<const uint4*>(Vmem + r);
+  }
+#pragma unroll
+  for (int i = 0; i < kPieces; ++i) {
+    const int u = tid + i * kThreads;
+    const int s = u / (D / 8), e = (u % (D / 8)) * 8;
+    const uint32_t kw[4] = {kv[i].x, kv[i].y, kv[i].z, kv[i].w}, vw[4] = {vv[i].x, vv[i].y, vv[i].z, vv[i].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      Ks[s][e + 2 * j] = bf16_lo(kw[j]);
+      Ks[s][e + 2 * j + 1] = bf16_hi(kw[j]);
+      Vs[s][e + 2 * j] = bf16_lo(vw[j]);
+      Vs[s][e + 2 * j + 1] = bf16_hi(vw[j]);
+    }
   }
   for (int u = tid; u < G * D; u += kThreads) {
     const int hh = u / D, e = u % D;
@@ -308,6 +328,16 @@ cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void*
   }
   note_launches(1);
   return cudaGetLastError();
+}
+
+bool memory_device_readable(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return true;
+  return a.type == cudaMemoryTypeHost && a.devicePointer == p;
 }
 
 cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,

@@ -63,6 +63,8 @@ hsa_status_t hsa_decode_noalloc(const hsa_decode_shape_t* shape, const void* q, 
       if (p == nullptr || !aligned16(p)) return HSA_ERR_INVALID_ARG;
   }
   if (hsa::decode_workspace(D) > (size_t)HSA_DECODE_NOALLOC_SCRATCH_BYTES) return HSA_ERR_WORKSPACE;
+  if (D.Nc > 0 && !(hsa::memory_device_readable(K_mem) && hsa::memory_device_readable(V_mem)))
+    return HSA_ERR_INVALID_ARG;
   void* scratch = nullptr;
   if ((st = device_scratch(&scratch)) != HSA_OK) return st;
   return hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, scratch, stream) == cudaSuccess

@@ -334,6 +334,7 @@ def run_gpu(args, rank, world, local_rank):
     decode = None
     if not args.no_decode:
         decode = run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa)
+        decode["append"] = run_memory_append(args, dev, pk, barrier, max_over_ranks, hsa)
 
     return dict(value=value, ms_step=ms_step, kernels=kernels, roofline=roof, e2e=e2e, clocks=clocks,
                 launches=launches, decode=decode, wall_ms_step=wall / K * 1e3, variants=variants)
@@ -459,6 +460,69 @@ def run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa):
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm"], "unit": "GB/s",
                          "frac": round(achieved / pk["hbm"], 4), "algorithmic_bytes": nbytes,
                          "scan": "bf16 chunk summaries", "flops": flops}}
+
+
+def run_memory_append(args, dev, pk, barrier, max_over_ranks, hsa):
+    """Growing a decode memory: a 2^20-token prefill appended at once (rows stored, 2^14 chunks pooled and
+    indexed in one pass over the new rows), then tokens appended one by one as a decoder emits them."""
+    import torch
+
+    w = DECODE
+    T, Hkv, d = 1 << 20, w.Hkv, w.d
+    cap = T // w.S + 1
+    wk = w.with_(L=T)
+    Kn = synth.device_tensor(wk, "K", dev)
+    Vn = synth.device_tensor(wk, "V", dev)
+    Km = torch.empty((cap * w.S, Hkv, d), dtype=torch.bfloat16, device=dev)
+    Vm = torch.empty_like(Km)
+    kb = torch.zeros((cap, Hkv, d), dtype=torch.float32, device=dev)
+    shape = hsa.DecodeShape(Bq=1, Hq=w.Hq, Hkv=Hkv, d=d, n_chunks=0, topk=w.topk, capacity_chunks=cap)
+    index = hsa.decode_index(shape, kb)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn, n):
+        for _ in range(args.warmup):
+            fn()
+        barrier()
+        e0.record()
+        for _ in range(n):
+            fn()
+        e1.record()
+        barrier()
+        return max_over_ranks(e0.elapsed_time(e1)) / n
+
+    # the same rows rewritten each time: the result is the same memory
+    bulk_ms = timed(lambda: hsa.memory_append(shape, 0, Kn, Vn, Km, Vm, kb, index), max(args.steps, 10))
+    one_k, one_v = Kn[:w.S], Vn[:w.S]
+
+    def stream():  # the S tokens of the next chunk, one call per token
+        for t in range(w.S):
+            hsa.memory_append(shape, T + t, one_k[t:t + 1], one_v[t:t + 1], Km, Vm, kb, index)
+
+    token_ms = timed(stream, 5) / w.S  # eager: one host call per token (argument checks included)
+    # a serving loop replays its per-token launches from a CUDA graph
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, capture_error_mode="relaxed"):
+        stream()
+    token_graph_ms = timed(graph.replay, 5) / w.S
+    torch.cuda.synchronize()
+    kb_once = torch.empty((1, T // w.S, Hkv, d), dtype=torch.float32, device=dev)
+    hsa.chunk_pool(hsa.Shape(B=1, L=T, Hq=w.Hq, Hkv=Hkv, d=d, topk=w.topk), Kn.view(1, T, Hkv, d), kb_once, None,
+                   want_bf16=False)
+    identical = bool(torch.equal(kb[:T // w.S], kb_once[0])) and bool(torch.equal(Km[:T], Kn))
+    tok_bytes = Hkv * d * 2
+    nbytes = 4 * T * tok_bytes + (T // w.S) * Hkv * d * (4 + 4 + 2) + (T // w.S) * Hkv * 4
+    achieved = nbytes / (bulk_ms / 1e3) / 1e9
+    del Kn, Vn, Km, Vm, kb, index, kb_once, graph
+    torch.cuda.empty_cache()
+    return {"prefill_tokens": T, "prefill_append_ms": round(bulk_ms, 4),
+            "prefill_tokens_per_s": T / (bulk_ms / 1e3), "token_append_us": round(token_ms * 1e3, 2),
+            "token_append_us_graph": round(token_graph_ms * 1e3, 2),
+            "summaries_identical_to_chunk_pool": identical,
+            "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm"], "unit": "GB/s",
+                         "frac": round(achieved / pk["hbm"], 4), "algorithmic_bytes": nbytes,
+                         "counted": "read K_new, V_new; write K_mem, V_mem, K̄ fp32; index: read K̄, write bf16 "
+                                    "rows and norms"}}
 
 
 def mem_available_bytes():

@@ -86,6 +86,9 @@ typedef struct {
     float scale_sel;    /* <= 0 selects 1/sqrt((Hq/Hkv) * d) */
     float scale_attn;   /* <= 0 selects 1/sqrt(d) */
     int flags;          /* HSA_FLAG_*; 0: defaults */
+    long long capacity_chunks; /* chunks the memory and its decode index are laid
+                                  out for (a growing memory, see hsa_memory_append);
+                                  0 selects n_chunks; otherwise >= n_chunks */
 } hsa_decode_shape_t;
 
 typedef enum {
@@ -278,11 +281,15 @@ hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const vo
  * Decode index of a resident memory, built once per memory and reused by
  * every hsa_decode_indexed call (§3.2 "Inference": the chunk summaries are
  * what each decoding step scans). It holds the summaries rounded to bf16 in
- * [Hkv][n_chunks][d] order, |K̄_i| per chunk and its maximum over every 64
- * chunks. Size from hsa_decode_index_size (0 when topk > 16 or n_chunks = 0:
- * hsa_decode_indexed then needs no index). Only shape's Hkv, d, n_chunks and
- * topk matter; Bq may be 0.
- *   kbar32 [n_chunks, Hkv, d] fp32 (hsa_chunk_pool of the memory, B = 1).
+ * [Hkv][C][d] order, |K̄_i| per chunk and its maximum over every 64 chunks,
+ * laid out for C = capacity_chunks (n_chunks when 0) chunks; the n_chunks
+ * present are written and every other byte is zeroed, so that
+ * hsa_memory_append can enter chunks as they complete. Size from
+ * hsa_decode_index_size (0 when topk > 16 or C = 0: hsa_decode_indexed then
+ * needs no index). Only shape's Hkv, d, n_chunks, capacity_chunks and topk
+ * matter; Bq may be 0.
+ *   kbar32 [n_chunks, Hkv, d] fp32 (hsa_chunk_pool of the memory, B = 1);
+ *          may be NULL when n_chunks = 0.
  *   index  device memory, caller-owned, 16-byte aligned.
  */
 size_t hsa_decode_index_size(const hsa_decode_shape_t* shape);
@@ -332,6 +339,41 @@ hsa_status_t hsa_decode_indexed(const hsa_decode_shape_t* shape, const void* q, 
 hsa_status_t hsa_decode_noalloc(const hsa_decode_shape_t* shape, const void* q, const void* K_mem,
                                 const void* V_mem, const float* kbar32, void* O, int32_t* idx, float* s_sel,
                                 float* w, cudaStream_t stream);
+
+/*
+ * Append tokens to a growing decode memory (§3.2 "Inference": the memory grows
+ * as tokens are decoded, a chunk is summarised once its S tokens are present,
+ * and only completed chunks are selectable). One launch stores the new rows of
+ * K and V and pools every chunk they complete (the fp32 token-order sum and
+ * division of hsa_chunk_pool: summaries bit-identical to pooling the final
+ * memory at once); a second enters those chunks in the decode index (rows
+ * bit-identical to hsa_decode_index of the final memory with the same
+ * capacity).
+ *   shape    Hkv, d, S, topk, flags and capacity C = capacity_chunks (or
+ *            n_chunks when 0); Bq and Hq are unused but must be valid.
+ *   n_tokens tokens already in the memory (rows 0 .. n_tokens-1 written);
+ *            n_new tokens are appended: n_tokens + n_new <= C * S, else
+ *            HSA_ERR_INVALID_ARG.
+ *   K_new, V_new [n_new, Hkv, d] bf16. K_new may be the memory's own rows
+ *            from n_tokens on (a prefill that wrote them in place); otherwise
+ *            no argument may overlap another.
+ *   K_mem, V_mem [C*S, Hkv, d] bf16: device memory, or mapped page-locked host
+ *            memory as in hsa_decode (checked the same way, as are K_new, V_new).
+ *   kbar32   [C, Hkv, d] fp32, device memory: the summaries of the chunks that
+ *            the append completes are written; the rest is untouched.
+ *   index    the decode index (hsa_decode_index_size of shape, index_bytes at
+ *            least that, else HSA_ERR_WORKSPACE) built by hsa_decode_index with
+ *            the same capacity, before the first append (any n_chunks <= C,
+ *            including 0) and kept by every append since; or NULL when the
+ *            memory is only decoded with hsa_decode. A non-null index with
+ *            topk > 16 returns HSA_ERR_UNSUPPORTED.
+ * After the call, decode with n_chunks = floor((n_tokens + n_new) / S) and the
+ * same capacity_chunks. The trailing incomplete chunk's rows are stored but
+ * not selectable until an append completes it. Enqueued on `stream`.
+ */
+hsa_status_t hsa_memory_append(const hsa_decode_shape_t* shape, long long n_tokens, long long n_new,
+                               const void* K_new, const void* V_new, void* K_mem, void* V_mem, float* kbar32,
+                               void* index, size_t index_bytes, cudaStream_t stream);
 
 #ifdef __cplusplus
 }

@@ -25,6 +25,7 @@ from .binding import (  # noqa: F401
     decode_index,
     decode_indexed,
     decode_noalloc,
+    memory_append,
     decode_workspace_size,
     device_check,
     selftest_wait_timeout,

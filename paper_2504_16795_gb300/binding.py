@@ -35,7 +35,8 @@ class _Shape(ctypes.Structure):
 class _DecodeShape(ctypes.Structure):
     _fields_ = [("Bq", ctypes.c_int), ("Hq", ctypes.c_int), ("Hkv", ctypes.c_int), ("d", ctypes.c_int),
                 ("S", ctypes.c_int), ("topk", ctypes.c_int), ("n_chunks", ctypes.c_longlong),
-                ("scale_sel", ctypes.c_float), ("scale_attn", ctypes.c_float), ("flags", ctypes.c_int)]
+                ("scale_sel", ctypes.c_float), ("scale_attn", ctypes.c_float), ("flags", ctypes.c_int),
+                ("capacity_chunks", ctypes.c_longlong)]
 
 
 def _flags(inner: str, weights: str) -> int:
@@ -89,10 +90,11 @@ class DecodeShape:
     scale_attn: float = 0.0
     inner: str = "softmax"
     weights: str = "softmax"
+    capacity_chunks: int = 0  # a growing memory's capacity (0: n_chunks)
 
     def c(self) -> _DecodeShape:
         return _DecodeShape(self.Bq, self.Hq, self.Hkv, self.d, self.S, self.topk, self.n_chunks, self.scale_sel,
-                            self.scale_attn, _flags(self.inner, self.weights))
+                            self.scale_attn, _flags(self.inner, self.weights), self.capacity_chunks)
 
 
 _lib = None
@@ -141,8 +143,9 @@ def load():
     L.hsa_decode_indexed_workspace_size.restype = sz
     L.hsa_decode_indexed_workspace_size.argtypes = [dp]
     L.hsa_decode_indexed.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    L.hsa_memory_append.argtypes = [dp, ctypes.c_longlong, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, sz, vp]
     for f in (L.hsa_chunk_pool, L.hsa_select_topk, L.hsa_build_index, L.hsa_forward, L.hsa_backward,
-              L.hsa_decode, L.hsa_decode_noalloc, L.hsa_decode_index, L.hsa_decode_indexed):
+              L.hsa_decode, L.hsa_decode_noalloc, L.hsa_decode_index, L.hsa_decode_indexed, L.hsa_memory_append):
         f.restype = i
     _lib = L
     return L
@@ -379,6 +382,23 @@ def decode_indexed(shape: DecodeShape, q, K_mem, V_mem, kbar32, index, O=None, i
                                      _ptr(O), _ptr(idx), _ptr(s_sel), _ptr(w), _ptr(wsp), nb, _stream(dev)),
            "hsa_decode_indexed")
     return O, idx, s_sel, w
+
+
+def memory_append(shape: DecodeShape, n_tokens: int, K_new, V_new, K_mem, V_mem, kbar32, index=None) -> int:
+    """hsa_memory_append: append K_new, V_new [n_new, Hkv, d] to a memory holding n_tokens tokens (rows
+    stored, completed chunks pooled into kbar32 and entered in index); returns the new token count.
+
+    K_new, V_new, K_mem, V_mem may be CUDA tensors or pinned host tensors; kbar32 and index live on the device."""
+    n_new = int(K_new.shape[0])
+    for t, name in ((K_new, "K_new"), (V_new, "V_new")):
+        if t.dtype != torch.bfloat16 or tuple(t.shape) != (n_new, shape.Hkv, shape.d) or not t.is_contiguous():
+            raise ValueError(f"{name}: expected a contiguous bf16 tensor of shape {(n_new, shape.Hkv, shape.d)}")
+    nb = index.numel() * index.element_size() if index is not None else 0
+    s = shape.c()
+    _check(load().hsa_memory_append(ctypes.byref(s), int(n_tokens), n_new, _ptr(K_new), _ptr(V_new), _ptr(K_mem),
+                                    _ptr(V_mem), _ptr(kbar32), _ptr(index), nb, _stream(kbar32.device)),
+           "hsa_memory_append")
+    return int(n_tokens) + n_new
 
 
 class Workspaces:

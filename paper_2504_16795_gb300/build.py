@@ -19,7 +19,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libhsa.so")
 
 SOURCES = ["api.cu", "pool.cu", "select.cu", "select_tc.cu", "index.cu", "fwd.cu", "bwd.cu", "decode.cu", "decode_noalloc.cu",
-           "selftest.cu"]
+           "selftest.cu", "memory.cu"]
 HEADERS = ["common.cuh", "score_tile.cuh", "tc.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

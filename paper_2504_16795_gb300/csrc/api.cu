@@ -268,6 +268,9 @@ hsa_status_t resolve_decode(const hsa_decode_shape_t* s, hsa::DecodeDims* out) {
   if (s->S != hsa::kChunk) return HSA_ERR_UNSUPPORTED;
   if (s->topk > 32) return HSA_ERR_UNSUPPORTED;
   if (s->n_chunks >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
+  if (s->capacity_chunks < 0 || (s->capacity_chunks > 0 && s->capacity_chunks < s->n_chunks))
+    return HSA_ERR_INVALID_ARG;
+  if (s->capacity_chunks >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
   if (s->flags & ~(HSA_FLAG_SOFTMAX1 | HSA_FLAG_STICK_BREAKING)) return HSA_ERR_UNSUPPORTED;
   if ((long long)s->Bq * s->Hkv * s->topk >= (1LL << 31)) return HSA_ERR_UNSUPPORTED;
   hsa::DecodeDims D;
@@ -279,6 +282,7 @@ hsa_status_t resolve_decode(const hsa_decode_shape_t* s, hsa::DecodeDims* out) {
   D.topk = s->topk;
   D.G = G;
   D.Nc = s->n_chunks;
+  D.cap = s->capacity_chunks > 0 ? s->capacity_chunks : s->n_chunks;
   D.scale_sel = s->scale_sel > 0.f ? s->scale_sel : (float)(1.0 / std::sqrt((double)G * s->d));
   D.scale_attn = s->scale_attn > 0.f ? s->scale_attn : (float)(1.0 / std::sqrt((double)s->d));
   D.softmax1 = (s->flags & HSA_FLAG_SOFTMAX1) != 0;
@@ -320,7 +324,7 @@ hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const vo
 
 size_t hsa_decode_index_size(const hsa_decode_shape_t* shape) {
   hsa::DecodeDims D;
-  if (resolve_decode(shape, &D) != HSA_OK || !hsa::decode_tc_applies(D)) return 0;
+  if (resolve_decode(shape, &D) != HSA_OK) return 0;
   return hsa::decode_index_bytes(D);
 }
 
@@ -329,8 +333,8 @@ hsa_status_t hsa_decode_index(const hsa_decode_shape_t* shape, const float* kbar
   hsa::DecodeDims D;
   hsa_status_t st = resolve_decode(shape, &D);
   if (st != HSA_OK) return st;
-  if (!hsa::decode_tc_applies(D)) return D.Nc == 0 ? HSA_OK : HSA_ERR_UNSUPPORTED;
-  HSA_REQUIRE_PTR(kbar32);
+  if (!hsa::decode_index_applies(D)) return D.cap == 0 ? HSA_OK : HSA_ERR_UNSUPPORTED;
+  if (D.Nc > 0) HSA_REQUIRE_PTR(kbar32);
   const size_t need = hsa::decode_index_bytes(D);
   if (index_bytes < need || index == nullptr || !aligned16(index)) return HSA_ERR_WORKSPACE;
   return cuda_status(hsa::launch_decode_index(D, kbar32, index, stream));
@@ -371,6 +375,30 @@ hsa_status_t hsa_decode_indexed(const hsa_decode_shape_t* shape, const void* q, 
   if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
   if (!(hsa::memory_device_readable(K_mem) && hsa::memory_device_readable(V_mem))) return HSA_ERR_INVALID_ARG;
   return cuda_status(hsa::launch_decode_tc(D, q, K_mem, V_mem, kbar32, index, O, idx, s_sel, w, ws, stream));
+}
+
+hsa_status_t hsa_memory_append(const hsa_decode_shape_t* shape, long long n_tokens, long long n_new,
+                               const void* K_new, const void* V_new, void* K_mem, void* V_mem, float* kbar32,
+                               void* index, size_t index_bytes, cudaStream_t stream) {
+  hsa::DecodeDims D;
+  hsa_status_t st = resolve_decode(shape, &D);
+  if (st != HSA_OK) return st;
+  if (n_tokens < 0 || n_new < 0 || n_tokens > D.cap * D.S - n_new) return HSA_ERR_INVALID_ARG;
+  if (n_new == 0) return HSA_OK;
+  HSA_REQUIRE_PTR(K_new);
+  HSA_REQUIRE_PTR(V_new);
+  HSA_REQUIRE_PTR(K_mem);
+  HSA_REQUIRE_PTR(V_mem);
+  HSA_REQUIRE_PTR(kbar32);
+  if (index != nullptr) {
+    if (!hsa::decode_index_applies(D)) return HSA_ERR_UNSUPPORTED;
+    if (index_bytes < hsa::decode_index_bytes(D) || !aligned16(index)) return HSA_ERR_WORKSPACE;
+  }
+  const void* rows[] = {K_new, V_new, K_mem, V_mem};
+  for (const void* p : rows)
+    if (!hsa::memory_device_readable(p)) return HSA_ERR_INVALID_ARG;
+  return cuda_status(
+      hsa::launch_memory_append(D, n_tokens, n_new, K_new, V_new, K_mem, V_mem, kbar32, index, stream));
 }
 
 }  // extern "C"

@@ -256,6 +256,7 @@ struct DecodeDims {
   long long Nc;
   float scale_sel, scale_attn;
   bool softmax1, stick;  // variants as in Dims
+  long long cap;         // chunks the memory and its index are laid out for (>= Nc)
 };
 size_t decode_workspace(const DecodeDims& D);
 // True when a kernel of the current device may read p at that address: device or
@@ -268,9 +269,19 @@ cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, con
 cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void* K, const void* V,
                                  const int32_t* idx, const float* w, void* O, float* opart, cudaStream_t st);
 // Decode over a memory index (bf16 summaries, norms): tensor-core scan with exact rescoring (topk <= 16).
-bool decode_tc_applies(const DecodeDims& D);
+bool decode_index_applies(const DecodeDims& D);  // topk <= 16: the memory has an index
+bool decode_tc_applies(const DecodeDims& D);     // ... and at least one chunk
 size_t decode_index_bytes(const DecodeDims& D);
 cudaError_t launch_decode_index(const DecodeDims& D, const float* kbar32, void* index, cudaStream_t st);
+// Index rows of chunks [c0, c1) from kbar32 (the memory's [cap, Hkv, d] summaries).
+cudaError_t launch_index_rows(const DecodeDims& D, const float* kbar32, void* index, long long c0, long long c1,
+                              cudaStream_t st);
+// Append n_new tokens (K_new, V_new [n_new, Hkv, d]) to a memory holding n_tokens:
+// rows written, newly completed chunks pooled into kbar32 and, when index is not
+// null, entered in the decode index.
+cudaError_t launch_memory_append(const DecodeDims& D, long long n_tokens, long long n_new, const void* K_new,
+                                 const void* V_new, void* K_mem, void* V_mem, float* kbar32, void* index,
+                                 cudaStream_t st);
 size_t decode_tc_workspace(const DecodeDims& D);
 cudaError_t launch_decode_tc(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
                              const void* index, void* O, int32_t* idx, float* s_sel, float* w, void* ws,

@@ -92,12 +92,13 @@ struct SelTcArgs {
   const float* qn;        // [B*Hkv*L] |q̂|
   const float* kbar32;    // [B, Nc, Hkv, D]
   const float* kn;        // [B*Hkv, Ncp] |K̄_i|
-  const float* ktmax;     // [B*Hkv, Ncp/128, 4] max |K̄_i| over each tile of 128 chunks (in [0])
+  const float* ktmax;     // [B*Hkv, Ncp/64, 4] max |K̄_i| over each tile of 64 chunks (in [0])
   int32_t* idx;
   float* s_sel;
   unsigned* nflag;        // rows handed to the exact pass
   int32_t* flags;
   int L, Lp, Hkv, Nc, Ncp, topk, n_qt, BH;
+  int Nrow;  // rows of the bf16 summaries per (b, g): Nc, or a growing memory's capacity
   float scale_sel;
   // decode against a resident memory: rows are query tokens (all chunks
   // visible); block (split, g, query tile) scans chunks [split*range, +range)
@@ -238,7 +239,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
         tc::mbar_arrive_expect_tx(bar(BAR_FULL + s), kStageBytes);
 #pragma unroll
         for (int kb = 0; kb < D / 64; ++kb)
-          tc::tma_load_2d(ubase + s * kStageBytes + kb * kCt * 128, &tmap_k, kb * 64, bg * a.Nc + c_begin + n * kCt,
+          tc::tma_load_2d(ubase + s * kStageBytes + kb * kCt * 128, &tmap_k, kb * 64, bg * a.Nrow + c_begin + n * kCt,
                           bar(BAR_FULL + s));
       }
     }
@@ -559,11 +560,14 @@ __global__ void __launch_bounds__(256) sel_qhat_kernel(const uint16_t* __restric
 }
 
 // K̄ in bf16 with rows reordered to [b][g][i], |K̄_i| in fp32 ([b*Hkv+g][Ncp])
-// and the largest |K̄_i| of every tile of 128 chunks.
+// and the largest |K̄_i| of every tile of 64 chunks. The input holds Nc chunks
+// per batch row, chunk c0 first; they land at chunks c0 .. c0+Nc-1 of an
+// output laid out for Nrow chunks per (b, g) (c0 = 0, Nrow = Nc for a whole
+// memory; a growing memory appends its newly completed chunks).
 template <int D>
 __global__ void __launch_bounds__(256) sel_kbar_kernel(const float* __restrict__ kbar32, uint16_t* __restrict__ kb16,
                                                        float* __restrict__ kn, unsigned* __restrict__ ktmax,
-                                                       long long rows, int Nc, int Ncp, int Hkv) {
+                                                       long long rows, int Nc, int Ncp, int Hkv, int c0, int Nrow) {
   constexpr int D8 = D / 8;
   const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   const long long row = u / D8;  // input row (b, i, g)
@@ -577,13 +581,13 @@ __global__ void __launch_bounds__(256) sel_kbar_kernel(const float* __restrict__
   if (valid) {
     const int g = (int)(row % Hkv);
     const long long bi = row / Hkv;
-    i = (int)(bi % Nc);
+    i = c0 + (int)(bi % Nc);
     const long long b = bi / Nc;
     bg = b * Hkv + g;
     const float4* src = reinterpret_cast<const float4*>(kbar32 + row * D + e8 * 8);
     const float4 lo = __ldg(src), hi = __ldg(src + 1);
     x[0] = lo.x, x[1] = lo.y, x[2] = lo.z, x[3] = lo.w, x[4] = hi.x, x[5] = hi.y, x[6] = hi.z, x[7] = hi.w;
-    *reinterpret_cast<uint4*>(kb16 + (bg * Nc + i) * D + e8 * 8) = make_uint4(
+    *reinterpret_cast<uint4*>(kb16 + (bg * Nrow + i) * D + e8 * 8) = make_uint4(
         pack_bf16x2(x[0], x[1]), pack_bf16x2(x[2], x[3]), pack_bf16x2(x[4], x[5]), pack_bf16x2(x[6], x[7]));
   }
   float ss = 0.f;
@@ -961,7 +965,7 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int Ncp = padded_chunks(Dm);
   sel_kbar_kernel<DD><<<(unsigned)((krows * D8 + 255) / 256), 256, 0, st>>>(kbar32, kb16, kn, ktmax, krows, Dm.Nc,
-                                                                           Ncp, Dm.Hkv);
+                                                                           Ncp, Dm.Hkv, 0, Dm.Nc);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
@@ -987,6 +991,7 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   a.Hkv = Dm.Hkv;
   a.Nc = Dm.Nc;
   a.Ncp = Ncp;
+  a.Nrow = Dm.Nc;
   a.topk = Dm.topk;
   a.n_qt = (Dm.L + kTok - 1) / kTok;
   a.BH = BH;
@@ -1018,9 +1023,11 @@ struct DecIndexLayout {
   size_t kb16, kn, ktmax, total;
 };
 
+// Laid out for the memory's capacity (D.cap chunks per head), so that a growing
+// memory keeps every offset as chunks are appended.
 DecIndexLayout dec_index_layout(const DecodeDims& D) {
-  const size_t ncp = (size_t)((D.Nc + kCt - 1) / kCt * kCt);
-  const size_t krows = std::max<size_t>((size_t)D.Hkv * D.Nc, kCt);
+  const size_t ncp = (size_t)((D.cap + kCt - 1) / kCt * kCt);
+  const size_t krows = std::max<size_t>((size_t)D.Hkv * D.cap, kCt);
   DecIndexLayout lo{};
   size_t o = 0;
   lo.kb16 = o;
@@ -1096,7 +1103,7 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
   memset(&tq, 0, sizeof(tq));
   memset(&tk, 0, sizeof(tk));
   memset(&unused, 0, sizeof(unused));
-  const unsigned long long krows = std::max<unsigned long long>((unsigned long long)Dm.Hkv * Dm.Nc, kCt);
+  const unsigned long long krows = std::max<unsigned long long>((unsigned long long)Dm.Hkv * Dm.cap, kCt);
   if (!tc::make_rows_tmap(&tq, qh16, (unsigned long long)qrows, DD, kTok)) return cudaErrorNotSupported;
   if (!tc::make_rows_tmap(&tk, ib + ix.kb16, krows, DD, kCt)) return cudaErrorNotSupported;
   SelTcArgs a{};
@@ -1107,7 +1114,8 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
   a.L = 1;
   a.Hkv = Dm.Hkv;
   a.Nc = (int)Dm.Nc;
-  a.Ncp = (int)((Dm.Nc + kCt - 1) / kCt * kCt);
+  a.Ncp = (int)((Dm.cap + kCt - 1) / kCt * kCt);
+  a.Nrow = (int)Dm.cap;
   a.topk = Dm.topk;
   a.n_qt = lo.n_qt;
   a.BH = Dm.Hkv;
@@ -1145,28 +1153,40 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
 
 }  // namespace
 
-bool decode_tc_applies(const DecodeDims& D) { return D.topk <= 16 && D.Nc > 0 && D.Nc * (long long)D.Hkv < (1LL << 31); }
+bool decode_index_applies(const DecodeDims& D) {
+  return D.topk <= 16 && D.cap > 0 && D.cap * (long long)D.Hkv < (1LL << 31);
+}
 
-size_t decode_index_bytes(const DecodeDims& D) { return D.Nc > 0 ? dec_index_layout(D).total : 0; }
+bool decode_tc_applies(const DecodeDims& D) { return decode_index_applies(D) && D.Nc > 0; }
 
-cudaError_t launch_decode_index(const DecodeDims& Dm, const float* kbar32, void* index, cudaStream_t st) {
-  if (Dm.Nc == 0) return cudaSuccess;
+size_t decode_index_bytes(const DecodeDims& D) { return decode_index_applies(D) ? dec_index_layout(D).total : 0; }
+
+cudaError_t launch_index_rows(const DecodeDims& Dm, const float* kbar32, void* index, long long c0, long long c1,
+                              cudaStream_t st) {
+  if (c1 <= c0) return cudaSuccess;
   const DecIndexLayout ix = dec_index_layout(Dm);
   char* base = (char*)index;
-  const int Ncp = (int)((Dm.Nc + kCt - 1) / kCt * kCt);
-  cudaError_t e;
-  if ((e = cudaMemsetAsync(base + ix.ktmax, 0, ix.total - ix.ktmax, st)) != cudaSuccess) return e;
-  const long long krows = Dm.Nc * Dm.Hkv;  // input rows (i, g) of the one-batch memory
+  const int Ncp = (int)((Dm.cap + kCt - 1) / kCt * kCt);
+  const long long krows = (c1 - c0) * Dm.Hkv;  // input rows (i, g) of the one-batch memory, chunk c0 first
+  const float* src = kbar32 + c0 * Dm.Hkv * Dm.d;
   if (Dm.d == 64)
     sel_kbar_kernel<64><<<(unsigned)((krows * 8 + 255) / 256), 256, 0, st>>>(
-        kbar32, (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows, (int)Dm.Nc,
-        Ncp, Dm.Hkv);
+        src, (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows,
+        (int)(c1 - c0), Ncp, Dm.Hkv, (int)c0, (int)Dm.cap);
   else
     sel_kbar_kernel<128><<<(unsigned)((krows * 16 + 255) / 256), 256, 0, st>>>(
-        kbar32, (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows, (int)Dm.Nc,
-        Ncp, Dm.Hkv);
+        src, (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows,
+        (int)(c1 - c0), Ncp, Dm.Hkv, (int)c0, (int)Dm.cap);
   note_launches(1);
   return cudaGetLastError();
+}
+
+cudaError_t launch_decode_index(const DecodeDims& Dm, const float* kbar32, void* index, cudaStream_t st) {
+  // every byte starts at zero (rows and norms of chunks not yet in the memory,
+  // tile maxima before the atomic max), then the Nc chunks present are written
+  cudaError_t e = cudaMemsetAsync(index, 0, dec_index_layout(Dm).total, st);
+  if (e != cudaSuccess) return e;
+  return launch_index_rows(Dm, kbar32, index, 0, Dm.Nc, st);
 }
 
 size_t decode_tc_workspace(const DecodeDims& D) {

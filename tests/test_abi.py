@@ -177,6 +177,41 @@ def test_decode_index_sizes_and_fallback(lib):
     assert lib.hsa_decode_indexed(ctypes.byref(c), *[vp(FAKE)] * 4, vp(0), *[vp(FAKE)] * 5, 1 << 40, None) == INVALID
 
 
+def test_growing_memory_capacity_and_append_validation(lib):
+    vp, ll = ctypes.c_void_p, ctypes.c_longlong
+    # the index of a growing memory is laid out for its capacity, whatever it holds now
+    grown = hsa.DecodeShape(Bq=8, Hq=8, Hkv=2, d=64, n_chunks=1000).c()
+    empty = hsa.DecodeShape(Bq=8, Hq=8, Hkv=2, d=64, n_chunks=0, capacity_chunks=1000).c()
+    part = hsa.DecodeShape(Bq=8, Hq=8, Hkv=2, d=64, n_chunks=371, capacity_chunks=1000).c()
+    n = lib.hsa_decode_index_size(ctypes.byref(grown))
+    assert n > 0 and lib.hsa_decode_index_size(ctypes.byref(empty)) == n == lib.hsa_decode_index_size(
+        ctypes.byref(part))
+    assert lib.hsa_decode_index(ctypes.byref(empty), vp(FAKE), vp(FAKE), n - 16, None) == WORKSPACE
+    # capacity below the chunks present
+    bad = hsa.DecodeShape(Bq=8, Hq=8, Hkv=2, d=64, n_chunks=10, capacity_chunks=9).c()
+    assert lib.hsa_decode_workspace_size(ctypes.byref(bad)) == 0
+    assert lib.hsa_decode_index(ctypes.byref(bad), vp(FAKE), vp(FAKE), 1 << 30, None) == INVALID
+    ptrs = [vp(FAKE)] * 5
+
+    def append(shape, n_tokens, n_new, index=None, nbytes=0, p=ptrs):
+        return lib.hsa_memory_append(ctypes.byref(shape), ll(n_tokens), ll(n_new), *p, index, nbytes, None)
+
+    assert append(empty, 0, 0) == OK
+    assert append(empty, 1000 * 64, 0) == OK
+    assert append(empty, 1000 * 64 - 5, 6) == INVALID  # past the capacity
+    assert append(empty, -1, 4) == INVALID
+    assert append(empty, 0, -4) == INVALID
+    assert append(empty, 0, 64, p=[vp(FAKE), vp(0), vp(FAKE), vp(FAKE), vp(FAKE)]) == INVALID
+    assert append(empty, 0, 64, p=[vp(FAKE)] * 4 + [vp(FAKE + 4)]) == INVALID
+    assert append(empty, 0, 64, vp(FAKE), n - 1) == WORKSPACE
+    assert append(empty, 0, 64, vp(FAKE + 8), n) == WORKSPACE
+    big_k = hsa.DecodeShape(Bq=8, Hq=8, Hkv=2, d=64, n_chunks=0, capacity_chunks=1000, topk=20).c()
+    assert lib.hsa_decode_index_size(ctypes.byref(big_k)) == 0
+    assert append(big_k, 0, 64, vp(FAKE), 1 << 30) == UNSUPPORTED
+    odd = hsa.DecodeShape(Bq=8, Hq=8, Hkv=2, d=96, n_chunks=0, capacity_chunks=1000).c()
+    assert append(odd, 0, 64) == UNSUPPORTED
+
+
 def test_workspace_sizes_scale_with_the_problem(lib):
     s = shape(B=2, L=32768, Hq=32, Hkv=4)
     slots = 2 * 32768 * 4 * 8

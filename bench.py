@@ -54,8 +54,8 @@ def select_workload(number, batch):
 # has changed).
 NCU_TRAFFIC = {
     # bwd_delta + bwd_chunk + bwd_dq_merge at the long-context workload (B=2, L=32768), one launch each
-    "hsa_backward": {"bytes_per_launch": 14956860928, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
-                     "sha256": "94af4fae1d913bb0424fcd97893ad41cebaf173355fa87f46e7577dd498e886a"},
+    "hsa_backward": {"bytes_per_launch": 14965160192, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
+                     "sha256": "ae3da11b0fc69a8a51bed871078604f846f1f8559af42c900ab29db2051690ce"},
 }
 
 
@@ -107,9 +107,13 @@ def work_model(w):
         "hsa_chunk_pool": dict(flops=kv, bytes=kv * bf + kb * (f4 + bf)),
         "hsa_select_topk": dict(flops=2 * w.d * visible_pairs(w) + q, bytes=q * bf + kb * f4 + sel * (4 + f4)),
         "hsa_build_index": dict(flops=0, bytes=sel * 4 * 3 + w.B * w.Hkv * w.Nc * 4),
-        "hsa_forward": dict(flops=4 * w.S * w.d * u, bytes=q * bf * 2 + 2 * kv * bf + sel * (4 + f4 + f4)),
+        # gathered: the K and V rows of every selected chunk, once per (t, g, j) (the token-major loads of
+        # Algorithm 1); the backward gathers them again with dO and the partial gradients, about twice
+        "hsa_forward": dict(flops=4 * w.S * w.d * u, bytes=q * bf * 2 + 2 * kv * bf + sel * (4 + f4 + f4),
+                            gathered=sel * 2 * w.S * w.d * bf),
         "hsa_backward": dict(flops=10 * w.S * w.d * u,
-                             bytes=3 * q * bf + 2 * kv * bf + kb * f4 + q * f4 + 2 * kv * f4 + sel * (4 + f4)),
+                             bytes=3 * q * bf + 2 * kv * bf + kb * f4 + q * f4 + 2 * kv * f4 + sel * (4 + f4),
+                             gathered=2 * sel * 2 * w.S * w.d * bf),
     }
 
 
@@ -217,7 +221,7 @@ def run_gpu(args, rank, world, local_rank):
              dV=torch.empty(X["V"].shape, dtype=f32, device=dev))
     calls = ["hsa_chunk_pool", "hsa_select_topk", "hsa_build_index", "hsa_forward", "hsa_backward"]
 
-    def step(ev=None):
+    def step(ev=None, X=X, Y=Y):
         def mark(i):
             if ev is not None:
                 ev[i].record()
@@ -286,6 +290,9 @@ def run_gpu(args, rank, world, local_rank):
         kernels[c] = {"ms": round(per_call[c], 4), "bound": bound, "achieved": round(ach, 2), "peak": peak,
                       "unit": unit, "frac": round(ach / peak, 4), "algorithmic_flops": m["flops"],
                       "algorithmic_bytes": m["bytes"], "roofline_ms": round(t_min * 1e3, 4)}
+        if "gathered" in m:  # the gather reading: chunk rows delivered per second (reuse makes it exceed HBM)
+            kernels[c]["gathered_bytes"] = m["gathered"]
+            kernels[c]["gathered_gbs"] = round(m["gathered"] / sec / 1e9, 1)
     dom = max(calls, key=lambda c: per_call[c])
     tr = NCU_TRAFFIC.get(dom)
     traffic = None
@@ -307,26 +314,69 @@ def run_gpu(args, rank, world, local_rank):
         h2d = sum(t.numel() * t.element_size() for t in host_in.values())
         d2h = sum(t.numel() * t.element_size() for t in host_out.values())
 
-        def e2e_step():
-            for n, t in host_in.items():
-                X[n].copy_(t, non_blocking=True)
-            step()
-            for n, t in host_out.items():
-                t.copy_(Y[n], non_blocking=True)
+        # two sets of device inputs and outputs: the next step's inputs go up on one copy stream and the
+        # previous step's outputs come down on another while the compute stream runs the current step
+        X2 = {n: torch.empty_like(X[n]) for n in host_in}
+        Y2 = dict(Y, **{n: torch.empty_like(Y[n]) for n in host_out})
+        sets = [(X, Y), (X2, Y2)]
+        main = torch.cuda.current_stream(dev)
+        up, down = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
 
-        for _ in range(max(1, min(args.warmup, 2))):
-            e2e_step()
+        def e2e_run(n):
+            comp_done, out_done = [None, None], [None, None]
+            up.wait_stream(main)
+            down.wait_stream(main)
+            for i in range(n):
+                b = i % 2
+                Xb, Yb = sets[b]
+                with torch.cuda.stream(up):
+                    if comp_done[b] is not None:
+                        up.wait_event(comp_done[b])  # step i-2 no longer reads these inputs
+                    for nm, t in host_in.items():
+                        Xb[nm].copy_(t, non_blocking=True)
+                    ready = torch.cuda.Event()
+                    ready.record(up)
+                main.wait_event(ready)
+                if out_done[b] is not None:
+                    main.wait_event(out_done[b])  # step i-2's outputs have left
+                step(None, Xb, Yb)
+                comp_done[b] = torch.cuda.Event()
+                comp_done[b].record(main)
+                with torch.cuda.stream(down):
+                    down.wait_event(comp_done[b])
+                    for nm, t in host_out.items():
+                        t.copy_(Yb[nm], non_blocking=True)
+                    out_done[b] = torch.cuda.Event()
+                    out_done[b].record(down)
+            main.wait_stream(up)
+            main.wait_stream(down)
+
+        e2e_run(max(2, min(args.warmup, 4)))
         barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
-        for _ in range(K):
-            e2e_step()
+        e2e_run(K)
         e1.record()
         barrier()
         ms_e2e = max_over_ranks(e0.elapsed_time(e1))
+        # the link alone: each direction's copies of one step, timed by themselves
+        e0.record()
+        for nm, t in host_in.items():
+            X[nm].copy_(t, non_blocking=True)
+        e1.record()
+        barrier()
+        h2d_ms = e0.elapsed_time(e1)
+        e0.record()
+        for nm, t in host_out.items():
+            t.copy_(Y[nm], non_blocking=True)
+        e1.record()
+        barrier()
+        d2h_ms = e0.elapsed_time(e1)
         e2e = {"value": world * tokens * K / (ms_e2e / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e / K}
-        del host_in, host_out
+               "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e / K,
+               "h2d_gbs": round(h2d / (h2d_ms / 1e3) / 1e9, 1), "d2h_gbs": round(d2h / (d2h_ms / 1e3) / 1e9, 1),
+               "overlap": "inputs of step i+1 up and outputs of step i-1 down on two copy streams while step i runs"}
+        del host_in, host_out, X2, Y2, sets
 
     del X, Y, wss
     torch.cuda.empty_cache()
@@ -704,6 +754,7 @@ def main():
         dev = torch.device("cuda", local_rank)
         torch.cuda.set_device(dev)
         d = run_decode(args, dev, 1, peaks(), torch.cuda.synchronize, lambda x: x, hsa)
+        d["append"] = run_memory_append(args, dev, peaks(), torch.cuda.synchronize, lambda x: x, hsa)
         print(json.dumps({"decode": d}), flush=True)
         return
     import torch.distributed as dist

@@ -40,6 +40,24 @@ PREFILL = synth.WORKLOADS[3]
 DECODE = synth.WORKLOADS[5]
 
 
+def rank_shard(w, rank):
+    """The batch rank `rank` processes: the same shapes, its own seeds (rank 0 keeps the workload's), so
+    that N ranks process N distinct batches with no exchange (weak scaling)."""
+    return w if rank == 0 else w.with_(number=w.number + 100 * rank)
+
+
+def reduce_max(x, world, device):
+    """The largest of the ranks' values (every rank gets it); the step time a job reports."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def select_workload(number, batch):
     """The timed prefill workload (default: the long-context one); smaller ones serve profiling."""
     global PREFILL
@@ -203,7 +221,7 @@ def run_gpu(args, rank, world, local_rank):
             dist.barrier()
     hsa.load()
     pk = peaks()
-    w = PREFILL
+    w = rank_shard(PREFILL, rank)
     shape = hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk)
     log(f"[rank {rank}] generating inputs for {w.name}")
     X = {n: synth.device_tensor(w, n, dev) for n in ("q", "K", "V", "dO")}
@@ -245,11 +263,7 @@ def run_gpu(args, rank, world, local_rank):
             dist.barrier()
 
     def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return reduce_max(x, world, dev)
 
     for _ in range(args.warmup):
         step()
@@ -448,7 +462,7 @@ def run_variants(args, dev, pk, hsa, w, X, Y, barrier, model):
 def run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa):
     import torch
 
-    w = DECODE
+    w = rank_shard(DECODE, getattr(args, "rank", 0))
     T, Nc = w.L, w.Nc
     log(f"generating the {T}-token decode memory")
     Kmem = synth.device_tensor(w, "K", dev)
@@ -739,6 +753,7 @@ def main():
     args = ap.parse_args()
     select_workload(args.workload, args.batch)
     rank = int(os.environ.get("RANK", "0"))
+    args.rank = rank
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":

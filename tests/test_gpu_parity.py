@@ -183,10 +183,13 @@ def slice_bits(w, b, g, names):
     return out
 
 
-@pytest.mark.parametrize("cfg", [2, 3])
-def test_full_size_sampled(cfg):
+@pytest.mark.parametrize("cfg,inner,weights", [(2, "softmax", "softmax"), (3, "softmax", "softmax"),
+                                               (3, "softmax1", "stick")])
+def test_full_size_sampled(cfg, inner, weights):
+    # the variants (softmax-off-by-one inside chunks, stick-breaking chunk
+    # weights) at the long-context size, in the bench's launch configuration
     w = synth.WORKLOADS[cfg]
-    shape = shape_of(w)
+    shape = shape_of(w, inner, weights)
     dev = device_inputs(w, ("q", "K", "V", "dO"))
     wss = hsa.Workspaces(shape, dev["q"].device)
     fwd = hsa.hsa_forward_path(shape, dev["q"], dev["K"], dev["V"], wss)
@@ -211,7 +214,7 @@ def test_full_size_sampled(cfg):
     toks = np.unique(np.concatenate([rng.choice(w.L, 384, replace=False), [w.L - 1, 64, 65, 127]]))
     mask = np.zeros((1, w.L), np.uint8)
     mask[0, toks] = 1
-    O, wts = oracle.forward(q, K, V, idx, s_sel, w.S, token_mask=mask)
+    O, wts = oracle.forward(q, K, V, idx, s_sel, w.S, token_mask=mask, inner=inner, weights=weights)
     gotO = bf16_tensor_to_f64(fwd["O"][b, toks, g * G:(g + 1) * G])
     assert_close("O sampled", gotO, O[0, toks])
     # backward: dq on the sampled tokens; dK, dV on sampled chunks, with every
@@ -222,12 +225,15 @@ def test_full_size_sampled(cfg):
     mask2 = mask.copy()
     mask2[0, sel_any] = 1
     kbar64 = oracle.pool(K, w.S)
-    ref = oracle.backward(q, K, V, kbar64, idx, s_sel, dO, w.S, token_mask=mask2)
+    ref = oracle.backward(q, K, V, kbar64, idx, s_sel, dO, w.S, token_mask=mask2, inner=inner, weights=weights)
     assert_close("dq sampled", dq[b, toks, g * G:(g + 1) * G].cpu().numpy(), ref["dq"][0, toks])
     for c in chunks:
         rows = slice(c * w.S, (c + 1) * w.S)
         assert_close(f"dK chunk {c}", dK[b, rows, g].cpu().numpy(), ref["dK"][0, rows, 0])
         assert_close(f"dV chunk {c}", dV[b, rows, g].cpu().numpy(), ref["dV"][0, rows, 0])
+    assert_close("w sampled", fwd["w"][b, toks, g].cpu().numpy(), wts[0, toks, 0], max_abs=1e-5, rel=1e-5)
+    if (inner, weights) != ("softmax", "softmax"):
+        return
     # properties at any size: the value gradients add up to dO over tokens with a selection
     keff = (fwd["idx"] >= 0).sum(-1)  # [B, L, Hkv]
     m = (keff > 0).repeat_interleave(G, dim=2).unsqueeze(-1).float()

@@ -63,22 +63,26 @@ struct SelCfg {
 
 __device__ unsigned g_sel_status;
 
-template <int D, int KT>
+// Decode blocks (DEC) keep no exact keys: the merge rescores their candidates.
+template <int D, int KT, bool DEC = false>
 struct SelTcSmem {
   using Cfg = SelCfg<KT>;
   static constexpr int kStages = Cfg::kStages, kAcc = Cfg::kAcc, kBuf = Cfg::kBuf;
+  // chunk norms of a tile travel in their own ring, requested by the loader as
+  // soon as the scan has released the slot (kKn tiles ahead of the scan)
+  static constexpr int kKn = 6;
   // barrier slots
   static constexpr int BAR_A = 0, BAR_Q32 = 1, BAR_FULL = 2, BAR_EMPTY = 2 + kStages,
                        BAR_ACC_FULL = 2 + 2 * kStages, BAR_ACC_EMPTY = BAR_ACC_FULL + kAcc,
-                       BAR_KN = BAR_ACC_EMPTY + kAcc, kBars = BAR_KN + kAcc;
+                       BAR_KN = BAR_ACC_EMPTY + kAcc, BAR_KNE = BAR_KN + kKn, kBars = BAR_KNE + kKn;
   // A and B are adjacent: once every MMA is done they hold the rows' fp32 q̂ ([e][row], 128 * D floats)
   uint16_t A[kTok * D];                  // q̂ (bf16) of the block's rows, K-major SW128
   uint16_t B[kStages][kCt * D];          // chunk-summary tiles, K-major SW128
   float bl[kBuf][kTok];                  // second-pass entries: lower bounds, later exact scores
   float bu[kBuf][kTok];                  //   upper bounds
   int bi[kBuf][kTok];                    //   chunk indices
-  unsigned long long chosen[KT][kTok];   // the k best exact keys
-  float knt[kAcc][kCt + 4];              // |K̄_i| of the tile in accumulator ab, then the tile's max
+  unsigned long long chosen[DEC ? 1 : KT][kTok];  // the k best exact keys (prefill)
+  float knt[kKn][kCt + 4];               // |K̄_i| of a tile, then the tile's max (ring of kKn)
   uint64_t bar[kBars];
   uint32_t tmem_base;
   int abort_flag;
@@ -169,10 +173,11 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     sel_tc_kernel(SelTcArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                   const __grid_constant__ CUtensorMap tmap_q32t) {
   extern __shared__ unsigned char smem_raw[];
-  using Smem = SelTcSmem<D, KT>;
-  constexpr int kStages = Smem::kStages, kAcc = Smem::kAcc, kTmemCols = SelCfg<KT>::kTmemCols;
+  using Smem = SelTcSmem<D, KT, DEC>;
+  constexpr int kStages = Smem::kStages, kAcc = Smem::kAcc, kKn = Smem::kKn, kTmemCols = SelCfg<KT>::kTmemCols;
   constexpr int BAR_A = Smem::BAR_A, BAR_Q32 = Smem::BAR_Q32, BAR_FULL = Smem::BAR_FULL, BAR_EMPTY = Smem::BAR_EMPTY,
-                BAR_ACC_FULL = Smem::BAR_ACC_FULL, BAR_ACC_EMPTY = Smem::BAR_ACC_EMPTY, BAR_KN = Smem::BAR_KN;
+                BAR_ACC_FULL = Smem::BAR_ACC_FULL, BAR_ACC_EMPTY = Smem::BAR_ACC_EMPTY, BAR_KN = Smem::BAR_KN,
+                BAR_KNE = Smem::BAR_KNE;
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int qt, bg, split = 0, c_begin = 0, vis_max;
@@ -211,7 +216,10 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     for (int i = 0; i < kAcc; ++i) {
       tc::mbar_init(bar(BAR_ACC_FULL + i), 1);
       tc::mbar_init(bar(BAR_ACC_EMPTY + i), 128);
+    }
+    for (int i = 0; i < kKn; ++i) {
       tc::mbar_init(bar(BAR_KN + i), 1);
+      tc::mbar_init(bar(BAR_KNE + i), 128);
     }
     sm.abort_flag = 0;
     tc::fence_mbar_init();
@@ -234,7 +242,14 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
                         bar(BAR_A));
       for (int it = 0; it < 2 * ntiles; ++it) {  // two passes over the tiles
         const int n = tile_of(it);
-        const int s = it % kStages;
+        const int s = it % kStages, kq = it % kKn;
+        // the tile's chunk norms (the scan of tile it - kKn has released the slot)
+        if (!tc::mbar_wait(bar(BAR_KNE + kq), ((it / kKn) & 1) ^ 1, abort_flag, status)) break;
+        tc::mbar_arrive_expect_tx(bar(BAR_KN + kq), (kCt + 4) * 4);
+        tc::bulk_load(smem_u32(sm.knt[kq]), a.kn + (long long)bg * a.Ncp + c_begin + n * kCt, kCt * 4,
+                      bar(BAR_KN + kq));
+        tc::bulk_load(smem_u32(&sm.knt[kq][kCt]),
+                      a.ktmax + ((long long)bg * (a.Ncp / kCt) + c_begin / kCt + n) * 4, 16, bar(BAR_KN + kq));
         if (!tc::mbar_wait(bar(BAR_EMPTY + s), ((it / kStages) & 1) ^ 1, abort_flag, status)) break;
         tc::mbar_arrive_expect_tx(bar(BAR_FULL + s), kStageBytes);
 #pragma unroll
@@ -255,12 +270,6 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
         if (!tc::mbar_wait(bar(BAR_FULL + s), (it / kStages) & 1, abort_flag, status)) break;
         if (!tc::mbar_wait(bar(BAR_ACC_EMPTY + ab), ((it / kAcc) & 1) ^ 1, abort_flag, status)) break;
         tc::fence_after_sync();
-        // the tile's chunk norms travel with its accumulator (the scan has released both)
-        tc::mbar_arrive_expect_tx(bar(BAR_KN + ab), (kCt + 4) * 4);
-        tc::bulk_load(smem_u32(sm.knt[ab]), a.kn + (long long)bg * a.Ncp + c_begin + n * kCt, kCt * 4,
-                      bar(BAR_KN + ab));
-        tc::bulk_load(smem_u32(&sm.knt[ab][kCt]),
-                      a.ktmax + ((long long)bg * (a.Ncp / kCt) + c_begin / kCt + n) * 4, 16, bar(BAR_KN + ab));
         const uint32_t bbase = ubase + s * kStageBytes;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
@@ -310,9 +319,10 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       const int ab = it % kAcc;
       if (it == ntiles) lam_lo = bm[KT - 1];
       if (!tc::mbar_wait(bar(BAR_ACC_FULL + ab), (it / kAcc) & 1, abort_flag, status)) break;
-      if (!tc::mbar_wait(bar(BAR_KN + ab), (it / kAcc) & 1, abort_flag, status)) break;
+      const int kq = it % kKn;
+      if (!tc::mbar_wait(bar(BAR_KN + kq), (it / kKn) & 1, abort_flag, status)) break;
       tc::fence_after_sync();
-      const float* knt = sm.knt[ab];
+      const float* knt = sm.knt[kq];
       const float emax = fmaf(cq, knt[kCt], kEpsAbs);  // the tile's largest eps_i
 #pragma unroll 1
       for (int h = 0; h < kCt / 32; ++h) {
@@ -387,6 +397,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       }
       tc::fence_before_sync();
       tc::mbar_arrive(bar(BAR_ACC_EMPTY + ab));
+      tc::mbar_arrive(bar(BAR_KNE + kq));
     }
     if (ntiles == 0) cnt = 0;
     // lambda of the kept entries: at most the row's true lambda (a subset's k-th largest)
@@ -1129,7 +1140,7 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
   a.cand_n = (int32_t*)(base + lo.cn);
   a.cand_d = (float*)(base + lo.cd);
   a.cand_s = (float4*)(base + lo.cs);
-  const size_t smem = sizeof(SelTcSmem<DD, KT>) + 1024;
+  const size_t smem = sizeof(SelTcSmem<DD, KT, true>) + 1024;
   if ((e = cudaFuncSetAttribute(sel_tc_kernel<DD, KT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)smem)) != cudaSuccess)
     return e;

@@ -463,6 +463,8 @@ def run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa):
     import torch
 
     w = rank_shard(DECODE, getattr(args, "rank", 0))
+    if getattr(args, "decode_tokens", None):  # a smaller memory (profiling captures)
+        w = w.with_(L=args.decode_tokens)
     T, Nc = w.L, w.Nc
     log(f"generating the {T}-token decode memory")
     Kmem = synth.device_tensor(w, "K", dev)
@@ -748,6 +750,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", type=int, default=3, help="prefill workload number (3 is the headline)")
     ap.add_argument("--batch", type=int, default=0, help="override the workload's batch (profiling)")
+    ap.add_argument("--decode-tokens", type=int, default=None,
+                    help="decode memory length (default: the 2^26-token workload); for profiling captures")
     ap.add_argument("--decode-only", action="store_true",
                     help="run only the decode sub-benchmark and print its object (profiling)")
     args = ap.parse_args()

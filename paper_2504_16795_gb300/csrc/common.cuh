@@ -265,9 +265,11 @@ size_t decode_workspace(const DecodeDims& D);
 bool memory_device_readable(const void* p);
 cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, const void* V, const float* kbar32,
                           void* O, int32_t* idx, float* s_sel, float* w, void* ws, cudaStream_t st);
-// Token-level attention over the selected chunks and the weighted sum (the last two decode steps).
+// Token-level attention over the selected chunks and the weighted sum (the last two decode steps);
+// scratch: decode_attend_scratch(D) bytes, 256-byte aligned (partials, then one counter per row).
+size_t decode_attend_scratch(const DecodeDims& D);
 cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void* K, const void* V,
-                                 const int32_t* idx, const float* w, void* O, float* opart, cudaStream_t st);
+                                 const int32_t* idx, const float* w, void* O, void* scratch, cudaStream_t st);
 // Decode over a memory index (bf16 summaries, norms): tensor-core scan with exact rescoring (topk <= 16).
 bool decode_index_applies(const DecodeDims& D);  // topk <= 16: the memory has an index
 bool decode_tc_applies(const DecodeDims& D);     // ... and at least one chunk

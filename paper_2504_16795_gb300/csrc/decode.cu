@@ -134,26 +134,32 @@ __global__ void dec_merge_kernel(const unsigned long long* __restrict__ cand, in
   if (lane < topk) w[o + lane] = wj;
 }
 
+// K and V rows stay bf16 in shared memory, each row padded by 16 bytes so that
+// the lanes of a warp reading 16 bytes of 32 different rows hit distinct banks.
 template <int D>
 struct AttSmem {
-  float K[kChunk][D + 1];
-  float V[kChunk][D];
+  static constexpr int kRow = D + 8;  // bf16 elements per staged row
+  uint16_t K[kChunk * kRow];
+  uint16_t V[kChunk * kRow];
   float q[16][D];
   float P[16][kChunk];
 };
 
-// Token-level attention of one (query, group) over one selected chunk.
+// Token-level attention of one (query, group) over one selected chunk. The
+// block that finishes last for its (query, group) also forms the output
+// O = sum_j w_j O_j, in slot order (a per-row counter, zeroed before the launch,
+// tells it that the other partials are written). Each product keeps its fused
+// multiply-adds in index order (scores over the head dimension, outputs over the
+// chunk's tokens); threads hold several of them at once so that one shared-memory
+// read feeds several products.
 template <int D>
-__global__ void __launch_bounds__(kThreads) dec_attend_kernel(const uint16_t* __restrict__ q,
-                                                              const uint16_t* __restrict__ Kmem,
-                                                              const uint16_t* __restrict__ Vmem,
-                                                              const int32_t* __restrict__ idx, float* __restrict__ Opart,
-                                                              int Hq, int Hkv, int G, int topk, float scale_attn,
-                                                              int softmax1) {
+__global__ void __launch_bounds__(kThreads) dec_attend_kernel(
+    const uint16_t* __restrict__ q, const uint16_t* __restrict__ Kmem, const uint16_t* __restrict__ Vmem,
+    const int32_t* __restrict__ idx, float* Opart, const float* __restrict__ w, uint16_t* __restrict__ O,
+    unsigned* __restrict__ counters, int Hq, int Hkv, int G, int topk, float scale_attn, int softmax1) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   AttSmem<D>& sm = *reinterpret_cast<AttSmem<D>*>(smem_raw);
-  auto& Ks = sm.K;
-  auto& Vs = sm.V;
+  constexpr int kRow = AttSmem<D>::kRow, D8 = D / 8;
   auto& qsm = sm.q;
   auto& P = sm.P;
   const int slot = blockIdx.x;  // ((b * Hkv + g) * topk + j)
@@ -164,44 +170,63 @@ __global__ void __launch_bounds__(kThreads) dec_attend_kernel(const uint16_t* __
   const int c = idx[slot];
   if (c < 0) {
     for (int u = tid; u < G * D; u += kThreads) out[u] = 0.f;
-    return;
-  }
+  } else {
   // the chunk's rows in 16-byte pieces, every piece of a thread requested before
-  // the first is used (the memory may also sit in host memory, read over the
+  // the first is stored (the memory may also sit in host memory, read over the
   // CPU-GPU link, where a round trip costs microseconds)
-  constexpr int kPieces = kChunk * (D / 8) / kThreads;
-  static_assert(kPieces * kThreads == kChunk * (D / 8), "whole pieces per thread");
+  constexpr int kPieces = kChunk * D8 / kThreads;
+  static_assert(kPieces * kThreads == kChunk * D8, "whole pieces per thread");
   uint4 kv[kPieces], vv[kPieces];
 #pragma unroll
   for (int i = 0; i < kPieces; ++i) {
     const int u = tid + i * kThreads;
-    const long long r = (((long long)c * kChunk + u / (D / 8)) * Hkv + g) * D + (u % (D / 8)) * 8;
+    const long long r = (((long long)c * kChunk + u / D8) * Hkv + g) * D + (u % D8) * 8;
     kv[i] = *reinterpret_cast<const uint4*>(Kmem + r);
     vv[i] = *reinterpret_cast<const uint4*>(Vmem + r);
   }
 #pragma unroll
   for (int i = 0; i < kPieces; ++i) {
     const int u = tid + i * kThreads;
-    const int s = u / (D / 8), e = (u % (D / 8)) * 8;
-    const uint32_t kw[4] = {kv[i].x, kv[i].y, kv[i].z, kv[i].w}, vw[4] = {vv[i].x, vv[i].y, vv[i].z, vv[i].w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      Ks[s][e + 2 * j] = bf16_lo(kw[j]);
-      Ks[s][e + 2 * j + 1] = bf16_hi(kw[j]);
-      Vs[s][e + 2 * j] = bf16_lo(vw[j]);
-      Vs[s][e + 2 * j + 1] = bf16_hi(vw[j]);
-    }
+    const int o = (u / D8) * kRow + (u % D8) * 8;
+    *reinterpret_cast<uint4*>(&sm.K[o]) = kv[i];
+    *reinterpret_cast<uint4*>(&sm.V[o]) = vv[i];
   }
   for (int u = tid; u < G * D; u += kThreads) {
     const int hh = u / D, e = u % D;
     qsm[hh][e] = bf16_bits_to_f32(q[((long long)b * Hq + (long long)g * G + hh) * D + e]);
   }
   __syncthreads();
-  for (int u = tid; u < G * kChunk; u += kThreads) {
-    const int hh = u / kChunk, s = u % kChunk;
-    float acc = 0.f;
-    for (int e = 0; e < D; ++e) acc = fmaf(qsm[hh][e], Ks[s][e], acc);
-    P[hh][s] = acc * scale_attn;
+  {
+    // scores: thread (token s, heads hq, hq + 4, ...): one K read serves its heads
+    static_assert(kThreads == 4 * kChunk, "four head groups of one thread per token");
+    const int s = tid % kChunk, hq = tid / kChunk;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint16_t* krow = &sm.K[s * kRow];
+#pragma unroll 4
+    for (int e8 = 0; e8 < D8; ++e8) {
+      const uint4 kp = *reinterpret_cast<const uint4*>(krow + e8 * 8);
+      const float kf[8] = {bf16_lo(kp.x), bf16_hi(kp.x), bf16_lo(kp.y), bf16_hi(kp.y),
+                           bf16_lo(kp.z), bf16_hi(kp.z), bf16_lo(kp.w), bf16_hi(kp.w)};
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        const int hh = hq + 4 * m;
+        if (hh < G) {
+          const float4 q0 = *reinterpret_cast<const float4*>(&qsm[hh][e8 * 8]);
+          const float4 q1 = *reinterpret_cast<const float4*>(&qsm[hh][e8 * 8 + 4]);
+          acc[m] = fmaf(q0.x, kf[0], acc[m]);
+          acc[m] = fmaf(q0.y, kf[1], acc[m]);
+          acc[m] = fmaf(q0.z, kf[2], acc[m]);
+          acc[m] = fmaf(q0.w, kf[3], acc[m]);
+          acc[m] = fmaf(q1.x, kf[4], acc[m]);
+          acc[m] = fmaf(q1.y, kf[5], acc[m]);
+          acc[m] = fmaf(q1.z, kf[6], acc[m]);
+          acc[m] = fmaf(q1.w, kf[7], acc[m]);
+        }
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < 4; ++m)
+      if (hq + 4 * m < G) P[hq + 4 * m][s] = acc[m] * scale_attn;
   }
   __syncthreads();
   for (int hh = warp; hh < G; hh += kThreads / 32) {
@@ -213,23 +238,43 @@ __global__ void __launch_bounds__(kThreads) dec_attend_kernel(const uint16_t* __
     P[hh][lane + 32] = e1 / z;
   }
   __syncthreads();
-  for (int u = tid; u < G * D; u += kThreads) {
-    const int hh = u / D, e = u % D;
-    float acc = 0.f;
-    for (int s = 0; s < kChunk; ++s) acc = fmaf(P[hh][s], Vs[s][e], acc);
-    out[u] = acc;
+  // outputs: thread (8 consecutive dimensions, head): one V read serves 8 products
+  for (int u = tid; u < G * D8; u += kThreads) {
+    const int hh = u / D8, e8 = u % D8;
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+    for (int t = 0; t < kChunk; ++t) {
+      const uint4 vp = *reinterpret_cast<const uint4*>(&sm.V[t * kRow + e8 * 8]);
+      const float p = P[hh][t];
+      acc[0] = fmaf(p, bf16_lo(vp.x), acc[0]);
+      acc[1] = fmaf(p, bf16_hi(vp.x), acc[1]);
+      acc[2] = fmaf(p, bf16_lo(vp.y), acc[2]);
+      acc[3] = fmaf(p, bf16_hi(vp.y), acc[3]);
+      acc[4] = fmaf(p, bf16_lo(vp.z), acc[4]);
+      acc[5] = fmaf(p, bf16_hi(vp.z), acc[5]);
+      acc[6] = fmaf(p, bf16_lo(vp.w), acc[6]);
+      acc[7] = fmaf(p, bf16_hi(vp.w), acc[7]);
+    }
+    float4* o4 = reinterpret_cast<float4*>(out + hh * D + e8 * 8);
+    o4[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    o4[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
   }
-}
-
-template <int D>
-__global__ void dec_out_kernel(const float* __restrict__ Opart, const float* __restrict__ w, uint16_t* __restrict__ O,
-                               int G, int topk) {
-  const int bg = blockIdx.x;
-  for (int u = threadIdx.x; u < G * D; u += blockDim.x) {
+  }
+  // the last block of the row sums the partials
+  __shared__ int last;
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) last = atomicAdd(&counters[bg], 1u) == (unsigned)(topk - 1);
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  const float* parts = Opart + (long long)bg * topk * G * D;
+  for (int u = tid; u < G * D; u += kThreads) {
     float acc = 0.f;
-    for (int j = 0; j < topk; ++j) acc = fmaf(w[(long long)bg * topk + j], Opart[((long long)bg * topk + j) * G * D + u], acc);
+    for (int j = 0; j < topk; ++j) acc = fmaf(w[(long long)bg * topk + j], __ldcg(parts + (long long)j * G * D + u), acc);
     O[(long long)bg * G * D + u] = f32_to_bf16_bits(acc);
   }
+  if (tid == 0) counters[bg] = 0u;
 }
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -248,7 +293,7 @@ DecLayout dec_layout(const DecodeDims& D) {
   lo.cand = o;
   o = align256(o + sizeof(unsigned long long) * (size_t)D.Bq * D.Hkv * lo.nx * D.topk);
   lo.opart = o;
-  o = align256(o + sizeof(float) * (size_t)D.Bq * D.Hkv * D.topk * D.G * D.d);
+  o = align256(o + decode_attend_scratch(D));
   lo.total = o;
   return lo;
 }
@@ -260,7 +305,6 @@ cudaError_t run(const DecodeDims& D, const void* q, const void* K, const void* V
   char* base = (char*)ws;
   float* qhat = (float*)(base + lo.qhat);
   unsigned long long* cand = (unsigned long long*)(base + lo.cand);
-  float* opart = (float*)(base + lo.opart);
   const int rows = D.Bq * D.Hkv;
   cudaError_t e;
   dec_qhat_kernel<DD><<<rows, 128, 0, st>>>((const uint16_t*)q, qhat, D.Hq, D.Hkv, D.G);
@@ -283,48 +327,40 @@ cudaError_t run(const DecodeDims& D, const void* q, const void* K, const void* V
   dec_merge_kernel<<<(rows + 7) / 8, 256, 0, st>>>(cand, idx, s_sel, w, rows, lo.nx, D.topk, D.stick ? 1 : 0);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  const size_t att_smem = sizeof(AttSmem<DD>);
-  if ((e = cudaFuncSetAttribute(dec_attend_kernel<DD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)att_smem)) !=
-      cudaSuccess)
-    return e;
-  dec_attend_kernel<DD><<<rows * D.topk, kThreads, att_smem, st>>>((const uint16_t*)q, (const uint16_t*)K,
-                                                           (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk,
-                                                           D.scale_attn, D.softmax1 ? 1 : 0);
-  note_launches(1);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  dec_out_kernel<DD><<<rows, 256, 0, st>>>(opart, w, (uint16_t*)O, D.G, D.topk);
-  note_launches(1);
-  return cudaGetLastError();
+  return launch_decode_attend(D, q, K, V, idx, w, O, base + lo.opart, st);
 }
 
 }  // namespace
 
 size_t decode_workspace(const DecodeDims& D) { return dec_layout(D).total; }
 
+size_t decode_attend_scratch(const DecodeDims& D) {
+  const size_t rows = (size_t)D.Bq * D.Hkv;
+  return align256(sizeof(float) * rows * D.topk * D.G * D.d) + align256(sizeof(unsigned) * rows);
+}
+
 cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void* K, const void* V,
-                                 const int32_t* idx, const float* w, void* O, float* opart, cudaStream_t st) {
+                                 const int32_t* idx, const float* w, void* O, void* scratch, cudaStream_t st) {
   const int rows = D.Bq * D.Hkv;
-  cudaError_t e;
+  float* opart = (float*)scratch;
+  unsigned* counters =
+      (unsigned*)((char*)scratch + align256(sizeof(float) * (size_t)rows * D.topk * D.G * D.d));
+  cudaError_t e = cudaMemsetAsync(counters, 0, sizeof(unsigned) * (size_t)rows, st);
+  if (e != cudaSuccess) return e;
   if (D.d == 64) {
     if ((e = cudaFuncSetAttribute(dec_attend_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)sizeof(AttSmem<64>))) != cudaSuccess)
       return e;
     dec_attend_kernel<64><<<rows * D.topk, kThreads, sizeof(AttSmem<64>), st>>>(
-        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk, D.scale_attn,
-        D.softmax1 ? 1 : 0);
-    note_launches(1);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    dec_out_kernel<64><<<rows, 256, 0, st>>>(opart, w, (uint16_t*)O, D.G, D.topk);
+        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, w, (uint16_t*)O, counters, D.Hq,
+        D.Hkv, D.G, D.topk, D.scale_attn, D.softmax1 ? 1 : 0);
   } else {
     if ((e = cudaFuncSetAttribute(dec_attend_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)sizeof(AttSmem<128>))) != cudaSuccess)
       return e;
     dec_attend_kernel<128><<<rows * D.topk, kThreads, sizeof(AttSmem<128>), st>>>(
-        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, D.Hq, D.Hkv, D.G, D.topk, D.scale_attn,
-        D.softmax1 ? 1 : 0);
-    note_launches(1);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    dec_out_kernel<128><<<rows, 256, 0, st>>>(opart, w, (uint16_t*)O, D.G, D.topk);
+        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, w, (uint16_t*)O, counters, D.Hq,
+        D.Hkv, D.G, D.topk, D.scale_attn, D.softmax1 ? 1 : 0);
   }
   note_launches(1);
   return cudaGetLastError();

@@ -1087,7 +1087,7 @@ DecTcLayout dec_tc_layout(const DecodeDims& D) {
   lo.cs = o;
   o = align256(o + rows * lo.n_split * 16);
   lo.opart = o;
-  o = align256(o + rows * D.topk * D.G * D.d * 4);
+  o = align256(o + decode_attend_scratch(D));
   lo.total = o;
   return lo;
 }
@@ -1159,7 +1159,7 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
       Dm.Hkv, (int)Dm.Nc, lo.n_split, lo.range, Dm.topk, Dm.scale_sel, Dm.stick ? 1 : 0);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  return launch_decode_attend(Dm, q, K, V, idx, w, O, (float*)(base + lo.opart), st);
+  return launch_decode_attend(Dm, q, K, V, idx, w, O, base + lo.opart, st);
 }
 
 }  // namespace

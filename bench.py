@@ -72,7 +72,7 @@ def select_workload(number, batch):
 # has changed).
 NCU_TRAFFIC = {
     # bwd_delta + bwd_chunk + bwd_dq_merge at the long-context workload (B=2, L=32768), one launch each
-    "hsa_backward": {"bytes_per_launch": 14965160192, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
+    "hsa_backward": {"bytes_per_launch": 14943142400, "source": "paper_2504_16795_gb300/csrc/bwd.cu",
                      "sha256": "ae3da11b0fc69a8a51bed871078604f846f1f8559af42c900ab29db2051690ce"},
 }
 
@@ -317,6 +317,7 @@ def run_gpu(args, rank, world, local_rank):
                  "peak_source": f"{pk['source']} ({'bf16 sustained' if roof['bound'] == 'tensor' else 'hbm copy'})"})
 
     variants = None if args.no_variants else run_variants(args, dev, pk, hsa, w, X, Y, barrier, model)
+    small = None if args.no_variants else run_small_configs(args, dev, pk, hsa)
 
     # end to end through host buffers: H2D inputs, the path, D2H outputs, every step
     e2e = None
@@ -401,7 +402,7 @@ def run_gpu(args, rank, world, local_rank):
         decode["append"] = run_memory_append(args, dev, pk, barrier, max_over_ranks, hsa)
 
     return dict(value=value, ms_step=ms_step, kernels=kernels, roofline=roof, e2e=e2e, clocks=clocks,
-                launches=launches, decode=decode, wall_ms_step=wall / K * 1e3, variants=variants)
+                launches=launches, decode=decode, wall_ms_step=wall / K * 1e3, variants=variants, small=small)
 
 
 def run_variants(args, dev, pk, hsa, w, X, Y, barrier, model):
@@ -589,6 +590,44 @@ def run_memory_append(args, dev, pk, barrier, max_over_ranks, hsa):
                          "frac": round(achieved / pk["hbm"], 4), "algorithmic_bytes": nbytes,
                          "counted": "read K_new, V_new; write K_mem, V_mem, K̄ fp32; index: read K̄, write bf16 "
                                     "rows and norms"}}
+
+
+def run_small_configs(args, dev, pk, hsa):
+    """The smaller workloads, timed the same way (one step = pool, select, index, forward, backward):
+    the tiny one is bound by launch latency, not by the hardware."""
+    import torch
+
+    out = {}
+    for number in (1, 2):
+        w = synth.WORKLOADS[number]
+        shape = hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk)
+        X = {n: synth.device_tensor(w, n, dev) for n in ("q", "K", "V", "dO")}
+        wss = hsa.Workspaces(shape, dev)
+
+        def step():
+            fwd = hsa.hsa_forward_path(shape, X["q"], X["K"], X["V"], wss)
+            hsa.hsa_backward_path(shape, X["q"], X["K"], X["V"], fwd, X["dO"], wss)
+
+        for _ in range(max(args.warmup, 3)):
+            step()
+        torch.cuda.synchronize()
+        n = 20
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(n):
+            step()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / n
+        model = work_model(w)
+        t_min = sum(bound_of(m["flops"], m["bytes"], pk)[1] for m in model.values())
+        out[w.name] = {"ms_per_step": round(ms, 4), "tokens_per_s": w.B * w.L / (ms / 1e3),
+                       "roofline_ms": round(t_min * 1e3, 4), "frac": round(t_min * 1e3 / ms, 4),
+                       "bound": "launch latency" if t_min * 1e3 < 0.01 * ms else "hbm/tensor",
+                       "shape": f"B={w.B} L={w.L} Hq={w.Hq} Hkv={w.Hkv} d={w.d} k={w.topk}"}
+        del X, wss
+    torch.cuda.empty_cache()
+    return out
 
 
 def mem_available_bytes():
@@ -793,7 +832,7 @@ def main():
                 "warmup": args.warmup, "ms_per_step": r["ms_step"], "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_obj(),
                 "roofline": r["roofline"], "cpu_baseline": cpu, "e2e": r["e2e"], "gpu_launches": r["launches"],
-                "clocks": r["clocks"], "kernels": r["kernels"], "decode": r["decode"], "variants": r["variants"],
+                "clocks": r["clocks"], "kernels": r["kernels"], "decode": r["decode"], "variants": r["variants"], "small_configs": r["small"],
                 "wall_ms_per_step": r["wall_ms_step"]}
         print(json.dumps(line), flush=True)
     if world > 1:

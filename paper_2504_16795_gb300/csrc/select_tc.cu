@@ -758,7 +758,8 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
   __shared__ int rn[kMaxSplit];     // per range: exported entries
   __shared__ float red[kMergeWarps];
   __shared__ float lam_s;
-  __shared__ int any_unsure, n_cand;
+  __shared__ int any_unsure, n_cand, n_hit;
+  __shared__ int hit[kMaxSplit];    // ranges whose bounds can reach the current threshold
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const int row = blockIdx.x;  // b * Hkv + g
   const int b = row / Hkv, g = row % Hkv;
@@ -777,23 +778,6 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
   }
   ls = warp_max(ls);
   if (lane == 0) red[wib] = ls;
-  __syncthreads();
-  if (wib == 0) {  // the k-th largest of the ranges' largest lower bounds
-    unsigned long long top = 0ull;
-    for (int sp0 = 0; sp0 < n_split; sp0 += 32) {
-      const int sp = sp0 + lane;
-      const unsigned long long key =
-          sp < n_split && rs[sp].y > -INFINITY ? ((unsigned long long)order_bits(rs[sp].y) << 32) | (uint32_t)sp : 0ull;
-      warp_topk_offer(top, key, topk, lane);
-    }
-    const unsigned long long kth = __shfl_sync(0xFFFFFFFFu, top, topk - 1);
-    if (lane == 0) lam_s = kth != 0ull ? order_bits_to_float((uint32_t)(kth >> 32)) : -INFINITY;
-  }
-  __syncthreads();
-  float lam_star = lam_s;
-#pragma unroll
-  for (int k = 0; k < kMergeWarps; ++k) lam_star = fmaxf(lam_star, red[k]);
-  __syncthreads();  // lam_s is written again below
   auto krow = [&](int c) { return kbar32 + ((long long)c * Hkv + g) * D; };
   auto combine = [&](unsigned long long mine) {  // top-k of the warp lists, in warp 0
     lists[wib][lane] = mine;
@@ -804,24 +788,53 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
     __syncthreads();
     return all;
   };
+  // the ranges whose bound `field` reaches t, listed in shared memory (any order)
+  auto list_ranges = [&](int field, float t) {
+    if (threadIdx.x == 0) n_hit = 0;
+    __syncthreads();
+    for (int sp = threadIdx.x; sp < n_split; sp += kMergeWarps * 32) {
+      const float4 v = rs[sp];
+      if ((field == 1 ? v.y : v.z) >= t) hit[atomicAdd(&n_hit, 1)] = sp;
+    }
+    __syncthreads();
+    return n_hit;
+  };
+  __syncthreads();
+  {  // the k-th largest of the ranges' largest lower bounds (each warp a share of the ranges)
+    unsigned long long top = 0ull;
+    for (int sp0 = wib * 32; sp0 < n_split; sp0 += kMergeWarps * 32) {
+      const int sp = sp0 + lane;
+      const unsigned long long key =
+          sp < n_split && rs[sp].y > -INFINITY ? ((unsigned long long)order_bits(rs[sp].y) << 32) | (uint32_t)sp : 0ull;
+      warp_topk_offer(top, key, topk, lane);
+    }
+    const unsigned long long all = combine(top);
+    if (wib == 0) {
+      const unsigned long long kth = __shfl_sync(0xFFFFFFFFu, all, topk - 1);
+      if (lane == 0) lam_s = kth != 0ull ? order_bits_to_float((uint32_t)(kth >> 32)) : -INFINITY;
+    }
+  }
+  __syncthreads();
+  float lam_star = lam_s;
+#pragma unroll
+  for (int k = 0; k < kMergeWarps; ++k) lam_star = fmaxf(lam_star, red[k]);
+  __syncthreads();  // lam_s is written again below
   // ---- lambda over the entries (at or above lam_star) of the ranges that can
-  // hold them: lanes test 32 ranges at once, then the warp walks the hits
+  // hold them: the entries of the listed ranges, one per thread
   unsigned long long lst = 0ull;
-  for (int sp0 = wib * 32; sp0 < n_split; sp0 += kMergeWarps * 32) {
-    unsigned hits = __ballot_sync(0xFFFFFFFFu, sp0 + lane < n_split && rs[sp0 + lane].y >= lam_star);
-    while (hits) {
-      const int sp = sp0 + __ffs(hits) - 1;
-      hits &= hits - 1;
-      const int n = rn[sp];
-      for (int j0 = 0; j0 < n; j0 += 32) {
-        const int j = j0 + lane;
-        unsigned long long key = 0ull;
-        if (j < n) {
+  {
+    const int nh = list_ranges(1, lam_star);
+    for (int base = wib * 32; base < nh * kbuf; base += kMergeWarps * 32) {
+      const int i = base + lane;
+      unsigned long long key = 0ull;
+      if (i < nh * kbuf) {
+        const int sp = hit[i / kbuf], j = i % kbuf;
+        if (j < rn[sp]) {
           const float l = cand_l[(cbase + sp) * kbuf + j];
           if (l >= lam_star) key = ((unsigned long long)order_bits(l) << 32) | (uint32_t)(sp * kbuf + j);
         }
-        warp_topk_offer(lst, key, topk, lane);
       }
+      warp_topk_offer(lst, key, topk, lane);
     }
   }
   {
@@ -838,16 +851,14 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
   // ---- the candidates: entries with upper bound at or above lambda, listed
   // (past the list's capacity they are scored here, one per lane)
   unsigned long long fin = 0ull;
-  for (int sp0 = wib * 32; sp0 < n_split; sp0 += kMergeWarps * 32) {
-    unsigned hits = __ballot_sync(0xFFFFFFFFu, sp0 + lane < n_split && rs[sp0 + lane].z >= lam);
-    while (hits) {
-      const int sp = sp0 + __ffs(hits) - 1;
-      hits &= hits - 1;
-      const int n = rn[sp];
-      for (int j0 = 0; j0 < n; j0 += 32) {
-        const int j = j0 + lane;
-        unsigned long long key = 0ull;
-        if (j < n && cand_u[(cbase + sp) * kbuf + j] >= lam) {
+  {
+    const int nh = list_ranges(2, lam);
+    for (int base = wib * 32; base < nh * kbuf; base += kMergeWarps * 32) {
+      const int i = base + lane;
+      unsigned long long key = 0ull;
+      if (i < nh * kbuf) {
+        const int sp = hit[i / kbuf], j = i % kbuf;
+        if (j < rn[sp] && cand_u[(cbase + sp) * kbuf + j] >= lam) {
           const int c = cand_c[(cbase + sp) * kbuf + j];
           const int pos = atomicAdd(&n_cand, 1);
           if (pos < kMergeCand)
@@ -855,8 +866,8 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
           else
             key = rank_key(exact_dot<D>(qs, krow(c)) * scale_sel, (uint32_t)c);
         }
-        warp_topk_offer(fin, key, topk, lane);
       }
+      warp_topk_offer(fin, key, topk, lane);
     }
   }
   __syncthreads();
@@ -866,9 +877,11 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
 #pragma unroll
     for (int e = 0; e < D; ++e) qr[e] = qs[e];
     const int nlist = min(n_cand, kMergeCand);
-    for (int base = wib * 32; base < nlist; base += kMergeWarps * 32) {
+    // each warp rescores an equal share (up to 32 rows at a time)
+    const int per = min(32, (nlist + kMergeWarps - 1) / kMergeWarps);
+    for (int base = wib * per; base < nlist; base += kMergeWarps * per) {
       const int i = base + lane;
-      const int c = i < nlist ? cands[i] : -1;
+      const int c = (lane < per && i < nlist) ? cands[i] : -1;
       stage_kbar_rows<D>(stage, kbar32 + (long long)g * D, (long long)Hkv * D, c, lane);
       const unsigned long long key =
           c >= 0 ? rank_key(staged_dot<D>(qr, stage, lane) * scale_sel, (uint32_t)c) : 0ull;

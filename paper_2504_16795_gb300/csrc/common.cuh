@@ -258,6 +258,23 @@ struct DecodeDims {
   bool softmax1, stick;  // variants as in Dims
   long long cap;         // chunks the memory and its index are laid out for (>= Nc)
 };
+// Launch `kernel` as a programmatic dependent of the previous kernel in `st`
+// (it must call tc::griddep_wait before reading that kernel's results).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                             Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
 size_t decode_workspace(const DecodeDims& D);
 // True when a kernel of the current device may read p at that address: device or
 // managed memory, or page-locked host memory mapped at the same address (a decode
@@ -268,8 +285,12 @@ cudaError_t launch_decode(const DecodeDims& D, const void* q, const void* K, con
 // Token-level attention over the selected chunks and the weighted sum (the last two decode steps);
 // scratch: decode_attend_scratch(D) bytes, 256-byte aligned (partials, then one counter per row).
 size_t decode_attend_scratch(const DecodeDims& D);
+unsigned* decode_attend_counters(const DecodeDims& D, void* scratch);
+// counters_zeroed: the kernel before has zeroed the per-row counters (no memset);
+// dependent: launched as a programmatic dependent of that kernel.
 cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void* K, const void* V,
-                                 const int32_t* idx, const float* w, void* O, void* scratch, cudaStream_t st);
+                                 const int32_t* idx, const float* w, void* O, void* scratch, cudaStream_t st,
+                                 bool counters_zeroed = false, bool dependent = false);
 // Decode over a memory index (bf16 summaries, norms): tensor-core scan with exact rescoring (topk <= 16).
 bool decode_index_applies(const DecodeDims& D);  // topk <= 16: the memory has an index
 bool decode_tc_applies(const DecodeDims& D);     // ... and at least one chunk

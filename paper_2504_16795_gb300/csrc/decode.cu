@@ -15,6 +15,7 @@
 //      group's heads.
 //   5. O = sum_j w_j O_j.
 #include "score_tile.cuh"
+#include "tc.cuh"
 
 namespace hsa {
 namespace {
@@ -167,6 +168,7 @@ __global__ void __launch_bounds__(kThreads) dec_attend_kernel(
   const int b = bg / Hkv, g = bg % Hkv;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   float* out = Opart + (long long)slot * G * D;
+  tc::griddep_wait();  // the selection (idx, w) and the zeroed counters
   const int c = idx[slot];
   if (c < 0) {
     for (int u = tid; u < G * D; u += kThreads) out[u] = 0.f;
@@ -339,31 +341,47 @@ size_t decode_attend_scratch(const DecodeDims& D) {
   return align256(sizeof(float) * rows * D.topk * D.G * D.d) + align256(sizeof(unsigned) * rows);
 }
 
+unsigned* decode_attend_counters(const DecodeDims& D, void* scratch) {
+  const size_t rows = (size_t)D.Bq * D.Hkv;
+  return (unsigned*)((char*)scratch + align256(sizeof(float) * rows * D.topk * D.G * D.d));
+}
+
+namespace {
+template <int DD>
+cudaError_t run_attend(const DecodeDims& D, const void* q, const void* K, const void* V, const int32_t* idx,
+                   const float* w, void* O, float* opart, unsigned* counters, cudaStream_t st, bool dependent) {
+  const int rows = D.Bq * D.Hkv;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(dec_attend_kernel<DD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)sizeof(AttSmem<DD>))) != cudaSuccess)
+    return e;
+  const float scale = D.scale_attn;
+  const int sm1 = D.softmax1 ? 1 : 0;
+  if (dependent)
+    e = launch_dependent(dec_attend_kernel<DD>, dim3((unsigned)(rows * D.topk)), dim3(kThreads), sizeof(AttSmem<DD>),
+                         st, (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, w, (uint16_t*)O,
+                         counters, D.Hq, D.Hkv, D.G, D.topk, scale, sm1);
+  else
+    dec_attend_kernel<DD><<<rows * D.topk, kThreads, sizeof(AttSmem<DD>), st>>>(
+        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, w, (uint16_t*)O, counters, D.Hq,
+        D.Hkv, D.G, D.topk, scale, sm1);
+  note_launches(1);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+}  // namespace
+
 cudaError_t launch_decode_attend(const DecodeDims& D, const void* q, const void* K, const void* V,
-                                 const int32_t* idx, const float* w, void* O, void* scratch, cudaStream_t st) {
+                                 const int32_t* idx, const float* w, void* O, void* scratch, cudaStream_t st,
+                                 bool counters_zeroed, bool dependent) {
   const int rows = D.Bq * D.Hkv;
   float* opart = (float*)scratch;
-  unsigned* counters =
-      (unsigned*)((char*)scratch + align256(sizeof(float) * (size_t)rows * D.topk * D.G * D.d));
-  cudaError_t e = cudaMemsetAsync(counters, 0, sizeof(unsigned) * (size_t)rows, st);
-  if (e != cudaSuccess) return e;
-  if (D.d == 64) {
-    if ((e = cudaFuncSetAttribute(dec_attend_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)sizeof(AttSmem<64>))) != cudaSuccess)
-      return e;
-    dec_attend_kernel<64><<<rows * D.topk, kThreads, sizeof(AttSmem<64>), st>>>(
-        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, w, (uint16_t*)O, counters, D.Hq,
-        D.Hkv, D.G, D.topk, D.scale_attn, D.softmax1 ? 1 : 0);
-  } else {
-    if ((e = cudaFuncSetAttribute(dec_attend_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)sizeof(AttSmem<128>))) != cudaSuccess)
-      return e;
-    dec_attend_kernel<128><<<rows * D.topk, kThreads, sizeof(AttSmem<128>), st>>>(
-        (const uint16_t*)q, (const uint16_t*)K, (const uint16_t*)V, idx, opart, w, (uint16_t*)O, counters, D.Hq,
-        D.Hkv, D.G, D.topk, D.scale_attn, D.softmax1 ? 1 : 0);
+  unsigned* counters = decode_attend_counters(D, scratch);
+  if (!counters_zeroed) {
+    cudaError_t e = cudaMemsetAsync(counters, 0, sizeof(unsigned) * (size_t)rows, st);
+    if (e != cudaSuccess) return e;
   }
-  note_launches(1);
-  return cudaGetLastError();
+  return D.d == 64 ? run_attend<64>(D, q, K, V, idx, w, O, opart, counters, st, dependent)
+                   : run_attend<128>(D, q, K, V, idx, w, O, opart, counters, st, dependent);
 }
 
 bool memory_device_readable(const void* p) {

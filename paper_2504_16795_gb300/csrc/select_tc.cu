@@ -228,6 +228,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
+  tc::griddep_wait();  // decode: the query rows and norms of the kernel before
   const uint32_t tmem = sm.tmem_base;
   const uint32_t abase = smem_u32(sm.A), ubase = smem_u32(sm.B);
   constexpr uint32_t kStageBytes = kCt * D * 2;
@@ -748,7 +749,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
     const int32_t* __restrict__ cand_n, const float* __restrict__ cand_d, const float4* __restrict__ cand_s, int kbuf,
     const float* __restrict__ qh32, const float* __restrict__ kbar32, int32_t* __restrict__ idx,
     float* __restrict__ s_sel, float* __restrict__ w, int Bq, int Hkv, int Nc, int n_split, int range, int topk,
-    float scale_sel, int stick) {
+    float scale_sel, int stick, unsigned* __restrict__ counters) {
   extern __shared__ __align__(16) unsigned char mg_smem[];
   float* stage_all = reinterpret_cast<float*>(mg_smem);  // [warps][32 rows][D]
   float* qs = stage_all + kMergeWarps * 32 * D;           // [D]
@@ -765,7 +766,11 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
   const int b = row / Hkv, g = row % Hkv;
   const long long cbase = ((long long)g * Bq + b) * n_split;
   const uint32_t stage = smem_u32(stage_all + wib * 32 * D);
-  if (threadIdx.x == 0) any_unsure = 0, n_cand = 0;
+  tc::griddep_wait();  // the scan's exported candidates
+  if (threadIdx.x == 0) {
+    any_unsure = 0, n_cand = 0;
+    counters[row] = 0u;  // for the attention kernel that follows (its output sum)
+  }
   for (int e = threadIdx.x; e < D; e += kMergeWarps * 32) qs[e] = qh32[(long long)row * D + e];
   // the ranges' summaries into shared memory, and the largest range lambda
   float ls = -INFINITY;
@@ -1157,22 +1162,27 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
   if ((e = cudaFuncSetAttribute(sel_tc_kernel<DD, KT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)smem)) != cudaSuccess)
     return e;
-  sel_tc_kernel<DD, KT, true><<<dim3((unsigned)lo.n_split, (unsigned)Dm.Hkv, (unsigned)lo.n_qt), kThreads, smem, st>>>(
-      a, tq, tk, unused);
+  // the scan, the merge and the attention each start as programmatic dependents
+  // of the kernel before (their setup overlaps its tail)
+  e = launch_dependent(sel_tc_kernel<DD, KT, true>, dim3((unsigned)lo.n_split, (unsigned)Dm.Hkv, (unsigned)lo.n_qt),
+                       dim3(kThreads), smem, st, a, tq, tk, unused);
   note_launches(1);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
   const int rows = Dm.Bq * Dm.Hkv;
   if (lo.n_split > kMaxSplit) return cudaErrorNotSupported;
   const size_t mg_smem = ((size_t)kMergeWarps * 32 * DD + DD) * 4 + (size_t)kMergeCand * 4;
   if ((e = cudaFuncSetAttribute(dtc_merge_kernel<DD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mg_smem)) !=
       cudaSuccess)
     return e;
-  dtc_merge_kernel<DD><<<(unsigned)rows, kMergeWarps * 32, mg_smem, st>>>(
-      a.cand_l, a.cand_u, a.cand_c, a.cand_n, a.cand_d, a.cand_s, SelCfg<KT>::kBuf, qh32, kbar32, idx, s_sel, w, Dm.Bq,
-      Dm.Hkv, (int)Dm.Nc, lo.n_split, lo.range, Dm.topk, Dm.scale_sel, Dm.stick ? 1 : 0);
+  unsigned* counters = decode_attend_counters(Dm, base + lo.opart);
+  e = launch_dependent(dtc_merge_kernel<DD>, dim3((unsigned)rows), dim3(kMergeWarps * 32), mg_smem, st,
+                       (const float*)a.cand_l, (const float*)a.cand_u, (const int32_t*)a.cand_c,
+                       (const int32_t*)a.cand_n, (const float*)a.cand_d, (const float4*)a.cand_s,
+                       (int)SelCfg<KT>::kBuf, (const float*)qh32, kbar32, idx, s_sel, w, Dm.Bq, Dm.Hkv, (int)Dm.Nc,
+                       lo.n_split, lo.range, Dm.topk, Dm.scale_sel, Dm.stick ? 1 : 0, counters);
   note_launches(1);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  return launch_decode_attend(Dm, q, K, V, idx, w, O, base + lo.opart, st);
+  if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;
+  return launch_decode_attend(Dm, q, K, V, idx, w, O, base + lo.opart, st, true, true);
 }
 
 }  // namespace

@@ -22,6 +22,13 @@ namespace tc {
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
 enum : unsigned { kStatusTimeout = 1u };
 
+// Programmatic dependent launch: a kernel launched as a dependent of the
+// previous kernel in its stream waits here until that grid has completed and
+// its writes are visible; for a kernel launched the ordinary way it returns at
+// once. The work before it (barrier setup, tensor-memory allocation) overlaps
+// the previous grid's tail.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ unsigned long long globaltimer() {
   unsigned long long t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

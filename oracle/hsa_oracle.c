@@ -26,8 +26,7 @@
  *     selection scores, K̄ and K (Appendix A: the scores receive gradients
  *     because w takes part in the forward pass)
  *
- * Readings where the paper leaves a convention open (each also listed in
- * the design doc):
+ * Readings where the paper leaves a convention open:
  *   - token t (0-indexed) sees only completed chunks before its own: i < t / S;
  *   - fewer than k visible chunks: all are selected, the rest padded with -1;
  *     zero visible chunks give O = 0 and no gradient;

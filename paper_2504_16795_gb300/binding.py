@@ -323,6 +323,8 @@ def select_backward(shape: Shape, q_sel, kbar_sel, idx, ds, offsets, entries, dq
 
 
 def decode(shape: DecodeShape, q, K_mem, V_mem, kbar32, O=None, idx=None, s_sel=None, w=None, ws=None):
+    """hsa_decode. K_mem and V_mem may be CUDA tensors or pinned host tensors (read over the CPU-GPU
+    link); q, kbar32 and the outputs live on the device."""
     _need(q, "q", torch.bfloat16, (shape.Bq, shape.Hq, shape.d))
     dev = q.device
     O = torch.empty_like(q) if O is None else O
@@ -368,6 +370,7 @@ def decode_index(shape: DecodeShape, kbar32, index=None):
 
 def decode_indexed(shape: DecodeShape, q, K_mem, V_mem, kbar32, index, O=None, idx=None, s_sel=None, w=None,
                    ws=None):
+    """hsa_decode_indexed: as decode, scanning the memory index (decode_index) on the tensor cores."""
     _need(q, "q", torch.bfloat16, (shape.Bq, shape.Hq, shape.d))
     dev = q.device
     O = torch.empty_like(q) if O is None else O

@@ -160,3 +160,24 @@ def test_memory_grown_in_host_memory():
         t += n
     check_state(mem, bits)
     check_decode(mem, bits, w)
+
+
+def test_prefill_size_append_equals_building_at_once():
+    # a 2^20-token prefill (the long prefill workload's memory) appended in three
+    # ragged pieces, against pooling and indexing it at once
+    w = synth.WORKLOADS[5].with_(L=1 << 20)
+    T, Hkv, d = w.L, w.Hkv, w.d
+    Kn = synth.device_tensor(w, "K")
+    Vn = synth.device_tensor(w, "V")
+    mem = Memory(Hq=w.Hq, Hkv=Hkv, d=d, topk=w.topk, cap=T // S + 3)
+    for lo, hi in ((0, 12345), (12345, 12345 + 64 * 1000 + 1), (12345 + 64 * 1000 + 1, T)):
+        mem.append(Kn[lo:hi], Vn[lo:hi])
+    torch.cuda.synchronize()
+    hsa.device_check()
+    assert mem.T == T
+    assert torch.equal(mem.K[:T], Kn) and torch.equal(mem.V[:T], Vn)
+    pshape = hsa.Shape(B=1, L=T, Hq=w.Hq, Hkv=Hkv, d=d, topk=w.topk)
+    kb_once, _ = hsa.chunk_pool(pshape, Kn.view(1, T, Hkv, d), want_bf16=False)
+    assert torch.equal(mem.kbar32[:T // S], kb_once.view(T // S, Hkv, d))
+    once = hsa.decode_index(mem.shape(Bq=1), kb_once.view(T // S, Hkv, d).contiguous())
+    assert torch.equal(mem.index, once)

@@ -230,3 +230,15 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     monkeypatch.setattr(b._build, "LIB", str(tmp_path / "absent.so"))
     with pytest.raises(RuntimeError, match="not built"):
         b.load()
+
+
+def test_memory_append_binding_checks_its_rows(lib):
+    torch = pytest.importorskip("torch")
+    shape = hsa.DecodeShape(Bq=1, Hq=8, Hkv=2, d=64, n_chunks=0, capacity_chunks=10)
+    good = torch.zeros((5, 2, 64), dtype=torch.bfloat16)
+    for bad in (torch.zeros((5, 2, 64), dtype=torch.float32), torch.zeros((5, 1, 64), dtype=torch.bfloat16),
+                torch.zeros((5, 2, 128), dtype=torch.bfloat16)[..., ::2]):
+        with pytest.raises(ValueError):
+            hsa.memory_append(shape, 0, bad, good, good, good, good)
+        with pytest.raises(ValueError):
+            hsa.memory_append(shape, 0, good, bad, good, good, good)

@@ -77,6 +77,9 @@ NCU_TRAFFIC = {
 }
 
 
+PEAK_NOTE = "bf16 burst: the timed region lasts well under a second"
+
+
 def log(*a):
     print(*a, file=sys.stderr, flush=True)
 
@@ -136,7 +139,9 @@ def work_model(w):
 
 
 def bound_of(flops, nbytes, pk):
-    t_tensor = flops / (pk["bf16_sus"] * 1e12)
+    # every timed region here lasts well under a second (a few hundred ms of
+    # back-to-back steps), so the tensor roofline is the burst bf16 figure
+    t_tensor = flops / (pk["bf16"] * 1e12)
     t_hbm = nbytes / (pk["hbm"] * 1e9)
     return ("tensor", t_tensor) if t_tensor >= t_hbm else ("hbm", t_hbm)
 
@@ -246,7 +251,7 @@ def run_gpu(args, rank, world, local_rank):
         mark(0)
         hsa.chunk_pool(shape, X["K"], Y["kbar32"], Y["kbar16"])
         mark(1)
-        hsa.select_topk(shape, X["q"], Y["kbar32"], Y["idx"], Y["s_sel"])
+        hsa.select_topk(shape, X["q"], Y["kbar32"], Y["idx"], Y["s_sel"], ws=wss.select)
         mark(2)
         hsa.build_index(shape, Y["idx"], Y["offsets"], Y["entries"], ws=wss.index)
         mark(3)
@@ -298,7 +303,7 @@ def run_gpu(args, rank, world, local_rank):
         bound, t_min = bound_of(m["flops"], m["bytes"], pk)
         sec = per_call[c] / 1e3
         if bound == "tensor":
-            ach, peak, unit = m["flops"] / sec / 1e12, pk["bf16_sus"], "TFLOP/s"
+            ach, peak, unit = m["flops"] / sec / 1e12, pk["bf16"], "TFLOP/s"
         else:
             ach, peak, unit = m["bytes"] / sec / 1e9, pk["hbm"], "GB/s"
         kernels[c] = {"ms": round(per_call[c], 4), "bound": bound, "achieved": round(ach, 2), "peak": peak,
@@ -314,7 +319,7 @@ def run_gpu(args, rank, world, local_rank):
         traffic = tr["bytes_per_launch"]
     roof = {k: kernels[dom][k] for k in ("bound", "achieved", "peak", "unit", "frac")}
     roof.update({"kernel": dom, "traffic": traffic,
-                 "peak_source": f"{pk['source']} ({'bf16 sustained' if roof['bound'] == 'tensor' else 'hbm copy'})"})
+                 "peak_source": f"{pk['source']} ({PEAK_NOTE if roof['bound'] == 'tensor' else 'hbm copy'})"})
 
     variants = None if args.no_variants else run_variants(args, dev, pk, hsa, w, X, Y, barrier, model)
     small = None if args.no_variants else run_small_configs(args, dev, pk, hsa)
@@ -401,8 +406,13 @@ def run_gpu(args, rank, world, local_rank):
         decode = run_decode(args, dev, world, pk, barrier, max_over_ranks, hsa)
         decode["append"] = run_memory_append(args, dev, pk, barrier, max_over_ranks, hsa)
 
+    prefill_1m = None
+    if not args.no_prefill_1m:
+        prefill_1m = run_prefill_1m(args, dev, pk, hsa, barrier, max_over_ranks)
+
     return dict(value=value, ms_step=ms_step, kernels=kernels, roofline=roof, e2e=e2e, clocks=clocks,
-                launches=launches, decode=decode, wall_ms_step=wall / K * 1e3, variants=variants, small=small)
+                launches=launches, decode=decode, wall_ms_step=wall / K * 1e3, variants=variants, small=small,
+                prefill_1m=prefill_1m)
 
 
 def run_variants(args, dev, pk, hsa, w, X, Y, barrier, model):
@@ -423,7 +433,7 @@ def run_variants(args, dev, pk, hsa, w, X, Y, barrier, model):
         return e0.elapsed_time(e1) / n
 
     def frac(call, ms):
-        return round(model[call]["flops"] / (ms / 1e3) / 1e12 / pk["bf16_sus"], 4)
+        return round(model[call]["flops"] / (ms / 1e3) / 1e12 / pk["bf16"], 4)
 
     n = max(args.steps, 5)
     out = {}
@@ -630,6 +640,102 @@ def run_small_configs(args, dev, pk, hsa):
     return out
 
 
+def needle_recall(w, idx):
+    """Needle queries of the 2^20-token workload: a needle query selects only needle chunks when at least k
+    of them are visible, else every visible one. Returns (queries meeting it, needle queries)."""
+    needles = np.sort(synth.needle_chunk_ids(w))
+    toks = synth.needle_query_tokens(w)
+    is_needle = np.zeros(w.Nc + 1, bool)
+    is_needle[needles] = True
+    nvis = np.searchsorted(needles, toks // w.S)
+    sel = idx[toks]
+    picked = np.where(sel >= 0, is_needle[np.clip(sel, 0, None)], False).sum(axis=1)
+    return int((picked == np.minimum(nvis, w.topk)).sum()), int(toks.size)
+
+
+def run_prefill_1m(args, dev, pk, hsa, barrier, max_over_ranks):
+    """The 2^20-token prefill (forward only: pool -> select -> index -> forward), where selection is the
+    quadratic, tensor-bound step. Per-call CUDA events on the launching stream; per-call rooflines."""
+    import torch
+
+    w = rank_shard(synth.WORKLOADS[4], getattr(args, "rank", 0))
+    shape = hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk)
+    log(f"generating the {w.L}-token prefill inputs")
+    X = {n: synth.device_tensor(w, n, dev) for n in ("q", "K", "V")}
+    f32, i32 = torch.float32, torch.int32
+    sel = (w.B, w.L, w.Hkv, w.topk)
+
+    def ws(op):
+        n = hsa.workspace_size(op, shape)
+        return torch.empty(n, dtype=torch.uint8, device=dev) if n else None
+
+    wsel, widx, wfwd = ws(hsa.HSA_OP_SELECT), ws(hsa.HSA_OP_INDEX), ws(hsa.HSA_OP_FORWARD)
+    Y = dict(kbar32=torch.empty((w.B, w.Nc, w.Hkv, w.d), dtype=f32, device=dev),
+             kbar16=torch.empty((w.B, w.Nc, w.Hkv, w.d), dtype=torch.bfloat16, device=dev),
+             idx=torch.empty(sel, dtype=i32, device=dev), s_sel=torch.empty(sel, dtype=f32, device=dev),
+             offsets=torch.empty(w.B * w.Hkv * w.Nc + 1, dtype=i32, device=dev),
+             entries=torch.empty(w.B * w.L * w.Hkv * w.topk, dtype=i32, device=dev),
+             O=torch.empty_like(X["q"]), w=torch.empty(sel, dtype=f32, device=dev))
+    calls = ["hsa_chunk_pool", "hsa_select_topk", "hsa_build_index", "hsa_forward"]
+
+    def step(ev=None):
+        def mark(i):
+            if ev is not None:
+                ev[i].record()
+        mark(0)
+        hsa.chunk_pool(shape, X["K"], Y["kbar32"], Y["kbar16"])
+        mark(1)
+        hsa.select_topk(shape, X["q"], Y["kbar32"], Y["idx"], Y["s_sel"], ws=wsel)
+        mark(2)
+        hsa.build_index(shape, Y["idx"], Y["offsets"], Y["entries"], ws=widx)
+        mark(3)
+        hsa.forward(shape, X["q"], X["K"], X["V"], Y["idx"], Y["s_sel"], Y["offsets"], Y["entries"], Y["O"], Y["w"],
+                    ws=wfwd)
+        mark(4)
+
+    for _ in range(max(3, min(args.warmup, 5))):
+        step()
+    barrier()
+    K = max(3, min(args.steps, 10))
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    with ClockSampler(dev.index or 0) as clk:
+        barrier()
+        for i in range(K):
+            step(evs[i])
+        barrier()
+    clocks = clk.summary()
+    ms_total = max_over_ranks(sum(evs[i][0].elapsed_time(evs[i][4]) for i in range(K)))
+    per_call = {c: statistics.mean(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K))
+                for j, c in enumerate(calls)}
+    ms_step = ms_total / K
+    log(f"prefill-1m: {ms_step:.3f} ms/step, per call (ms): " + ", ".join(f"{c} {v:.3f}" for c, v in per_call.items()))
+    model = work_model(w)
+    kernels = {}
+    for c in calls:
+        m = model[c]
+        bound, t_min = bound_of(m["flops"], m["bytes"], pk)
+        sec = per_call[c] / 1e3
+        if bound == "tensor":
+            ach, peak, unit = m["flops"] / sec / 1e12, pk["bf16"], "TFLOP/s"
+        else:
+            ach, peak, unit = m["bytes"] / sec / 1e9, pk["hbm"], "GB/s"
+        kernels[c] = {"ms": round(per_call[c], 4), "bound": bound, "achieved": round(ach, 2), "peak": peak,
+                      "unit": unit, "frac": round(ach / peak, 4), "algorithmic_flops": m["flops"],
+                      "algorithmic_bytes": m["bytes"], "roofline_ms": round(t_min * 1e3, 4)}
+        if "gathered" in m:
+            kernels[c]["gathered_bytes"] = m["gathered"]
+            kernels[c]["gathered_gbs"] = round(m["gathered"] / sec / 1e9, 1)
+            kernels[c]["gathered_frac_of_hbm"] = round(m["gathered"] / sec / 1e9 / pk["hbm"], 4)
+    ok, n_needle = needle_recall(w, Y["idx"][0, :, 0].cpu().numpy())
+    del X, Y, wsel, widx, wfwd
+    torch.cuda.empty_cache()
+    return {"workload": f"{w.name} forward only: B={w.B} L={w.L} S={w.S} Hq={w.Hq} Hkv={w.Hkv} d={w.d} k={w.topk}, "
+                        f"{w.needle_chunks} needle chunks, 1/{w.needle_query_every} of the queries carry the needle",
+            "steps": K, "ms_per_step": round(ms_step, 4), "value": w.B * w.L / (ms_step / 1e3), "unit": "tokens/s",
+            "kernels": kernels, "needle_queries_ok": f"{ok}/{n_needle}", "clocks": clocks,
+            "peak_note": PEAK_NOTE}
+
+
 def mem_available_bytes():
     try:
         with open("/proc/meminfo") as f:
@@ -742,6 +848,80 @@ def cpu_baseline(target_s=15.0):
                        f"pro rata; {sec2:.1f} s of CPU time")}
 
 
+def cpu_baseline_prefill_1m(target_s=12.0):
+    """The oracle's select + forward on a seeded sample of rows of the 2^20-token workload (the pooling of
+    the whole K timed in full), extrapolated to all rows: forward-only tokens/s. Rows are independent, so
+    the per-row cost scales; the sample is drawn uniformly over the sequence."""
+    import oracle
+
+    oracle.build()
+    w = synth.WORKLOADS[4]
+    K = synth.bf16_to_f64(synth.host_tensor(w, "K", (0, 0, 0, 0), w.dims("K")))
+    V = synth.bf16_to_f64(synth.host_tensor(w, "V", (0, 0, 0, 0), w.dims("V")))
+    t0 = time.perf_counter()
+    kbar32 = oracle.pool(K, w.S, f32=True)
+    t_pool = time.perf_counter() - t0
+    q = np.zeros((1, w.L, w.Hq, w.d))  # only the sampled rows are written (and read by the oracle)
+    rng = np.random.default_rng(5004)
+    done = np.zeros(w.L, bool)
+
+    def rows_sec(n):
+        toks = np.sort(rng.choice(np.nonzero(~done)[0], n, replace=False))
+        done[toks] = True
+        for t in toks:
+            q[0, t] = synth.bf16_to_f64(synth.host_tensor(w, "q", (0, t, 0, 0), (1, t + 1, w.Hq, w.d)))[0, 0]
+        mask = np.zeros((1, w.L), np.uint8)
+        mask[0, toks] = 1
+        t1 = time.perf_counter()
+        idx, s_sel, _ = oracle.select(q, kbar32, w.S, w.topk, f32=True, token_mask=mask)
+        oracle.forward(q, K, V, idx, s_sel, w.S, token_mask=mask)
+        return time.perf_counter() - t1
+
+    n0 = 64
+    sec0 = rows_sec(n0)
+    n1 = int(min(8192, max(n0, n0 * target_s / max(sec0, 1e-3))))
+    sec1 = rows_sec(n1)
+    per_row = sec1 / n1
+    total = t_pool + per_row * w.L
+    return {"value": w.L / total, "unit": "tokens/s", "cores": oracle.threads(), "kind": "oracle",
+            "sample": (f"select + forward of {n1} rows drawn uniformly from the 2^20 tokens ({sec1:.1f} s), "
+                       f"extrapolated to all rows; pooling of the whole K timed in full ({t_pool:.1f} s)"),
+            "extrapolated": True}
+
+
+def cpu_baseline_decode(target_s=8.0):
+    """The oracle's decode call (score every chunk summary, top-k, attention over the k chunks) for the 64
+    queries of the decode workload, on a prefix of its memory; the scoring scales with the number of chunks,
+    so its time is extrapolated to the full 2^20 chunks. As on the GPU, pooling the memory is not part of a
+    call. Returns queries/s."""
+    import oracle
+
+    oracle.build()
+    w = synth.WORKLOADS[5]
+    T = 1 << 20
+    wp = w.with_(L=T)
+    K = synth.bf16_to_f64(synth.host_tensor(wp, "K", (0, 0, 0, 0), (1, T, w.Hkv, w.d)))
+    V = synth.bf16_to_f64(synth.host_tensor(wp, "V", (0, 0, 0, 0), (1, T, w.Hkv, w.d)))
+    kb = oracle.pool(K, w.S, f32=True)[0]
+    q = synth.bf16_to_f64(synth.host_tensor(w, "q", (0, 0, 0, 0), w.dims("q")))[0]
+    reps, t_sel = 0, 0.0
+    while t_sel < target_s and reps < 1000:
+        t0 = time.perf_counter()
+        idx, s_sel, _ = oracle.decode_select(q, kb, w.topk, f32=True)
+        t_sel += time.perf_counter() - t0
+        reps += 1
+    Ks, Vs = oracle.gather_chunks(K[0], idx, w.S), oracle.gather_chunks(V[0], idx, w.S)
+    t0 = time.perf_counter()
+    oracle.decode_attend(q, Ks, Vs, idx, s_sel)
+    t_att = time.perf_counter() - t0
+    per_call = t_sel / reps * (w.Nc / (T // w.S)) + t_att
+    return {"value": w.Bq / per_call, "unit": "queries/s", "cores": oracle.threads(), "kind": "oracle",
+            "sample": (f"{reps} decode scoring passes of the {w.Bq} queries over a {T}-token prefix of the memory "
+                       f"({T // w.S} chunks, {t_sel:.1f} s), scaled to {w.Nc} chunks, plus one attention over "
+                       f"the {w.topk} selected chunks"),
+            "extrapolated": True}
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return
@@ -787,6 +967,7 @@ def main():
     ap.add_argument("--no-variants", action="store_true", help="skip the variant and shared-selection timings")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-prefill-1m", action="store_true", help="skip the 2^20-token forward-only prefill")
     ap.add_argument("--workload", type=int, default=3, help="prefill workload number (3 is the headline)")
     ap.add_argument("--batch", type=int, default=0, help="override the workload's batch (profiling)")
     ap.add_argument("--decode-tokens", type=int, default=None,
@@ -827,12 +1008,19 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         log("timing the CPU oracle baseline")
         cpu = cpu_baseline()
+        if r["decode"] is not None:
+            log("timing the CPU oracle decode baseline")
+            r["decode"]["cpu_baseline"] = cpu_baseline_decode()
+        if r["prefill_1m"] is not None:
+            log("timing the CPU oracle baseline of the 2^20-token prefill")
+            r["prefill_1m"]["cpu_baseline"] = cpu_baseline_prefill_1m()
     if rank == 0:
         line = {"metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": r["ms_step"], "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_obj(),
                 "roofline": r["roofline"], "cpu_baseline": cpu, "e2e": r["e2e"], "gpu_launches": r["launches"],
                 "clocks": r["clocks"], "kernels": r["kernels"], "decode": r["decode"], "variants": r["variants"], "small_configs": r["small"],
+                "prefill_1m": r["prefill_1m"],
                 "wall_ms_per_step": r["wall_ms_step"]}
         print(json.dumps(line), flush=True)
     if world > 1:

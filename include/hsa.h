@@ -23,7 +23,8 @@
  *   Memory   Every pointer is device memory owned by the caller, 16-byte
  *            aligned. The library never allocates or frees memory and keeps
  *            no state between calls; scratch comes from the caller's
- *            workspace (size from hsa_workspace_size). The one exception is
+ *            workspace (size from hsa_workspace_size), which starts with the
+ *            call's status word (see hsa_check). The one exception is
  *            hsa_decode_noalloc, whose scratch is a fixed array inside the
  *            library.
  *   Streams  All work is enqueued on `stream`; nothing synchronises the host.
@@ -110,24 +111,44 @@ int hsa_version(void);
  * diagnostic for launch accounting; counts launches, not their completion). */
 unsigned long long hsa_kernel_launches(void);
 
-/* Device-side health check. Pipelined kernels give up on any internal wait
- * that lasts longer than 2 s (instead of hanging the GPU) and record it in a
- * device status word; this call waits for the device to finish its work,
- * reads and clears that word and returns HSA_ERR_TIMEOUT if a wait gave up
- * since the previous check (the results of that launch are then invalid),
- * HSA_ERR_CUDA if the device reports an error, HSA_OK otherwise.
- * Synchronising: not for use inside a timed region. */
-hsa_status_t hsa_device_check(void);
+/* Bytes of the status header at the start of every workspace (256). */
+size_t hsa_status_bytes(void);
+
+/* Device-side health of the calls that used one workspace. The pipelined
+ * kernels (selection on the tensor cores, forward, backward, the indexed
+ * decode) give up on any internal wait that lasts longer than 2 s, instead
+ * of hanging the GPU, and record it in the status word that heads the
+ * workspace of their call (its first hsa_status_bytes() bytes, counted in
+ * every workspace size). The library keeps no status of its own, so calls
+ * on different workspaces (different streams, different threads) are
+ * checked separately.
+ *   ws, ws_bytes  a workspace given to earlier calls (device memory,
+ *                 16-byte aligned, ws_bytes >= hsa_status_bytes()).
+ * Waits for `stream` (the stream of those calls), reads and clears the
+ * word, and returns HSA_ERR_TIMEOUT if a wait gave up in a call that used
+ * this workspace since the word was last cleared (the results of those
+ * calls are then invalid), HSA_ERR_CUDA if the stream reports an error,
+ * HSA_OK otherwise; HSA_ERR_INVALID_ARG for a bad workspace.
+ * The word is sticky until checked, so a new workspace must start with it
+ * cleared: zero its first hsa_status_bytes() bytes after allocating it (or
+ * call hsa_check once and ignore the result).
+ * Synchronising: not for use inside a timed region or a stream capture. */
+hsa_status_t hsa_check(void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /* Self-test of that bound: launches one block that waits on a barrier nothing
- * ever completes, for at most limit_ns (1 ns to 1 s). The wait gives up, the
- * block returns, and the next hsa_device_check reports HSA_ERR_TIMEOUT once;
- * the context stays usable. No device fault and no hang is involved.
- * Asynchronous on `stream`; HSA_ERR_INVALID_ARG for a limit outside the range. */
-hsa_status_t hsa_selftest_wait_timeout(unsigned long long limit_ns, cudaStream_t stream);
+ * ever completes, for at most limit_ns (1 ns to 1 s). The wait gives up, sets
+ * the status word of `ws` (a workspace of at least hsa_status_bytes() bytes)
+ * and the block returns, so the next hsa_check of that workspace reports
+ * HSA_ERR_TIMEOUT once; the context stays usable. No device fault and no
+ * hang is involved. Asynchronous on `stream`; HSA_ERR_INVALID_ARG for a limit
+ * outside the range, HSA_ERR_WORKSPACE for a bad workspace. */
+hsa_status_t hsa_selftest_wait_timeout(unsigned long long limit_ns, void* ws, size_t ws_bytes,
+                                       cudaStream_t stream);
 
-/* Workspace bytes that `op` needs for `shape` (0 when it needs none). Returns
- * 0 too for an invalid shape; the call itself then reports the error. */
+/* Workspace bytes that `op` needs for `shape`: the status header (see
+ * hsa_check) and the op's scratch. 0 for an empty problem (B or L zero),
+ * whose call launches nothing and takes no workspace, and for an invalid
+ * shape (the call itself then reports the error). */
 size_t hsa_workspace_size(int op, const hsa_shape_t* shape);
 
 /* Workspace bytes of hsa_decode for `shape`. */
@@ -158,9 +179,9 @@ hsa_status_t hsa_chunk_pool(const hsa_shape_t* shape, const void* K, float* kbar
  * matrix is never written to memory. For topk <= 16 the scan runs as bf16
  * tensor-core products whose rounding error is bounded per score; only the
  * chunks the bound cannot rule out are rescored with the fp32 chain, so idx
- * and s_sel are exactly those of the definition above. That path needs
- * workspace HSA_OP_SELECT; for topk > 16 every score is computed with the
- * fp32 chain and the workspace size is 0 (ws may then be NULL).
+ * and s_sel are exactly those of the definition above. Needs workspace
+ * HSA_OP_SELECT (for topk > 16, where every score is computed with the fp32
+ * chain, only its status header).
  */
 hsa_status_t hsa_select_topk(const hsa_shape_t* shape, const void* q, const float* kbar32, int32_t* idx,
                              float* s_sel, void* ws, size_t ws_bytes, cudaStream_t stream);

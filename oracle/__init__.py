@@ -126,7 +126,7 @@ def forward(q, K, V, idx, s_sel, S, scale_attn=None, token_mask=None, inner="sof
     topk = idx.shape[-1]
     if scale_attn is None:
         scale_attn = default_scales(Hq // Hkv, d)[1]
-    O = np.zeros_like(q)
+    O = np.zeros(q.shape)  # zero pages on demand: a masked call writes only its rows
     w = np.zeros((B, L, Hkv, topk))
     m = _mask(token_mask, B, L)
     lib().hsa_oracle_forward(_p(q), _p(K), _p(V), _p(idx), _p(s_sel), B, L, Hq, Hkv, d, S, topk, float(scale_attn),

@@ -27,7 +27,9 @@ from .binding import (  # noqa: F401
     decode_noalloc,
     memory_append,
     decode_workspace_size,
-    device_check,
+    check,
+    new_workspace,
+    status_bytes,
     selftest_wait_timeout,
     forward,
     hsa_backward_path,

@@ -120,10 +120,12 @@ def load():
     L.hsa_version.restype = i
     L.hsa_kernel_launches.restype = ctypes.c_ulonglong
     L.hsa_kernel_launches.argtypes = []
-    L.hsa_device_check.restype = i
-    L.hsa_device_check.argtypes = []
+    L.hsa_status_bytes.restype = sz
+    L.hsa_status_bytes.argtypes = []
+    L.hsa_check.restype = i
+    L.hsa_check.argtypes = [vp, sz, vp]
     L.hsa_selftest_wait_timeout.restype = i
-    L.hsa_selftest_wait_timeout.argtypes = [ctypes.c_ulonglong, vp]
+    L.hsa_selftest_wait_timeout.argtypes = [ctypes.c_ulonglong, vp, sz, vp]
     L.hsa_workspace_size.restype = sz
     L.hsa_workspace_size.argtypes = [i, sp]
     L.hsa_decode_workspace_size.restype = sz
@@ -156,15 +158,24 @@ def kernel_launches() -> int:
     return int(load().hsa_kernel_launches())
 
 
-def device_check() -> None:
-    """Synchronise and raise if a device-side wait gave up since the last check."""
-    _check(load().hsa_device_check(), "hsa_device_check")
+def status_bytes() -> int:
+    """Bytes of the status header that starts every workspace."""
+    return int(load().hsa_status_bytes())
 
 
-def selftest_wait_timeout(limit_ns: int, device=None) -> None:
-    """Launch the bounded-wait self-test (a wait nothing completes, given up after limit_ns)."""
-    dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
-    _check(load().hsa_selftest_wait_timeout(int(limit_ns), _stream(dev)), "hsa_selftest_wait_timeout")
+def check(ws: Optional[torch.Tensor]) -> None:
+    """hsa_check: wait for the current stream of ws's device and raise HsaError if a bounded wait gave up in a
+    call that used this workspace since its last check (the status word is cleared). None: nothing to check."""
+    if ws is None:
+        return
+    _check(load().hsa_check(_ptr(ws), ws.numel() * ws.element_size(), _stream(ws.device)), "hsa_check")
+
+
+def selftest_wait_timeout(limit_ns: int, ws: torch.Tensor) -> None:
+    """Launch the bounded-wait self-test (a wait nothing completes, given up after limit_ns); it sets the
+    status word of workspace ws, which the next check(ws) reports."""
+    _check(load().hsa_selftest_wait_timeout(int(limit_ns), _ptr(ws), ws.numel() * ws.element_size(),
+                                            _stream(ws.device)), "hsa_selftest_wait_timeout")
 
 
 def status_string(status: int) -> str:
@@ -203,12 +214,21 @@ def decode_workspace_size(shape: DecodeShape) -> int:
     return int(load().hsa_decode_workspace_size(ctypes.byref(s)))
 
 
+def new_workspace(nbytes: int, device) -> Optional[torch.Tensor]:
+    """A caller-owned workspace of nbytes (None for 0) with its status header cleared."""
+    if nbytes == 0:
+        return None
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=device)
+    ws[:min(nbytes, status_bytes())].zero_()
+    return ws
+
+
 def _workspace(nbytes: int, device, ws: Optional[torch.Tensor]):
     if nbytes == 0:
         return None
     if ws is not None and ws.numel() * ws.element_size() >= nbytes:
         return ws
-    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+    return new_workspace(nbytes, device)
 
 
 def chunk_pool(shape: Shape, K: torch.Tensor, kbar32=None, kbar16=None, want_bf16: bool = True):
@@ -351,8 +371,9 @@ def decode_noalloc(shape: DecodeShape, q, K_mem, V_mem, kbar32, O, idx, s_sel, w
     _need(s_sel, "s_sel", torch.float32, out)
     _need(w, "w", torch.float32, out)
     s = shape.c()
-    _check(load().hsa_decode_noalloc(ctypes.byref(s), _ptr(q), _ptr(K_mem), _ptr(V_mem), _ptr(kbar32), _ptr(O),
-                                     _ptr(idx), _ptr(s_sel), _ptr(w), _stream(q.device)), "hsa_decode_noalloc")
+    with torch.cuda.device(q.device):  # the library looks up its scratch on the current device
+        _check(load().hsa_decode_noalloc(ctypes.byref(s), _ptr(q), _ptr(K_mem), _ptr(V_mem), _ptr(kbar32), _ptr(O),
+                                         _ptr(idx), _ptr(s_sel), _ptr(w), _stream(q.device)), "hsa_decode_noalloc")
     return O, idx, s_sel, w
 
 
@@ -413,6 +434,11 @@ class Workspaces:
         self.index = _workspace(workspace_size(HSA_OP_INDEX, shape), device, None)
         self.forward = _workspace(workspace_size(HSA_OP_FORWARD, shape), device, None)
         self.backward = _workspace(workspace_size(HSA_OP_BACKWARD, shape), device, None)
+
+    def check(self) -> None:
+        """check() every workspace of the set."""
+        for ws in (self.select, self.index, self.forward, self.backward):
+            check(ws)
 
 
 def hsa_forward_path(shape: Shape, q, K, V, wss: Optional[Workspaces] = None):

@@ -66,6 +66,17 @@ hsa_status_t cuda_status(cudaError_t e) { return e == cudaSuccess ? HSA_OK : HSA
     if ((p) == nullptr || !aligned16(p)) return HSA_ERR_INVALID_ARG; \
   } while (0)
 
+using hsa::kStatusBytes;
+
+// A caller workspace is the status header followed by `body` bytes of scratch:
+// checks its size and alignment and returns the two parts.
+hsa_status_t split_ws(void* ws, size_t ws_bytes, size_t body, unsigned** status, void** scratch) {
+  if (ws == nullptr || !aligned16(ws) || ws_bytes < kStatusBytes + body) return HSA_ERR_WORKSPACE;
+  *status = (unsigned*)ws;
+  *scratch = (char*)ws + kStatusBytes;
+  return HSA_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -86,17 +97,26 @@ int hsa_version(void) { return 100; }
 
 unsigned long long hsa_kernel_launches(void) { return hsa::g_launches.load(std::memory_order_relaxed); }
 
-hsa_status_t hsa_device_check(void) {
-  if (cudaDeviceSynchronize() != cudaSuccess) return HSA_ERR_CUDA;
-  const unsigned s1 = hsa::forward_take_status(), s2 = hsa::backward_take_status(),
-                 s3 = hsa::select_take_status(), s4 = hsa::selftest_take_status();
-  if (s1 == ~0u || s2 == ~0u || s3 == ~0u || s4 == ~0u) return HSA_ERR_CUDA;
-  return (s1 | s2 | s3 | s4) ? HSA_ERR_TIMEOUT : HSA_OK;
+hsa_status_t hsa_check(void* ws, size_t ws_bytes, cudaStream_t stream) {
+  if (ws == nullptr || !aligned16(ws) || ws_bytes < kStatusBytes) return HSA_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(stream) != cudaSuccess) return HSA_ERR_CUDA;
+  unsigned v = 0;
+  if (cudaMemcpyAsync(&v, ws, sizeof(v), cudaMemcpyDeviceToHost, stream) != cudaSuccess ||
+      cudaMemsetAsync(ws, 0, sizeof(v), stream) != cudaSuccess || cudaStreamSynchronize(stream) != cudaSuccess)
+    return HSA_ERR_CUDA;
+  return v ? HSA_ERR_TIMEOUT : HSA_OK;
 }
 
-hsa_status_t hsa_selftest_wait_timeout(unsigned long long limit_ns, cudaStream_t stream) {
+size_t hsa_status_bytes(void) { return kStatusBytes; }
+
+hsa_status_t hsa_selftest_wait_timeout(unsigned long long limit_ns, void* ws, size_t ws_bytes,
+                                       cudaStream_t stream) {
   if (limit_ns == 0 || limit_ns > 1000000000ull) return HSA_ERR_INVALID_ARG;
-  return hsa::launch_selftest_wait(limit_ns, stream) == cudaSuccess ? HSA_OK : HSA_ERR_CUDA;
+  unsigned* status = nullptr;
+  void* scratch = nullptr;
+  hsa_status_t st = split_ws(ws, ws_bytes, 0, &status, &scratch);
+  if (st != HSA_OK) return st;
+  return hsa::launch_selftest_wait(limit_ns, status, stream) == cudaSuccess ? HSA_OK : HSA_ERR_CUDA;
 }
 
 size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {
@@ -104,12 +124,12 @@ size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {
   if (resolve(shape, &D) != HSA_OK) return 0;
   if (empty(D)) return 0;
   switch (op) {
-    case HSA_OP_SELECT: return hsa::select_tc_workspace(D);
-    case HSA_OP_INDEX: return hsa::index_workspace(D);
-    case HSA_OP_FORWARD: return hsa::forward_workspace(D);
-    case HSA_OP_BACKWARD: return hsa::backward_workspace(D);
-    case HSA_OP_BACKWARD_ATTENTION: return hsa::backward_attention_workspace(D);
-    case HSA_OP_SELECT_BACKWARD: return hsa::select_backward_workspace(D);
+    case HSA_OP_SELECT: return kStatusBytes + (hsa::select_tc_applies(D) ? hsa::select_tc_workspace(D) : 0);
+    case HSA_OP_INDEX: return kStatusBytes + hsa::index_workspace(D);
+    case HSA_OP_FORWARD: return kStatusBytes + hsa::forward_workspace(D);
+    case HSA_OP_BACKWARD: return kStatusBytes + hsa::backward_workspace(D);
+    case HSA_OP_BACKWARD_ATTENTION: return kStatusBytes + hsa::backward_attention_workspace(D);
+    case HSA_OP_SELECT_BACKWARD: return kStatusBytes + hsa::select_backward_workspace(D);
   }
   return 0;
 }
@@ -136,11 +156,11 @@ hsa_status_t hsa_select_topk(const hsa_shape_t* shape, const void* q, const floa
   HSA_REQUIRE_PTR(idx);
   HSA_REQUIRE_PTR(s_sel);
   if (D.Nc > 0) HSA_REQUIRE_PTR(kbar32);
-  if (hsa::select_tc_applies(D)) {
-    const size_t need = hsa::select_tc_workspace(D);
-    if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
-    return cuda_status(hsa::launch_select_tc(D, q, kbar32, idx, s_sel, ws, stream));
-  }
+  const bool tc = hsa::select_tc_applies(D);
+  void* scratch = nullptr;
+  st = split_ws(ws, ws_bytes, tc ? hsa::select_tc_workspace(D) : 0, &D.status, &scratch);
+  if (st != HSA_OK) return st;
+  if (tc) return cuda_status(hsa::launch_select_tc(D, q, kbar32, idx, s_sel, scratch, stream));
   return cuda_status(hsa::launch_select(D, q, kbar32, idx, s_sel, stream));
 }
 
@@ -153,9 +173,9 @@ hsa_status_t hsa_build_index(const hsa_shape_t* shape, const int32_t* idx, int32
   if (empty(D)) return HSA_OK;
   HSA_REQUIRE_PTR(idx);
   HSA_REQUIRE_PTR(entries);
-  const size_t need = hsa::index_workspace(D);
-  if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
-  return cuda_status(hsa::launch_index(D, idx, offsets, entries, ws, stream));
+  void* scratch = nullptr;
+  if ((st = split_ws(ws, ws_bytes, hsa::index_workspace(D), &D.status, &scratch)) != HSA_OK) return st;
+  return cuda_status(hsa::launch_index(D, idx, offsets, entries, scratch, stream));
 }
 
 hsa_status_t hsa_forward(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
@@ -174,9 +194,9 @@ hsa_status_t hsa_forward(const hsa_shape_t* shape, const void* q, const void* K,
   HSA_REQUIRE_PTR(entries);
   HSA_REQUIRE_PTR(O);
   HSA_REQUIRE_PTR(w);
-  const size_t need = hsa::forward_workspace(D);
-  if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
-  return cuda_status(hsa::launch_forward(D, q, K, V, idx, s_sel, offsets, entries, O, w, ws, stream));
+  void* scratch = nullptr;
+  if ((st = split_ws(ws, ws_bytes, hsa::forward_workspace(D), &D.status, &scratch)) != HSA_OK) return st;
+  return cuda_status(hsa::launch_forward(D, q, K, V, idx, s_sel, offsets, entries, O, w, scratch, stream));
 }
 
 hsa_status_t hsa_backward(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
@@ -200,10 +220,10 @@ hsa_status_t hsa_backward(const hsa_shape_t* shape, const void* q, const void* K
   HSA_REQUIRE_PTR(dq);
   HSA_REQUIRE_PTR(dK);
   HSA_REQUIRE_PTR(dV);
-  const size_t need = hsa::backward_workspace(D);
-  if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  if ((st = split_ws(ws, ws_bytes, hsa::backward_workspace(D), &D.status, &scratch)) != HSA_OK) return st;
   return cuda_status(
-      hsa::launch_backward(D, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq, dK, dV, ws, stream));
+      hsa::launch_backward(D, q, K, V, kbar32, idx, w, O, dO, offsets, entries, dq, dK, dV, scratch, stream));
 }
 
 hsa_status_t hsa_backward_attention(const hsa_shape_t* shape, const void* q, const void* K, const void* V,
@@ -226,10 +246,10 @@ hsa_status_t hsa_backward_attention(const hsa_shape_t* shape, const void* q, con
   HSA_REQUIRE_PTR(dK);
   HSA_REQUIRE_PTR(dV);
   HSA_REQUIRE_PTR(ds_accum);
-  const size_t need = hsa::backward_attention_workspace(D);
-  if (ws_bytes < need || (need > 0 && (ws == nullptr || !aligned16(ws)))) return HSA_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  if ((st = split_ws(ws, ws_bytes, hsa::backward_attention_workspace(D), &D.status, &scratch)) != HSA_OK) return st;
   return cuda_status(hsa::launch_backward_attention(D, q, K, V, idx, w, dO, offsets, entries, dq, dK, dV, ds_accum,
-                                                    ws, stream));
+                                                    scratch, stream));
 }
 
 hsa_status_t hsa_select_backward(const hsa_shape_t* shape, const void* q_sel, const float* kbar_sel,
@@ -247,10 +267,10 @@ hsa_status_t hsa_select_backward(const hsa_shape_t* shape, const void* q_sel, co
   HSA_REQUIRE_PTR(entries);
   HSA_REQUIRE_PTR(dq_sel);
   HSA_REQUIRE_PTR(dK_sel);
-  const size_t need = hsa::select_backward_workspace(D);
-  if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  if ((st = split_ws(ws, ws_bytes, hsa::select_backward_workspace(D), &D.status, &scratch)) != HSA_OK) return st;
   return cuda_status(
-      hsa::launch_select_backward(D, q_sel, kbar_sel, idx, ds, offsets, entries, dq_sel, dK_sel, ws, stream));
+      hsa::launch_select_backward(D, q_sel, kbar_sel, idx, ds, offsets, entries, dq_sel, dK_sel, scratch, stream));
 }
 
 namespace {
@@ -295,7 +315,7 @@ hsa_status_t resolve_decode(const hsa_decode_shape_t* s, hsa::DecodeDims* out) {
 size_t hsa_decode_workspace_size(const hsa_decode_shape_t* shape) {
   hsa::DecodeDims D;
   if (resolve_decode(shape, &D) != HSA_OK || D.Bq == 0) return 0;
-  return hsa::decode_workspace(D);
+  return kStatusBytes + hsa::decode_workspace(D);
 }
 
 hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const void* K_mem, const void* V_mem,
@@ -315,11 +335,11 @@ hsa_status_t hsa_decode(const hsa_decode_shape_t* shape, const void* q, const vo
     HSA_REQUIRE_PTR(V_mem);
     HSA_REQUIRE_PTR(kbar32);
   }
-  const size_t need = hsa::decode_workspace(D);
-  if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  if ((st = split_ws(ws, ws_bytes, hsa::decode_workspace(D), &D.status, &scratch)) != HSA_OK) return st;
   if (D.Nc > 0 && !(hsa::memory_device_readable(K_mem) && hsa::memory_device_readable(V_mem)))
     return HSA_ERR_INVALID_ARG;
-  return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, ws, stream));
+  return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, scratch, stream));
 }
 
 size_t hsa_decode_index_size(const hsa_decode_shape_t* shape) {
@@ -343,7 +363,7 @@ hsa_status_t hsa_decode_index(const hsa_decode_shape_t* shape, const float* kbar
 size_t hsa_decode_indexed_workspace_size(const hsa_decode_shape_t* shape) {
   hsa::DecodeDims D;
   if (resolve_decode(shape, &D) != HSA_OK || D.Bq == 0) return 0;
-  return hsa::decode_tc_applies(D) ? hsa::decode_tc_workspace(D) : hsa::decode_workspace(D);
+  return kStatusBytes + (hsa::decode_tc_applies(D) ? hsa::decode_tc_workspace(D) : hsa::decode_workspace(D));
 }
 
 hsa_status_t hsa_decode_indexed(const hsa_decode_shape_t* shape, const void* q, const void* K_mem, const void* V_mem,
@@ -363,18 +383,17 @@ hsa_status_t hsa_decode_indexed(const hsa_decode_shape_t* shape, const void* q, 
     HSA_REQUIRE_PTR(V_mem);
     HSA_REQUIRE_PTR(kbar32);
   }
+  void* scratch = nullptr;
   if (!hsa::decode_tc_applies(D)) {  // k > 16 or an empty memory: the CUDA-core scan of hsa_decode
-    const size_t need = hsa::decode_workspace(D);
-    if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+    if ((st = split_ws(ws, ws_bytes, hsa::decode_workspace(D), &D.status, &scratch)) != HSA_OK) return st;
     if (D.Nc > 0 && !(hsa::memory_device_readable(K_mem) && hsa::memory_device_readable(V_mem)))
       return HSA_ERR_INVALID_ARG;
-    return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, ws, stream));
+    return cuda_status(hsa::launch_decode(D, q, K_mem, V_mem, kbar32, O, idx, s_sel, w, scratch, stream));
   }
   HSA_REQUIRE_PTR(index);
-  const size_t need = hsa::decode_tc_workspace(D);
-  if (ws_bytes < need || ws == nullptr || !aligned16(ws)) return HSA_ERR_WORKSPACE;
+  if ((st = split_ws(ws, ws_bytes, hsa::decode_tc_workspace(D), &D.status, &scratch)) != HSA_OK) return st;
   if (!(hsa::memory_device_readable(K_mem) && hsa::memory_device_readable(V_mem))) return HSA_ERR_INVALID_ARG;
-  return cuda_status(hsa::launch_decode_tc(D, q, K_mem, V_mem, kbar32, index, O, idx, s_sel, w, ws, stream));
+  return cuda_status(hsa::launch_decode_tc(D, q, K_mem, V_mem, kbar32, index, O, idx, s_sel, w, scratch, stream));
 }
 
 hsa_status_t hsa_memory_append(const hsa_decode_shape_t* shape, long long n_tokens, long long n_new,

@@ -48,8 +48,6 @@ constexpr int kThreads = 512;  // warps 0-3 and 12-15 softmax/gradients, 4-7 epi
 constexpr int kLoaders = 3;
 constexpr int kTmemCols = 512;
 
-__device__ unsigned g_bwd_status;
-
 template <int D>
 struct BwdSmem {
   uint16_t Q[2][kRows * D];       // gathered query rows (grouped K-major SW128, tc::grp_offset)
@@ -106,6 +104,7 @@ struct BwdArgs {
   int dw_mode;    // write dw per slot and leave the selection terms to later passes
                   // (stick-breaking weights, or the attention-only backward)
   float* dw_out;  // [slots] (dw_mode only)
+  unsigned* status;  // the call's status word (a bounded wait that gives up sets it)
 };
 
 // TMEM columns
@@ -146,7 +145,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int slot_div = a.Hkv * a.topk;
   auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
   volatile int* abort_flag = &sm.abort_flag;
-  unsigned* status = &g_bwd_status;
+  unsigned* status = a.status;
 
   if (tid == 0) {
     for (int i = 0; i < 2; ++i) {
@@ -955,6 +954,7 @@ cudaError_t run(const Dims& Dm, BwdMode mode, const void* q, const void* K, cons
     a.softmax1 = Dm.softmax1 ? 1 : 0;
     a.dw_mode = dw_mode ? 1 : 0;
     a.dw_out = dwb;
+    a.status = Dm.status;
     const size_t smem = sizeof(BwdSmem<D>) + 1024;
     if ((e = cudaFuncSetAttribute(bwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
         cudaSuccess)
@@ -1014,13 +1014,6 @@ cudaError_t run_select_backward(const Dims& Dm, const void* q_sel, const float* 
 }
 
 }  // namespace
-
-unsigned backward_take_status() {
-  unsigned v = 0, zero = 0;
-  if (cudaMemcpyFromSymbol(&v, g_bwd_status, sizeof(v)) != cudaSuccess) return ~0u;
-  cudaMemcpyToSymbol(g_bwd_status, &zero, sizeof(zero));
-  return v;
-}
 
 size_t backward_workspace(const Dims& D) { return bwd_layout(D, BwdMode::kFull).total; }
 size_t backward_attention_workspace(const Dims& D) { return bwd_layout(D, BwdMode::kAttention).total; }

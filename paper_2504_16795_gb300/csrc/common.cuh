@@ -32,11 +32,17 @@ __device__ __forceinline__ void block_key(int Nc, int n_bg, int& c, int& bg) {
 }
 constexpr int kWarp = 32;
 
+// Every workspace starts with this header: the status word that the
+// pipelined kernels of a call set when one of their bounded waits gives up
+// (read and cleared by hsa_check). The rest of the workspace follows it.
+constexpr size_t kStatusBytes = 256;
+
 // Resolved shape shared by host launchers.
 struct Dims {
   int B, L, Hq, Hkv, d, S, topk, G, Nc;
   float scale_sel, scale_attn;
   bool softmax1, stick;  // variants: softmax-off-by-one inside chunks, stick-breaking chunk weights
+  unsigned* status = nullptr;  // the call's status word (device memory, the workspace header)
   long long slots() const { return (long long)B * L * Hkv * topk; }
   long long keys() const { return (long long)B * Hkv * Nc; }
 };
@@ -220,7 +226,6 @@ cudaError_t launch_pool(const Dims& D, const void* K, float* kbar32, void* kbar1
 // Tensor-core selection with exact rescoring (topk <= 16); needs select_tc_workspace bytes.
 bool select_tc_applies(const Dims& D);
 size_t select_tc_workspace(const Dims& D);
-unsigned select_take_status();
 cudaError_t launch_select_tc(const Dims& D, const void* q, const float* kbar32, int32_t* idx, float* s_sel, void* ws,
                              cudaStream_t st);
 cudaError_t launch_select(const Dims& D, const void* q, const float* kbar32, int32_t* idx, float* s_sel,
@@ -229,12 +234,10 @@ size_t index_workspace(const Dims& D);
 cudaError_t launch_index(const Dims& D, const int32_t* idx, int32_t* offsets, int32_t* entries, void* ws,
                          cudaStream_t st);
 size_t forward_workspace(const Dims& D);
-unsigned forward_take_status();
 cudaError_t launch_forward(const Dims& D, const void* q, const void* K, const void* V, const int32_t* idx,
                            const float* s_sel, const int32_t* offsets, const int32_t* entries, void* O, float* w,
                            void* ws, cudaStream_t st);
 size_t backward_workspace(const Dims& D);
-unsigned backward_take_status();
 size_t backward_attention_workspace(const Dims& D);
 cudaError_t launch_backward_attention(const Dims& D, const void* q, const void* K, const void* V, const int32_t* idx,
                                       const float* w, const void* dO, const int32_t* offsets,
@@ -244,9 +247,9 @@ size_t select_backward_workspace(const Dims& D);
 cudaError_t launch_select_backward(const Dims& D, const void* q_sel, const float* kbar_sel, const int32_t* idx,
                                    const float* ds, const int32_t* offsets, const int32_t* entries, float* dq_sel,
                                    float* dK_sel, void* ws, cudaStream_t st);
-// Self-test of the bounded waits: one block waits on a barrier nothing arrives at.
-cudaError_t launch_selftest_wait(unsigned long long limit_ns, cudaStream_t st);
-unsigned selftest_take_status();
+// Self-test of the bounded waits: one block waits on a barrier nothing arrives at
+// and records the timeout in `status`.
+cudaError_t launch_selftest_wait(unsigned long long limit_ns, unsigned* status, cudaStream_t st);
 cudaError_t launch_backward(const Dims& D, const void* q, const void* K, const void* V, const float* kbar32,
                             const int32_t* idx, const float* w, const void* O, const void* dO,
                             const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,
@@ -257,6 +260,7 @@ struct DecodeDims {
   float scale_sel, scale_attn;
   bool softmax1, stick;  // variants as in Dims
   long long cap;         // chunks the memory and its index are laid out for (>= Nc)
+  unsigned* status = nullptr;  // as in Dims
 };
 // Launch `kernel` as a programmatic dependent of the previous kernel in `st`
 // (it must call tc::griddep_wait before reading that kernel's results).

@@ -28,8 +28,6 @@ constexpr int kThreads = 384;  // warps 0-3 softmax, 4-7 epilogue, 8, 10, 11 loa
 constexpr int kLoaders = 3;    // a TMA issue costs the issuing warp tens of ns per box: spread the boxes
 constexpr int kTmemCols = 512;
 
-__device__ unsigned g_fwd_status;
-
 template <int D>
 struct FwdSmem {
   uint16_t Q[kQStages][kRows * D];  // gathered query rows, grouped K-major SW128 (tc::grp_offset)
@@ -67,6 +65,7 @@ struct FwdArgs {
   int use_tma;  // G >= 8: each slot's G rows arrive as one swizzled TMA box
   float scale_log2;  // c_att * log2(e)
   int softmax1;      // softmax-off-by-one inside the chunk
+  unsigned* status;  // the call's status word (a bounded wait that gives up sets it)
 };
 
 template <int D>
@@ -89,7 +88,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int slot_div = a.Hkv * a.topk;
   auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
   volatile int* abort_flag = &sm.abort_flag;
-  unsigned* status = &g_fwd_status;
+  unsigned* status = a.status;
 
   if (tid == 0) {
     for (int i = 0; i < 3; ++i) {
@@ -438,6 +437,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     a.Nc = Dm.Nc;
     a.scale_log2 = Dm.scale_attn * 1.4426950408889634f;
     a.softmax1 = Dm.softmax1 ? 1 : 0;
+    a.status = Dm.status;
     const size_t smem = sizeof(FwdSmem<D>) + 1024;
     cudaError_t e = cudaFuncSetAttribute(fwd_chunk_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -461,13 +461,6 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
 }
 
 }  // namespace
-
-unsigned forward_take_status() {
-  unsigned v = 0, zero = 0;
-  if (cudaMemcpyFromSymbol(&v, g_fwd_status, sizeof(v)) != cudaSuccess) return ~0u;
-  cudaMemcpyToSymbol(g_fwd_status, &zero, sizeof(zero));
-  return v;
-}
 
 size_t forward_workspace(const Dims& D) { return (size_t)D.slots() * D.G * D.d * sizeof(uint16_t); }
 

@@ -61,8 +61,6 @@ struct SelCfg {
   static constexpr int kTmemCols = kAcc * kCt;
 };
 
-__device__ unsigned g_sel_status;
-
 // Decode blocks (DEC) keep no exact keys: the merge rescores their candidates.
 template <int D, int KT, bool DEC = false>
 struct SelTcSmem {
@@ -114,6 +112,7 @@ struct SelTcArgs {
   int32_t* cand_n; // [Hkv, Bq, n_split] entry count
   float* cand_d;   // [Hkv, Bq, n_split] largest upper bound the row's buffer dropped (-inf: none)
   float4* cand_s;  // [Hkv, Bq, n_split] (lambda of the range, largest exported lower bound, largest upper bound)
+  unsigned* status;  // the call's status word (a bounded wait that gives up sets it)
 };
 
 // x[c] for a run-time c in [0, 32): a five-level select tree.
@@ -204,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
   };
   auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
   volatile int* abort_flag = &sm.abort_flag;
-  unsigned* status = &g_sel_status;
+  unsigned* status = a.status;
 
   if (tid == 0) {
     tc::mbar_init(bar(BAR_A), 1);
@@ -1006,6 +1005,7 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   if (!tc::make_rows_tmap(&tq, qh16, (unsigned long long)q_rows(Dm), DD, kTok)) return cudaErrorNotSupported;
   if (!tc::make_rows_tmap(&tk, kb16, (unsigned long long)k_rows(Dm), DD, kCt)) return cudaErrorNotSupported;
   SelTcArgs a{};
+  a.status = Dm.status;
   a.qh32t = qh32;
   a.qn = qn;
   a.kbar32 = kbar32;
@@ -1136,6 +1136,7 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
   if (!tc::make_rows_tmap(&tq, qh16, (unsigned long long)qrows, DD, kTok)) return cudaErrorNotSupported;
   if (!tc::make_rows_tmap(&tk, ib + ix.kb16, krows, DD, kCt)) return cudaErrorNotSupported;
   SelTcArgs a{};
+  a.status = Dm.status;
   a.qn = qn;
   a.kbar32 = kbar32;
   a.kn = (const float*)(ib + ix.kn);
@@ -1241,12 +1242,6 @@ bool select_tc_applies(const Dims& D) { return D.topk <= 16 && D.Nc > 0; }
 
 size_t select_tc_workspace(const Dims& D) { return select_tc_applies(D) ? sel_layout(D).total : 0; }
 
-unsigned select_take_status() {
-  unsigned v = 0, zero = 0;
-  if (cudaMemcpyFromSymbol(&v, g_sel_status, sizeof(v)) != cudaSuccess) return ~0u;
-  cudaMemcpyToSymbol(g_sel_status, &zero, sizeof(zero));
-  return v;
-}
 
 cudaError_t launch_select_tc(const Dims& D, const void* q, const float* kbar32, int32_t* idx, float* s_sel, void* ws,
                              cudaStream_t st) {

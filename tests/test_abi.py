@@ -102,7 +102,7 @@ def test_stick_breaking_backward_needs_its_extra_workspace(lib):
     assert stick == base - rows * 4 + 2 * slots * 4 + rows * s.d * 4
     att = hsa.workspace_size(hsa.HSA_OP_BACKWARD_ATTENTION, s)
     assert att == base - rows * 4 + slots * 4  # dq partials and dw
-    assert hsa.workspace_size(hsa.HSA_OP_SELECT_BACKWARD, s) == rows * s.d * 4
+    assert hsa.workspace_size(hsa.HSA_OP_SELECT_BACKWARD, s) == hsa.status_bytes() + rows * s.d * 4
 
 
 def test_null_and_misaligned_pointers_are_rejected(lib):
@@ -217,11 +217,52 @@ def test_workspace_sizes_scale_with_the_problem(lib):
     slots = 2 * 32768 * 4 * 8
     # selection on the tensor cores keeps q̂ (bf16 and fp32) per (b, g, t) row
     assert hsa.workspace_size(hsa.HSA_OP_SELECT, s) >= 2 * 32768 * 4 * 128 * 6
-    assert hsa.workspace_size(hsa.HSA_OP_SELECT, shape(B=2, L=32768, Hq=32, Hkv=4, topk=24)) == 0
-    assert hsa.workspace_size(hsa.HSA_OP_FORWARD, s) == slots * 8 * 128 * 2
+    # the CUDA-core selection (k > 16) needs only the status header
+    assert hsa.workspace_size(hsa.HSA_OP_SELECT, shape(B=2, L=32768, Hq=32, Hkv=4, topk=24)) == hsa.status_bytes()
+    assert hsa.workspace_size(hsa.HSA_OP_FORWARD, s) == hsa.status_bytes() + slots * 8 * 128 * 2
     assert hsa.workspace_size(hsa.HSA_OP_BACKWARD, s) >= slots * 8 * 128 * 2
     assert hsa.workspace_size(hsa.HSA_OP_INDEX, s) >= slots * 16
     assert hsa.workspace_size(hsa.HSA_OP_FORWARD, shape(d=96)) == 0
+
+
+def test_every_workspace_starts_with_the_status_header(lib):
+    assert hsa.status_bytes() == 256
+    s = shape()
+    for op in (hsa.HSA_OP_SELECT, hsa.HSA_OP_INDEX, hsa.HSA_OP_FORWARD, hsa.HSA_OP_BACKWARD,
+               hsa.HSA_OP_BACKWARD_ATTENTION, hsa.HSA_OP_SELECT_BACKWARD):
+        assert hsa.workspace_size(op, s) > hsa.status_bytes(), op
+        assert hsa.workspace_size(op, shape(B=0)) == 0, op  # an empty problem takes none
+    d = hsa.DecodeShape(Bq=4, Hq=8, Hkv=1, d=128, n_chunks=100)
+    assert hsa.decode_workspace_size(d) > hsa.status_bytes()
+    c = d.c()
+    assert lib.hsa_decode_indexed_workspace_size(ctypes.byref(c)) > hsa.status_bytes()
+    # a workspace of the header alone is not enough for a call that needs scratch
+    assert call_forward(lib, s, ws_bytes=hsa.status_bytes()) == WORKSPACE
+
+
+def test_check_and_selftest_validate_their_workspace(lib):
+    vp = ctypes.c_void_p
+    n = hsa.status_bytes()
+    assert lib.hsa_check(vp(0), n, None) == INVALID
+    assert lib.hsa_check(vp(FAKE + 4), n, None) == INVALID
+    assert lib.hsa_check(vp(FAKE), n - 1, None) == INVALID
+    before = lib.hsa_kernel_launches()
+    assert lib.hsa_selftest_wait_timeout(1000, vp(0), n, None) == WORKSPACE
+    assert lib.hsa_selftest_wait_timeout(1000, vp(FAKE), n - 1, None) == WORKSPACE
+    assert lib.hsa_selftest_wait_timeout(0, vp(FAKE), n, None) == INVALID
+    assert lib.hsa_kernel_launches() == before
+
+
+def test_decode_noalloc_checks_the_size_before_the_memory(lib):
+    # an oversized shape is refused for its size even when the memory pointers
+    # are pageable host memory (which a fitting shape would have refused)
+    np = pytest.importorskip("numpy")
+    vp = ctypes.c_void_p
+    host = np.zeros(1 << 16, np.uint8)
+    hp = (host.ctypes.data + 15) // 16 * 16
+    big = hsa.DecodeShape(Bq=1024, Hq=8, Hkv=1, d=128, n_chunks=1 << 20).c()
+    args = [vp(FAKE), vp(hp), vp(hp), vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE)]
+    assert lib.hsa_decode_noalloc(ctypes.byref(big), *args, None) == WORKSPACE
 
 
 def test_missing_library_fails_loudly(monkeypatch, tmp_path):

@@ -54,7 +54,7 @@ def test_prefill_step_replays_bit_exactly(weights):
     for _ in range(3):
         g.replay()
     torch.cuda.synchronize()
-    hsa.device_check()
+    wss.check()
     for a, b in zip(out, eager):
         assert torch.equal(a, b)
 
@@ -73,7 +73,7 @@ def test_decode_chain_replays_bit_exactly():
             torch.empty((w.Bq, w.Hkv, w.topk), dtype=torch.float32, device=q.device),
             torch.empty((w.Bq, w.Hkv, w.topk), dtype=torch.float32, device=q.device)]
     nws = hsa.load().hsa_decode_indexed_workspace_size(__import__("ctypes").byref(ds.c()))
-    ws = torch.empty(int(nws), dtype=torch.uint8, device=q.device)
+    ws = hsa.new_workspace(int(nws), q.device)
 
     def call():
         return hsa.decode_indexed(ds, q, K, V, kb, index, *outs, ws=ws)
@@ -83,6 +83,6 @@ def test_decode_chain_replays_bit_exactly():
     for _ in range(3):
         g.replay()
     torch.cuda.synchronize()
-    hsa.device_check()
+    hsa.check(ws)
     for a, b in zip(out, eager):
         assert torch.equal(a, b)

@@ -69,7 +69,6 @@ def test_two_layers_sharing_one_selection_match_the_oracle(name, weights):
         got.append((O, dq.clone(), dK.clone(), dV.clone()))
     dq_sel, dK_sel = hsa.select_backward(sel, q_sel, kbar_sel, idx, ds, offsets, entries)
     torch.cuda.synchronize()
-    hsa.device_check()
 
     # oracle
     qs, Ks = synth.bf16_to_f64(qs_bits), synth.bf16_to_f64(Ks_bits)
@@ -119,7 +118,6 @@ def test_attention_part_plus_selection_chain_is_the_full_backward(size, weights)
                                                fwd["offsets"], fwd["entries"])
     dqs, dKs = hsa.select_backward(shape, X["q"], fwd["kbar32"], fwd["idx"], ds, fwd["offsets"], fwd["entries"])
     torch.cuda.synchronize()
-    hsa.device_check()
     assert torch.equal(dV, dVa)
     # same mathematics, different rounding: with softmax weights the full backward
     # carries the selection terms through the bf16 dS tile (dS + c_sel ds / S),

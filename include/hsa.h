@@ -145,6 +145,22 @@ hsa_status_t hsa_check(void* ws, size_t ws_bytes, cudaStream_t stream);
 hsa_status_t hsa_selftest_wait_timeout(unsigned long long limit_ns, void* ws, size_t ws_bytes,
                                        cudaStream_t stream);
 
+/* Diagnostic (no counterpart in the paper): the tensor-core score pass of
+ * hsa_select_topk and hsa_decode_indexed on one tile, so that the rounding of
+ * its fp32 accumulation, which the selection certificate bounds (see
+ * hsa_select_topk), can be measured on the device.
+ *   d      64 or 128 (else HSA_ERR_UNSUPPORTED).
+ *   A      [128, d] bf16, row-major (query rows); B [64, d] bf16, row-major
+ *          (chunk summaries); device memory, 16-byte aligned.
+ *   C      [128, 64] fp32, output: C[r][c] = sum_e A[r][e] B[c][e] as the
+ *          selection computes it (the same operand layout and the same
+ *          sequence of bf16 MMAs of K = 16, accumulated in tensor memory).
+ *   ws     a workspace of at least hsa_status_bytes() bytes (its status word
+ *          records a wait that gave up; see hsa_check).
+ * One block; asynchronous on `stream`. */
+hsa_status_t hsa_selftest_score_tile(int d, const void* A, const void* B, float* C, void* ws, size_t ws_bytes,
+                                     cudaStream_t stream);
+
 /* Workspace bytes that `op` needs for `shape`: the status header (see
  * hsa_check) and the op's scratch. 0 for an empty problem (B or L zero),
  * whose call launches nothing and takes no workspace, and for an invalid

@@ -30,6 +30,7 @@ from .binding import (  # noqa: F401
     check,
     new_workspace,
     status_bytes,
+    selftest_score_tile,
     selftest_wait_timeout,
     forward,
     hsa_backward_path,

@@ -126,6 +126,8 @@ def load():
     L.hsa_check.argtypes = [vp, sz, vp]
     L.hsa_selftest_wait_timeout.restype = i
     L.hsa_selftest_wait_timeout.argtypes = [ctypes.c_ulonglong, vp, sz, vp]
+    L.hsa_selftest_score_tile.restype = i
+    L.hsa_selftest_score_tile.argtypes = [i, vp, vp, vp, vp, sz, vp]
     L.hsa_workspace_size.restype = sz
     L.hsa_workspace_size.argtypes = [i, sp]
     L.hsa_decode_workspace_size.restype = sz
@@ -176,6 +178,19 @@ def selftest_wait_timeout(limit_ns: int, ws: torch.Tensor) -> None:
     status word of workspace ws, which the next check(ws) reports."""
     _check(load().hsa_selftest_wait_timeout(int(limit_ns), _ptr(ws), ws.numel() * ws.element_size(),
                                             _stream(ws.device)), "hsa_selftest_wait_timeout")
+
+
+def selftest_score_tile(A: torch.Tensor, B: torch.Tensor, ws: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """hsa_selftest_score_tile: A [128, d] and B [64, d] bf16 -> C [128, 64] fp32 from the selection's
+    tensor-core score pass (for measuring its accumulation rounding)."""
+    d = int(A.shape[1])
+    _need(A, "A", torch.bfloat16, (128, d))
+    _need(B, "B", torch.bfloat16, (64, d))
+    C = torch.empty((128, 64), dtype=torch.float32, device=A.device)
+    ws = ws if ws is not None else new_workspace(status_bytes(), A.device)
+    _check(load().hsa_selftest_score_tile(d, _ptr(A), _ptr(B), _ptr(C), _ptr(ws), ws.numel(), _stream(A.device)),
+           "hsa_selftest_score_tile")
+    return C
 
 
 def status_string(status: int) -> str:

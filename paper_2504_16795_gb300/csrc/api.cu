@@ -119,6 +119,19 @@ hsa_status_t hsa_selftest_wait_timeout(unsigned long long limit_ns, void* ws, si
   return hsa::launch_selftest_wait(limit_ns, status, stream) == cudaSuccess ? HSA_OK : HSA_ERR_CUDA;
 }
 
+hsa_status_t hsa_selftest_score_tile(int d, const void* A, const void* B, float* C, void* ws, size_t ws_bytes,
+                                     cudaStream_t stream) {
+  if (d != 64 && d != 128) return HSA_ERR_UNSUPPORTED;
+  HSA_REQUIRE_PTR(A);
+  HSA_REQUIRE_PTR(B);
+  HSA_REQUIRE_PTR(C);
+  unsigned* status = nullptr;
+  void* scratch = nullptr;
+  hsa_status_t st = split_ws(ws, ws_bytes, 0, &status, &scratch);
+  if (st != HSA_OK) return st;
+  return cuda_status(hsa::launch_selftest_score_tile(d, A, B, C, status, stream));
+}
+
 size_t hsa_workspace_size(int op, const hsa_shape_t* shape) {
   Dims D;
   if (resolve(shape, &D) != HSA_OK) return 0;

@@ -250,6 +250,9 @@ cudaError_t launch_select_backward(const Dims& D, const void* q_sel, const float
 // Self-test of the bounded waits: one block waits on a barrier nothing arrives at
 // and records the timeout in `status`.
 cudaError_t launch_selftest_wait(unsigned long long limit_ns, unsigned* status, cudaStream_t st);
+// The selection's tensor-core score pass on one 128 x 64 tile (rounding measurements).
+cudaError_t launch_selftest_score_tile(int d, const void* A, const void* B, float* C, unsigned* status,
+                                       cudaStream_t st);
 cudaError_t launch_backward(const Dims& D, const void* q, const void* K, const void* V, const float* kbar32,
                             const int32_t* idx, const float* w, const void* O, const void* dO,
                             const int32_t* offsets, const int32_t* entries, float* dq, float* dK, float* dV,

@@ -659,6 +659,8 @@ def run_prefill_1m(args, dev, pk, hsa, barrier, max_over_ranks):
     import torch
 
     w = rank_shard(synth.WORKLOADS[4], getattr(args, "rank", 0))
+    if getattr(args, "prefill_tokens", None):  # a shorter sequence (profiling captures)
+        w = w.with_(L=args.prefill_tokens)
     shape = hsa.Shape(B=w.B, L=w.L, Hq=w.Hq, Hkv=w.Hkv, d=w.d, S=w.S, topk=w.topk)
     log(f"generating the {w.L}-token prefill inputs")
     X = {n: synth.device_tensor(w, n, dev) for n in ("q", "K", "V")}
@@ -879,7 +881,7 @@ def cpu_baseline_prefill_1m(target_s=12.0):
 
     n0 = 64
     sec0 = rows_sec(n0)
-    n1 = int(min(8192, max(n0, n0 * target_s / max(sec0, 1e-3))))
+    n1 = int(min(32768, max(n0, n0 * target_s / max(sec0, 1e-3))))
     sec1 = rows_sec(n1)
     per_row = sec1 / n1
     total = t_pool + per_row * w.L
@@ -974,6 +976,10 @@ def main():
                     help="decode memory length (default: the 2^26-token workload); for profiling captures")
     ap.add_argument("--decode-only", action="store_true",
                     help="run only the decode sub-benchmark and print its object (profiling)")
+    ap.add_argument("--prefill-1m-only", action="store_true",
+                    help="run only the forward-only 2^20-token prefill and print its object (profiling)")
+    ap.add_argument("--prefill-tokens", type=int, default=None,
+                    help="sequence length of that prefill (default 2^20); for profiling captures")
     args = ap.parse_args()
     select_workload(args.workload, args.batch)
     rank = int(os.environ.get("RANK", "0"))
@@ -995,6 +1001,18 @@ def main():
         d = run_decode(args, dev, 1, peaks(), torch.cuda.synchronize, lambda x: x, hsa)
         d["append"] = run_memory_append(args, dev, peaks(), torch.cuda.synchronize, lambda x: x, hsa)
         print(json.dumps({"decode": d}), flush=True)
+        return
+    if args.prefill_1m_only:
+        import torch
+
+        import paper_2504_16795_gb300 as hsa
+
+        hsa.build()
+        hsa.load()
+        dev = torch.device("cuda", local_rank)
+        torch.cuda.set_device(dev)
+        p = run_prefill_1m(args, dev, peaks(), hsa, torch.cuda.synchronize, lambda x: x)
+        print(json.dumps({"prefill_1m": p}), flush=True)
         return
     import torch.distributed as dist
 

@@ -15,6 +15,13 @@
 // stick-breaking flag, the paper's stick-breaking weights over I' (§3.1.1),
 // slots in order j. The softmax-off-by-one flag (§3.1.2) adds the zero logit
 // to every chunk-local softmax.
+//
+// A chunk that many tokens selected (a chunk every needle query selects has
+// thousands of slots) would make one block run for milliseconds while the
+// other SMs idle. Each slot's result is independent of the others, so a
+// chunk's slot list is cut into segments of at most kSegTiles steps and every
+// segment is its own block (the chunk's K and V are staged by each of them).
+// A one-block pass lists the segments in the chunk order of block_key.
 #include <cstring>
 
 #include "tc.cuh"
@@ -27,6 +34,7 @@ constexpr int kQStages = 3;    // gathered query tiles in flight
 constexpr int kThreads = 384;  // warps 0-3 softmax, 4-7 epilogue, 8, 10, 11 loaders, 9 MMA
 constexpr int kLoaders = 3;    // a TMA issue costs the issuing warp tens of ns per box: spread the boxes
 constexpr int kTmemCols = 512;
+constexpr int kSegTiles = 128;  // longest segment of a chunk's slot list, in 128-row steps
 
 template <int D>
 struct FwdSmem {
@@ -57,7 +65,8 @@ struct FwdArgs {
   const uint16_t* q;
   const uint16_t* K;
   const uint16_t* V;
-  const int32_t* offsets;
+  const int4* segs;  // per block: (key, first entry, end entry, 0)
+  const int* nseg;   // number of segments (blocks past it exit)
   const int32_t* entries;
   uint16_t* Opart;  // [slots, G, D]
   int L, Hq, Hkv, G, log2G, topk, Nc;
@@ -76,12 +85,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int D8 = D / 8;
   constexpr uint32_t kColP = 2 * kChunk + 2 * D;  // tensor memory: S x2 | O' x2 | P x2 (32 columns each)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  int c, bg;
-  block_key(a.Nc, (int)(gridDim.x / (unsigned)a.Nc), c, bg);
-  const int key = bg * a.Nc + c;
+  if ((int)blockIdx.x >= *a.nseg) return;
+  const int4 seg = a.segs[blockIdx.x];
+  const int key = seg.x;
+  const int bg = key / a.Nc, c = key % a.Nc;
   const int b = bg / a.Hkv, g = bg % a.Hkv;
-  const int off = a.offsets[key];
-  const int cnt = a.offsets[key + 1] - off;
+  const int off = seg.y;
+  const int cnt = seg.z - seg.y;
   if (cnt <= 0) return;
   const int epi = kRows >> a.log2G;  // slots per step
   const int niter = (cnt + epi - 1) / epi;
@@ -360,6 +370,65 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// The segments of every chunk's slot list, chunks in the order of block_key
+// (key i of that order = the key block i would take), each list cut into
+// pieces of seg_slots entries. One block of 1024 threads, one scan: thread t
+// takes the run of keys [t * per, (t + 1) * per) of that order, counts their
+// segments, and after a block-wide exclusive scan writes them.
+__device__ __forceinline__ int key_in_order(int i, int Nc, int n_bg) {
+  const int head = min(kHeadChunks, Nc);
+  int c, bg;
+  if (i < head * n_bg) {
+    c = i / n_bg;
+    bg = i % n_bg;
+  } else {
+    const int r = i - head * n_bg, rest = Nc - head;
+    bg = r / rest;
+    c = head + r % rest;
+  }
+  return bg * Nc + c;
+}
+__global__ void __launch_bounds__(1024) fwd_segments_kernel(const int32_t* __restrict__ offsets, int Nc, int n_bg,
+                                                            int seg_slots, int4* __restrict__ segs,
+                                                            int* __restrict__ nseg) {
+  __shared__ int warp_sum[32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int keys = Nc * n_bg;
+  const int per = (keys + 1023) / 1024;
+  const int i0 = min(tid * per, keys), i1 = min(i0 + per, keys);
+  int n = 0;
+  for (int i = i0; i < i1; ++i) {
+    const int key = key_in_order(i, Nc, n_bg);
+    const int len = offsets[key + 1] - offsets[key];
+    n += len > 0 ? (len + seg_slots - 1) / seg_slots : 0;
+  }
+  int x = n;  // inclusive scan within the warp
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sum[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int v = warp_sum[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xFFFFFFFFu, v, o);
+      if (lane >= o) v += y;
+    }
+    warp_sum[lane] = v;  // inclusive over warps
+  }
+  __syncthreads();
+  int pos = (warp > 0 ? warp_sum[warp - 1] : 0) + x - n;
+  for (int i = i0; i < i1; ++i) {
+    const int key = key_in_order(i, Nc, n_bg);
+    const int o0 = offsets[key], o1 = offsets[key + 1];
+    for (int e = o0; e < o1; e += seg_slots) segs[pos++] = make_int4(key, e, min(e + seg_slots, o1), 0);
+  }
+  if (tid == 1023) *nseg = warp_sum[31];
+}
+
 // O_t = sum_j w_j O'_{t,j}; w = softmax over the selected scores or stick-breaking. One warp per (b, t, g).
 template <int D>
 __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict__ s_sel,
@@ -415,17 +484,47 @@ __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict_
   }
 }
 
+inline size_t align256f(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Forward workspace: the bf16 partials [slots, G, d], then the segment list
+// (at most one segment per key plus one per seg_slots entries) and its count.
+struct FwdLayout {
+  size_t segs, nseg, total;
+  long long max_segs;
+};
+FwdLayout fwd_layout(const Dims& D) {
+  FwdLayout lo{};
+  const long long seg_slots = (long long)kSegTiles * (kRows / D.G);
+  lo.max_segs = D.keys() + (D.slots() + seg_slots - 1) / seg_slots;
+  size_t o = align256f((size_t)D.slots() * D.G * D.d * sizeof(uint16_t));
+  lo.segs = o;
+  o = align256f(o + (size_t)lo.max_segs * sizeof(int4));
+  lo.nseg = o;
+  o = align256f(o + sizeof(int));
+  lo.total = o;
+  return lo;
+}
+
 template <int D>
 cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, const int32_t* idx, const float* s_sel,
                 const int32_t* offsets, const int32_t* entries, void* O, float* w, void* ws, cudaStream_t st) {
   const long long keys = Dm.keys();
+  const FwdLayout lo = fwd_layout(Dm);
   uint16_t* Opart = (uint16_t*)ws;
   if (keys > 0) {
+    int4* segs = (int4*)((char*)ws + lo.segs);
+    int* nseg = (int*)((char*)ws + lo.nseg);
+    const int seg_slots = kSegTiles * (kRows / Dm.G);
+    fwd_segments_kernel<<<1, 1024, 0, st>>>(offsets, Dm.Nc, Dm.B * Dm.Hkv, seg_slots, segs, nseg);
+    note_launches(1);
+    cudaError_t e0 = cudaGetLastError();
+    if (e0 != cudaSuccess) return e0;
     FwdArgs a;
     a.q = (const uint16_t*)q;
     a.K = (const uint16_t*)K;
     a.V = (const uint16_t*)V;
-    a.offsets = offsets;
+    a.segs = segs;
+    a.nseg = nseg;
     a.entries = entries;
     a.Opart = Opart;
     a.L = Dm.L;
@@ -449,7 +548,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     if (a.use_tma && !tc::make_group8_tmap(&tq, q, (unsigned long long)a.n_rows, D)) return cudaErrorNotSupported;
     if (a.use_tma && !tc::make_group8_tmap(&to, Opart, (unsigned long long)Dm.slots() * Dm.G, D))
       return cudaErrorNotSupported;
-    fwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq, to);
+    fwd_chunk_kernel<D><<<(unsigned)lo.max_segs, kThreads, smem, st>>>(a, tq, to);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
@@ -462,7 +561,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
 
 }  // namespace
 
-size_t forward_workspace(const Dims& D) { return (size_t)D.slots() * D.G * D.d * sizeof(uint16_t); }
+size_t forward_workspace(const Dims& D) { return fwd_layout(D).total; }
 
 cudaError_t launch_forward(const Dims& D, const void* q, const void* K, const void* V, const int32_t* idx,
                            const float* s_sel, const int32_t* offsets, const int32_t* entries, void* O, float* w,

@@ -219,7 +219,8 @@ def test_workspace_sizes_scale_with_the_problem(lib):
     assert hsa.workspace_size(hsa.HSA_OP_SELECT, s) >= 2 * 32768 * 4 * 128 * 6
     # the CUDA-core selection (k > 16) needs only the status header
     assert hsa.workspace_size(hsa.HSA_OP_SELECT, shape(B=2, L=32768, Hq=32, Hkv=4, topk=24)) == hsa.status_bytes()
-    assert hsa.workspace_size(hsa.HSA_OP_FORWARD, s) == hsa.status_bytes() + slots * 8 * 128 * 2
+    # the forward keeps one bf16 partial per slot and head, and the list of slot-list segments
+    assert hsa.workspace_size(hsa.HSA_OP_FORWARD, s) >= hsa.status_bytes() + slots * 8 * 128 * 2
     assert hsa.workspace_size(hsa.HSA_OP_BACKWARD, s) >= slots * 8 * 128 * 2
     assert hsa.workspace_size(hsa.HSA_OP_INDEX, s) >= slots * 16
     assert hsa.workspace_size(hsa.HSA_OP_FORWARD, shape(d=96)) == 0

@@ -20,14 +20,18 @@
 // (2^-10 |q̂||K̄_i|) that the final rounding by c_sel cannot create a tie.
 //
 // Per block: 128 consecutive tokens of one (b, g) against tiles of 64 chunk
-// summaries, in two passes over the tiles (the MMAs run twice). Thread r of
-// the four scan warps owns token row r (tensor-memory lane r).
-//   Pass 1: per group of columns, (largest bf16 score - the tile's largest
-//   eps) is at most the group's best lower bound; the k-th largest such term,
-//   lam_lo, is a lower bound of lambda (min/max only, no branches).
-//   Pass 2: every chunk whose upper bound reaches lam_lo goes to a per-row
-//   buffer (typically k plus a few); it holds every chunk whose lower bound
-//   reaches lambda, so lambda is the k-th largest lower bound in the buffer.
+// summaries, in one sweep over the tiles plus a second visit of its first few.
+// Thread r of the four scan warps owns token row r (tensor-memory lane r).
+//   Bound: per group of columns, (largest bf16 score - the tile's largest
+//   eps) is at most the group's best lower bound; the k-th largest such term
+//   seen so far is a lower bound of lambda (min/max only, no branches), and
+//   it only grows. Its final value is lam_lo.
+//   Collection: once the bound holds 2k terms, every chunk whose upper bound
+//   reaches the bound so far goes to a per-row buffer; the tiles swept before
+//   that are visited again against lam_lo. The buffer then holds every chunk
+//   whose upper bound reaches lam_lo (plus a few below it, typically k plus a
+//   few in all), so it holds every chunk whose lower bound reaches lambda,
+//   and lambda is the k-th largest lower bound in the buffer.
 // The buffer entries whose upper bound reaches lambda are rescored exactly in
 // fp32 and the top k emitted. A full buffer keeps the entries with the
 // largest upper bounds and remembers the largest upper bound it dropped; a
@@ -56,7 +60,8 @@ template <int KT>
 struct SelCfg {
   static constexpr int kStages = KT <= 8 ? 2 : 4;  // chunk-summary tiles in flight
   static constexpr int kAcc = KT <= 8 ? 2 : 4;     // score accumulators in tensor memory (kCt columns each)
-  static constexpr int kBuf = KT <= 8 ? 24 : 64;   // candidate entries per row (second pass)
+  static constexpr int kBuf = KT <= 8 ? 24 : 64;   // candidate entries per row (per thread)
+  static constexpr int kExport = 2 * kBuf;          // decode: exported entries per row and range (two buffers)
   static constexpr int kBlocksPerSm = KT <= 8 ? 2 : 1;
   static constexpr int kTmemCols = kAcc * kCt;
 };
@@ -76,18 +81,24 @@ struct SelTcSmem {
   // A and B are adjacent: once every MMA is done they hold the rows' fp32 q̂ ([e][row], 128 * D floats)
   uint16_t A[kTok * D];                  // q̂ (bf16) of the block's rows, K-major SW128
   uint16_t B[kStages][kCt * D];          // chunk-summary tiles, K-major SW128
-  float bl[kBuf][kTok];                  // second-pass entries: lower bounds, later exact scores
+  float bl[kBuf][kTok];                  // collected entries: lower bounds, later exact scores
   float bu[kBuf][kTok];                  //   upper bounds
   int bi[kBuf][kTok];                    //   chunk indices
   unsigned long long chosen[DEC ? 1 : KT][kTok];  // the k best exact keys (prefill)
   float knt[kKn][kCt + 4];               // |K̄_i| of a tile, then the tile's max (ring of kKn)
   uint64_t bar[kBars];
+  float xch[DEC ? 2 : 1][DEC ? 4 : 1][kTok];  // decode pairs: bound terms swapped after each tile
+  float xdrop[DEC ? kTok : 1];                 //   and, at the end, the dropped bound
+  int xcnt[DEC ? kTok : 1];                    //   and the entry count
   uint32_t tmem_base;
   int abort_flag;
 };
 // the rescoring stages 32 fp32 K̄ rows per scan warp in A and B
 static_assert(sizeof(SelTcSmem<128, 8>::A) + sizeof(SelTcSmem<128, 8>::B) >= 4 * 32 * 128 * 4, "staging");
 static_assert(sizeof(SelTcSmem<64, 8>::A) + sizeof(SelTcSmem<64, 8>::B) >= 4 * 32 * 64 * 4, "staging");
+// two blocks per SM with K_T = 8 (228 KB of shared memory, 1 KB reserved per block)
+static_assert(2 * (sizeof(SelTcSmem<128, 8>) + 2048) <= 233472, "two prefill blocks per SM");
+static_assert(2 * (sizeof(SelTcSmem<128, 8, true>) + 2048) <= 233472, "two decode blocks per SM");
 
 struct SelTcArgs {
   const float* qh32t;     // [B*Hkv, D, Lp] fp32 q̂, transposed (tokens adjacent)
@@ -106,7 +117,7 @@ struct SelTcArgs {
   // visible); block (split, g, query tile) scans chunks [split*range, +range)
   // and exports, per row, the chunks whose upper bound reaches its own lambda
   int Bq, n_split, range;
-  float* cand_l;   // [Hkv, Bq, n_split, kBuf] lower bounds
+  float* cand_l;   // [Hkv, Bq, n_split, kExport] lower bounds
   float* cand_u;   //                          upper bounds
   int32_t* cand_c; //                          chunk indices
   int32_t* cand_n; // [Hkv, Bq, n_split] entry count
@@ -204,6 +215,21 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
   auto bar = [&](int i) { return smem_u32(&sm.bar[i]); };
   volatile int* abort_flag = &sm.abort_flag;
   unsigned* status = a.status;
+  // The lower bound of lambda is the k-th largest of (max over a group of
+  // columns - the tile's largest eps): each group holds a chunk whose lower
+  // bound is at least its term. Groups of 32 or 8 columns, or single columns
+  // for short rows, keep at least 2k terms per row.
+  const int vis0 = DEC ? vis_max : min(t0 / kChunk, a.Nc);
+  const int gsz = vis0 >= 64 * a.topk ? 32 : (vis0 >= 16 * a.topk ? 8 : 1);
+  // Decode: one sweep over the tiles collects, past the first t_warm tiles
+  // (2k terms), every chunk whose upper bound reaches the bound built so far;
+  // the bound only grows, so this is a superset of the chunks reaching the
+  // final one. The t_warm tiles are then visited again against the final
+  // bound. Prefill rows (longer, k up to 16) collect far more chunks against
+  // the early bound than against the final one, so they sweep twice
+  // (t_warm = ntiles): the first sweep builds the bound, the second collects.
+  const int t_warm = DEC ? min(ntiles, (2 * a.topk * gsz + kCt - 1) / kCt) : ntiles;
+  const int n_iter = ntiles + t_warm;
 
   if (tid == 0) {
     tc::mbar_init(bar(BAR_A), 1);
@@ -240,7 +266,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       for (int kb = 0; kb < D / 64; ++kb)
         tc::tma_load_2d(abase + kb * kTok * 128, &tmap_q, kb * 64, DEC ? (g * a.n_qt + qt) * kTok : bg * a.L + t0,
                         bar(BAR_A));
-      for (int it = 0; it < 2 * ntiles; ++it) {  // two passes over the tiles
+      for (int it = 0; it < n_iter; ++it) {
         const int n = tile_of(it);
         const int s = it % kStages, kq = it % kKn;
         // the tile's chunk norms (the scan of tile it - kKn has released the slot)
@@ -264,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     if (lane == 0 && ntiles > 0) {
       constexpr uint32_t idesc = tc::idesc_bf16(kTok, kCt);
       bool ok = tc::mbar_wait(bar(BAR_A), 0, abort_flag, status);
-      for (int it = 0; ok && it < 2 * ntiles; ++it) {
+      for (int it = 0; ok && it < n_iter; ++it) {
         const int n = tile_of(it);
         const int s = it % kStages, ab = it % kAcc;
         if (!tc::mbar_wait(bar(BAR_FULL + s), (it / kStages) & 1, abort_flag, status)) break;
@@ -284,19 +310,22 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     __syncwarp();
   } else {
     // ---------------------------------------------------------------- scan (thread = token row)
+    // Decode blocks of at most 64 rows scan each row with two threads: the
+    // rows were stored twice, so tensor-memory lanes 64-127 repeat lanes 0-63.
+    // Thread r takes the lower 32 columns of every tile and thread r + 64 the
+    // upper 32; after each tile of the sweep they swap their bound terms
+    // through shared memory (named barrier 1), so both hold the row's bound.
+    // Each keeps its own buffer, and thread r exports both.
+    const bool pair = DEC && a.Bq <= kTok / 2 && gsz >= 8;
     const int r = tid;
-    const int t = t0 + r;
+    const int t = t0 + (pair ? (r & (kTok / 2 - 1)) : r);
     const bool row_ok = DEC ? t < a.Bq : t < a.L;
     const int vis = !row_ok ? 0 : (DEC ? vis_max : min(t / kChunk, a.Nc));
     constexpr int kBuf = Smem::kBuf;
     const long long qrow = DEC ? (long long)t * a.Hkv + g : (long long)bg * a.L + t;
     const float cq = vis > 0 ? kEpsRel * a.qn[qrow] : 0.f;  // eps_i = cq * |K̄_i| + kEpsAbs
-    // First pass: the k-th largest of (max over a group of columns - the
-    // tile's largest eps) is a lower bound of lambda, since each group holds a
-    // chunk whose lower bound is at least its term. Groups of 32 or 8 columns,
-    // or single columns for short rows, keep at least 2k terms per row.
-    const int vis0 = DEC ? vis_max : min(t0 / kChunk, a.Nc);
-    const int gsz = vis0 >= 64 * a.topk ? 32 : (vis0 >= 16 * a.topk ? 8 : 1);
+    const int h_begin = pair ? r / (kTok / 2) : 0, h_end = pair ? h_begin + 1 : kCt / 32;
+    const int nterm = gsz == 8 ? 4 : 1;  // terms per 32 columns (gsz >= 8)
     float bm[KT];  // slots [KT-k, KT): the k largest terms (descending); +inf above
 #pragma unroll
     for (int i = 0; i < KT; ++i) bm[i] = i < KT - a.topk ? INFINITY : -INFINITY;
@@ -308,57 +337,80 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
         bm[i] = hi;
       }
     };
-    float lam_lo = -INFINITY;
-    int cnt = 0;  // second-pass entries
+    float lam_lo = -INFINITY;  // the final bound (second visits)
+    int cnt = 0;  // collected entries
     float u_drop = -INFINITY;  // largest upper bound a full buffer dropped
+    auto scan_barrier = [&]() { asm volatile("barrier.sync 1, 128;" ::: "memory"); };
 
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-    for (int it = 0; it < 2 * ntiles; ++it) {
-      const bool second = it >= ntiles;
+    bool dead = false;  // a wait gave up; in pair mode the warp still meets every barrier
+    for (int it = 0; it < n_iter; ++it) {
+      const bool sweep = it < ntiles;     // first visit: the bound's terms
+      const bool collect = it >= t_warm;  // candidates against the bound so far (final on a second visit)
       const int n = tile_of(it);
-      const int ab = it % kAcc;
+      const int ab = it % kAcc, kq = it % kKn;
       if (it == ntiles) lam_lo = bm[KT - 1];
-      if (!tc::mbar_wait(bar(BAR_ACC_FULL + ab), (it / kAcc) & 1, abort_flag, status)) break;
-      const int kq = it % kKn;
-      if (!tc::mbar_wait(bar(BAR_KN + kq), (it / kKn) & 1, abort_flag, status)) break;
-      tc::fence_after_sync();
+      if (!dead) {
+        const bool ok = tc::mbar_wait(bar(BAR_ACC_FULL + ab), (it / kAcc) & 1, abort_flag, status) &&
+                        tc::mbar_wait(bar(BAR_KN + kq), (it / kKn) & 1, abort_flag, status);
+        dead = !__all_sync(0xFFFFFFFFu, ok);
+      }
+      if (dead && !pair) break;
+      if (!dead) tc::fence_after_sync();
       const float* knt = sm.knt[kq];
-      const float emax = fmaf(cq, knt[kCt], kEpsAbs);  // the tile's largest eps_i
+      const float emax = dead ? 0.f : fmaf(cq, knt[kCt], kEpsAbs);  // the tile's largest eps_i
 #pragma unroll 1
-      for (int h = 0; h < kCt / 32; ++h) {
+      for (int h = h_begin; h < h_end; ++h) {
         float x[32];
-        __syncwarp();
-        tc::tmem_ld32(tmem + lane_base + ab * kCt + h * 32, x);
-        tc::tmem_wait_ld();
+        float tv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};  // this half's terms
         const int c0 = n * kCt + h * 32;
         const int lim = vis - c0;
-        if (lim <= 0) continue;
-        if (!second) {
-          if (lim < 32) {
+        if (!dead) {
+          __syncwarp();
+          tc::tmem_ld32(tmem + lane_base + ab * kCt + h * 32, x);
+          tc::tmem_wait_ld();
+          if (sweep && lim > 0) {
+            if (lim < 32) {
 #pragma unroll
-            for (int c = 0; c < 32; ++c) x[c] = c < lim ? x[c] : -INFINITY;
-          }
-          if (gsz == 1) {
-#pragma unroll
-            for (int c = 0; c < 32; ++c) push(x[c] - emax);
-          } else {
-            float m8[4];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              m8[j] = fmaxf(fmaxf(fmaxf(x[8 * j], x[8 * j + 1]), fmaxf(x[8 * j + 2], x[8 * j + 3])),
-                            fmaxf(fmaxf(x[8 * j + 4], x[8 * j + 5]), fmaxf(x[8 * j + 6], x[8 * j + 7])));
+              for (int c = 0; c < 32; ++c) x[c] = c < lim ? x[c] : -INFINITY;
             }
-            if (gsz == 8) {
+            if (gsz == 1) {
 #pragma unroll
-              for (int j = 0; j < 4; ++j) push(m8[j] - emax);
+              for (int c = 0; c < 32; ++c) push(x[c] - emax);
             } else {
-              push(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])) - emax);
+              float m8[4];
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                m8[j] = fmaxf(fmaxf(fmaxf(x[8 * j], x[8 * j + 1]), fmaxf(x[8 * j + 2], x[8 * j + 3])),
+                              fmaxf(fmaxf(x[8 * j + 4], x[8 * j + 5]), fmaxf(x[8 * j + 6], x[8 * j + 7])));
+              }
+              if (gsz == 8) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) tv[j] = m8[j] - emax;
+              } else {
+                tv[0] = fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])) - emax;
+              }
+#pragma unroll
+              for (int j = 0; j < 4; ++j)
+                if (j < nterm) push(tv[j]);
             }
           }
-        } else {
-          // second pass: every chunk whose upper bound reaches lam_lo
+        }
+        if (pair && sweep) {  // the partner's terms of this tile
+          float(*xo)[kTok] = sm.xch[it & 1];
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (j < nterm) xo[j][r] = tv[j];
+          scan_barrier();
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (j < nterm) push(xo[j][r ^ (kTok / 2)]);
+        }
+        if (!dead && collect && lim > 0) {
+          // every chunk whose upper bound reaches the bound
+          const float thr = sweep ? bm[KT - 1] : lam_lo;
           uint32_t m = 0;
-          const float lo = lam_lo - emax;
+          const float lo = thr - emax;
 #pragma unroll
           for (int c = 0; c < 32; ++c) m |= x[c] >= lo ? (1u << c) : 0u;
           if (lim < 32) m &= (1u << lim) - 1u;
@@ -367,7 +419,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
             m &= m - 1;
             const float xc = pick32(x, c);
             const float e = fmaf(cq, knt[h * 32 + c], kEpsAbs);
-            if (xc + e >= lam_lo) {
+            if (xc + e >= thr) {
               const float lv = xc - e, uv = xc + e;
               int slot = cnt;
               if (cnt < kBuf) {
@@ -395,37 +447,57 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
           }
         }
       }
-      tc::fence_before_sync();
-      tc::mbar_arrive(bar(BAR_ACC_EMPTY + ab));
-      tc::mbar_arrive(bar(BAR_KNE + kq));
+      if (!dead) {
+        tc::fence_before_sync();
+        tc::mbar_arrive(bar(BAR_ACC_EMPTY + ab));
+        tc::mbar_arrive(bar(BAR_KNE + kq));
+      }
     }
     if (ntiles == 0) cnt = 0;
+    int cnt_p = 0;  // pair mode, thread r < 64: the partner's entries
+    if constexpr (DEC) {
+      if (pair) {
+        sm.xcnt[r] = cnt;
+        sm.xdrop[r] = u_drop;
+        scan_barrier();
+        if (r < kTok / 2) {
+          cnt_p = sm.xcnt[r + kTok / 2];
+          u_drop = fmaxf(u_drop, sm.xdrop[r + kTok / 2]);
+        }
+      }
+    }
     // lambda of the kept entries: at most the row's true lambda (a subset's k-th largest)
 #pragma unroll
     for (int i = 0; i < KT; ++i) bm[i] = i < KT - a.topk ? INFINITY : -INFINITY;
     for (int j = 0; j < cnt; ++j) push(sm.bl[j][r]);
+    for (int j = 0; j < cnt_p; ++j) push(sm.bl[j][r + kTok / 2]);
     const float lam_keep = bm[KT - 1];
 
     if constexpr (DEC) {
       // export the entries whose upper bound reaches this range's lambda, and
       // the largest upper bound the buffer dropped (the merge checks it against
       // the lambda of the whole memory)
-      if (row_ok && !*abort_flag) {
+      if (row_ok && !*abort_flag && (!pair || r < kTok / 2)) {
+        constexpr int kExp = SelCfg<KT>::kExport;  // holds both buffers of a pair
         const long long crow = ((long long)g * a.Bq + t) * a.n_split + split;
         int ne = 0;
         float lmax = -INFINITY, umax = -INFINITY;
-        for (int j = 0; j < cnt; ++j) {
-          const float u = sm.bu[j][r];
-          if (u >= lam_keep) {
-            const float l = sm.bl[j][r];
-            a.cand_l[crow * kBuf + ne] = l;
-            a.cand_u[crow * kBuf + ne] = u;
-            a.cand_c[crow * kBuf + ne] = sm.bi[j][r];
-            lmax = fmaxf(lmax, l);
-            umax = fmaxf(umax, u);
-            ++ne;
+        auto take = [&](int col, int n_ent) {
+          for (int j = 0; j < n_ent; ++j) {
+            const float u = sm.bu[j][col];
+            if (u >= lam_keep) {
+              const float l = sm.bl[j][col];
+              a.cand_l[crow * kExp + ne] = l;
+              a.cand_u[crow * kExp + ne] = u;
+              a.cand_c[crow * kExp + ne] = sm.bi[j][col];
+              lmax = fmaxf(lmax, l);
+              umax = fmaxf(umax, u);
+              ++ne;
+            }
           }
-        }
+        };
+        take(r, cnt);
+        take(r + kTok / 2, cnt_p);
         a.cand_n[crow] = ne;
         a.cand_d[crow] = u_drop;
         a.cand_s[crow] = make_float4(lam_keep, lmax, umax, 0.f);
@@ -679,11 +751,14 @@ __global__ void __launch_bounds__(256) dtc_qhat_kernel(const uint16_t* __restric
   const int b = (int)(row % ((long long)n_qt * kTok));
   const bool in = row < rows;
   const bool valid = in && b < Bq;
+  // at most kTok/2 rows: the bf16 rows are stored twice (rows b and b + 64),
+  // so that a selection block scans each row with two threads
+  const int bs = (Bq <= kTok / 2 && b >= kTok / 2) ? b - kTok / 2 : b;
   float acc[8];
 #pragma unroll
   for (int c = 0; c < 8; ++c) acc[c] = 0.f;
-  if (valid) {
-    const uint4* src = reinterpret_cast<const uint4*>(q + ((long long)b * Hq + (long long)g * G) * D) + e8;
+  if (in && bs < Bq) {
+    const uint4* src = reinterpret_cast<const uint4*>(q + ((long long)bs * Hq + (long long)g * G) * D) + e8;
     for (int hh = 0; hh < G; ++hh) {
       const uint4 w = __ldg(src + (long long)hh * D8);
       acc[0] = acc[0] + bf16_lo(w.x);
@@ -695,6 +770,8 @@ __global__ void __launch_bounds__(256) dtc_qhat_kernel(const uint16_t* __restric
       acc[6] = acc[6] + bf16_lo(w.w);
       acc[7] = acc[7] + bf16_hi(w.w);
     }
+  }
+  if (valid) {
     float4* d32 = reinterpret_cast<float4*>(qh32 + ((long long)b * Hkv + g) * D + e8 * 8);
     d32[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
     d32[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
@@ -1084,7 +1161,7 @@ DecTcLayout dec_tc_layout(const DecodeDims& D) {
   lo.range = (int)((per + kCt - 1) / kCt * kCt);
   lo.n_split = (int)((D.Nc + lo.range - 1) / lo.range);
   const size_t rows = (size_t)D.Bq * D.Hkv;
-  const size_t nc = rows * lo.n_split * SelCfg<KT>::kBuf;
+  const size_t nc = rows * lo.n_split * SelCfg<KT>::kExport;
   size_t o = 0;
   lo.qh32 = o;
   o = align256(o + rows * D.d * 4);
@@ -1179,7 +1256,7 @@ cudaError_t run_decode_tc(const DecodeDims& Dm, const void* q, const void* K, co
   e = launch_dependent(dtc_merge_kernel<DD>, dim3((unsigned)rows), dim3(kMergeWarps * 32), mg_smem, st,
                        (const float*)a.cand_l, (const float*)a.cand_u, (const int32_t*)a.cand_c,
                        (const int32_t*)a.cand_n, (const float*)a.cand_d, (const float4*)a.cand_s,
-                       (int)SelCfg<KT>::kBuf, (const float*)qh32, kbar32, idx, s_sel, w, Dm.Bq, Dm.Hkv, (int)Dm.Nc,
+                       (int)SelCfg<KT>::kExport, (const float*)qh32, kbar32, idx, s_sel, w, Dm.Bq, Dm.Hkv, (int)Dm.Nc,
                        lo.n_split, lo.range, Dm.topk, Dm.scale_sel, Dm.stick ? 1 : 0, counters);
   note_launches(1);
   if (e != cudaSuccess || (e = cudaGetLastError()) != cudaSuccess) return e;

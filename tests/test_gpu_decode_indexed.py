@@ -61,6 +61,9 @@ CASES = {
     "d64 k8 two groups": dict(L=64 * 300, Hq=8, Hkv=2, d=64, topk=8, Bq=70),
     "d128 k16 one group": dict(L=64 * 520, Hq=16, Hkv=1, d=128, topk=16, Bq=33),
     "d128 k4 G2": dict(L=64 * 130 + 17, Hq=4, Hkv=2, d=128, topk=4, Bq=129),
+    # at most 64 queries and groups of 8 columns: two scan threads per row
+    "d128 k4 two threads per row": dict(L=64 * 700, Hq=8, Hkv=1, d=128, topk=4, Bq=64),
+    "d64 k2 G2 two threads per row, ragged": dict(L=64 * 250 + 9, Hq=4, Hkv=2, d=64, topk=2, Bq=17),
 }
 
 
@@ -80,17 +83,19 @@ def test_decode_variants_match_oracle(variant, exact):
     check_against_oracle(w, inner=variant[0], weights=variant[1], exact=exact)
 
 
-def test_indexed_decode_equal_summaries_take_the_exact_path():
+@pytest.mark.parametrize("topk", [8, 4])
+def test_indexed_decode_equal_summaries_take_the_exact_path(topk):
     # every chunk of the memory equal: every score of a query ties, the
     # per-range candidate buffers overflow and the merge scores whole ranges
-    w = synth.Workload("dec-eq", 62, B=1, L=64 * 200, S=64, Hq=8, Hkv=1, d=64, topk=8, backward=False,
+    # (k = 4: two scan threads per row)
+    w = synth.Workload("dec-eq", 62, B=1, L=64 * 200, S=64, Hq=8, Hkv=1, d=64, topk=topk, backward=False,
                        decode=True, Bq=9)
     bits = {n: synth.host_tensor(w, n, (0, 0, 0, 0), w.dims(n)) for n in ("q", "K", "V")}
     K = bits["K"]
     for c in range(1, w.Nc):
         K[:, c * 64:(c + 1) * 64] = K[:, 0:64]
     idx = check_against_oracle(w, bits)
-    assert (idx[:, 0, :].cpu().numpy() == np.arange(7, -1, -1)).all()
+    assert (idx[:, 0, :].cpu().numpy() == np.arange(topk - 1, -1, -1)).all()
 
 
 def test_indexed_decode_64m_memory_matches_exact_decode():

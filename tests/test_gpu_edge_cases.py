@@ -100,7 +100,11 @@ def shape_scale(G, d):
     return oracle.default_scales(G, d)[0]
 
 
-@pytest.mark.parametrize("topk,nclu", [(8, 20), (8, 60)])
+# k = 4 on ranges of 64 chunks takes groups of 8 columns, so a block of at most
+# 64 queries scans each row with two threads (one per half of every tile);
+# with 150 cluster chunks a range holds about 30, more than one export buffer,
+# and the merge scores those ranges exactly.
+@pytest.mark.parametrize("topk,nclu", [(8, 20), (8, 60), (4, 20), (4, 150)])
 def test_indexed_decode_is_exact_under_dense_near_ties(topk, nclu):
     Nc, d, G = 300, 128, 8
     w = synth.Workload("dec-near-ties", 62, B=1, L=64 * Nc, S=64, Hq=G, Hkv=1, d=d, topk=topk, backward=False,

@@ -84,7 +84,6 @@ struct SelTcSmem {
   float bl[kBuf][kTok];                  // collected entries: lower bounds, later exact scores
   float bu[kBuf][kTok];                  //   upper bounds
   int bi[kBuf][kTok];                    //   chunk indices
-  unsigned long long chosen[DEC ? 1 : KT][kTok];  // the k best exact keys (prefill)
   float knt[kKn][kCt + 4];               // |K̄_i| of a tile, then the tile's max (ring of kKn)
   uint64_t bar[kBars];
   float xch[DEC ? 2 : 1][DEC ? 4 : 1][kTok];  // decode pairs: bound terms swapped after each tile
@@ -178,6 +177,26 @@ __device__ __forceinline__ float staged_dot(const float (&q)[D], uint32_t stage,
   return acc;
 }
 
+// The same chain for a row whose q̂ lives in lane src's registers: element e
+// comes over by shuffle (every lane of the warp takes part).
+template <int D>
+__device__ __forceinline__ float staged_dot_from(const float (&q)[D], int src, uint32_t stage, int lane) {
+  const uint32_t row = stage + (uint32_t)(lane * D) * 4u;
+  float acc = 0.f;
+#pragma unroll
+  for (int j = 0; j < D / 4; ++j) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(row + ((uint32_t)(j ^ (lane & 7)) << 4)));
+    acc = fmaf(__shfl_sync(0xFFFFFFFFu, q[4 * j], src), v.x, acc);
+    acc = fmaf(__shfl_sync(0xFFFFFFFFu, q[4 * j + 1], src), v.y, acc);
+    acc = fmaf(__shfl_sync(0xFFFFFFFFu, q[4 * j + 2], src), v.z, acc);
+    acc = fmaf(__shfl_sync(0xFFFFFFFFu, q[4 * j + 3], src), v.w, acc);
+  }
+  return acc;
+}
+
 template <int D, int KT, bool DEC>
 __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     sel_tc_kernel(SelTcArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
@@ -221,14 +240,14 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
   // for short rows, keep at least 2k terms per row.
   const int vis0 = DEC ? vis_max : min(t0 / kChunk, a.Nc);
   const int gsz = vis0 >= 64 * a.topk ? 32 : (vis0 >= 16 * a.topk ? 8 : 1);
-  // Decode: one sweep over the tiles collects, past the first t_warm tiles
-  // (2k terms), every chunk whose upper bound reaches the bound built so far;
-  // the bound only grows, so this is a superset of the chunks reaching the
-  // final one. The t_warm tiles are then visited again against the final
-  // bound. Prefill rows (longer, k up to 16) collect far more chunks against
-  // the early bound than against the final one, so they sweep twice
-  // (t_warm = ntiles): the first sweep builds the bound, the second collects.
-  const int t_warm = DEC ? min(ntiles, (2 * a.topk * gsz + kCt - 1) / kCt) : ntiles;
+  // One sweep over the tiles collects, past the first t_warm tiles, every
+  // chunk whose upper bound reaches the bound built so far; the bound only
+  // grows, so this is a superset of the chunks reaching the final one. The
+  // t_warm tiles are then visited again against the final bound. Decode
+  // starts collecting once the bound holds 2k terms; prefill rows (longer, k
+  // up to 16, a buffer per thread) once it holds 8k, which keeps the chunks
+  // the early bound admits from crowding their buffers.
+  const int t_warm = min(ntiles, ((DEC ? 2 : 8) * a.topk * gsz + kCt - 1) / kCt);
   const int n_iter = ntiles + t_warm;
 
   if (tid == 0) {
@@ -532,14 +551,33 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");
     {
+      // The warp's candidates, listed row after row, are rescored 32 at a
+      // time: lane l takes entry base + l, whatever row it belongs to, and
+      // reads that row's q̂ from the owning lane by shuffle.
       const int my_n = (live && !overflow) ? nc : 0;
-      const int rounds = __reduce_max_sync(0xFFFFFFFFu, (unsigned)my_n);
+      int incl = my_n;  // inclusive prefix of the entry counts over the warp's lanes
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += v;
+      }
+      const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
       const float* kb = a.kbar32 + ((long long)b * a.Nc * a.Hkv + g) * D;
       const uint32_t stage = abase + (uint32_t)(warp * 32 * D) * 4u;  // 32 rows per warp inside A and B
-      for (int j = 0; j < rounds; ++j) {
-        const int c = j < my_n ? sm.bi[j][r] : -1;
+      for (int base = 0; base < total; base += 32) {
+        const int e = base + lane;
+        int src = 0;  // the owning lane: the number of lanes whose prefix ends at or before e
+#pragma unroll
+        for (int step = 16; step >= 1; step >>= 1) {
+          const int v = __shfl_sync(0xFFFFFFFFu, incl, src + step - 1);
+          if (v <= e) src += step;
+        }
+        const int j = e - (__shfl_sync(0xFFFFFFFFu, incl, src) - __shfl_sync(0xFFFFFFFFu, my_n, src));
+        const int rs = warp * 32 + src;
+        const int c = e < total ? sm.bi[j][rs] : -1;
         stage_kbar_rows<D>(stage, kb, (long long)a.Hkv * D, c, lane);
-        if (c >= 0) sm.bl[j][r] = staged_dot<D>(qr, stage, lane) * a.scale_sel;
+        const float v = staged_dot_from<D>(qr, src, stage, lane);
+        if (c >= 0) sm.bl[j][rs] = v * a.scale_sel;
         __syncwarp();
       }
     }
@@ -551,26 +589,31 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       if (overflow) {
         a.flags[atomicAdd(a.nflag, 1u)] = (int32_t)p;
       } else {
-        unsigned long long(*chosen)[kTok] = sm.chosen;
-        // the keff largest keys (keys are distinct: they carry the chunk index)
-        unsigned long long prev = ~0ull;
-        for (int s = 0; s < keff; ++s) {
-          unsigned long long best = 0ull;
-          for (int j = 0; j < nc; ++j) {
-            const unsigned long long kj = rank_key(sm.bl[j][r], (uint32_t)sm.bi[j][r]);
-            if (kj < prev && kj > best) best = kj;
+        // the KT largest keys, in registers (keys are distinct: they carry the
+        // chunk index; 0 never beats a real key)
+        unsigned long long top[KT];
+#pragma unroll
+        for (int i = 0; i < KT; ++i) top[i] = 0ull;
+        for (int j = 0; j < nc; ++j) {
+          unsigned long long v = rank_key(sm.bl[j][r], (uint32_t)sm.bi[j][r]);
+#pragma unroll
+          for (int i = 0; i < KT; ++i) {
+            const unsigned long long hi = top[i] > v ? top[i] : v;
+            v = top[i] > v ? v : top[i];
+            top[i] = hi;
           }
-          chosen[s][r] = best;
-          prev = best;
         }
-        // emitted by decreasing chunk index
-        for (int s = 0; s < keff; ++s) {
-          const unsigned long long ks = chosen[s][r];
-          const uint32_t cs = key_chunk(ks);
-          int pos = 0;
-          for (int u = 0; u < keff; ++u) pos += key_chunk(chosen[u][r]) > cs ? 1 : 0;
-          out_i[pos] = (int32_t)cs;
-          out_s[pos] = key_score(ks);
+        // the keff best, emitted by decreasing chunk index
+#pragma unroll
+        for (int s = 0; s < KT; ++s) {
+          if (s < keff) {
+            const uint32_t cs = key_chunk(top[s]);
+            int pos = 0;
+#pragma unroll
+            for (int u = 0; u < KT; ++u) pos += (u < keff && key_chunk(top[u]) > cs) ? 1 : 0;
+            out_i[pos] = (int32_t)cs;
+            out_s[pos] = key_score(top[s]);
+          }
         }
         for (int s = keff; s < a.topk; ++s) {
           out_i[s] = -1;

@@ -879,7 +879,10 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
   __shared__ float red[kMergeWarps];
   __shared__ float lam_s;
   __shared__ int any_unsure, n_cand, n_hit;
-  __shared__ int hit[kMaxSplit];    // ranges whose bounds can reach the current threshold
+  __shared__ int hit[kMaxSplit];      // ranges whose bounds can reach the current threshold
+  __shared__ int hpre[kMaxSplit + 1];  // exclusive prefix of their entry counts
+  __shared__ unsigned long long rkey[kMaxSplit];  // per range: key of its largest lower bound (0: none)
+  __shared__ unsigned long long ranked[32];       // the k best keys of the warp lists, by rank
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const int row = blockIdx.x;  // b * Hkv + g
   const int b = row / Hkv, g = row % Hkv;
@@ -903,16 +906,27 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
   ls = warp_max(ls);
   if (lane == 0) red[wib] = ls;
   auto krow = [&](int c) { return kbar32 + ((long long)c * Hkv + g) * D; };
-  auto combine = [&](unsigned long long mine) {  // top-k of the warp lists, in warp 0
+  // top-k of the warp lists (lane l of each holds its rank-l key, 0: none),
+  // in warp 0: every listed key counts the keys above it (keys are distinct)
+  auto combine = [&](unsigned long long mine) {
     lists[wib][lane] = mine;
+    if (threadIdx.x < 32) ranked[threadIdx.x] = 0ull;
     __syncthreads();
-    unsigned long long all = 0ull;
-    if (wib == 0)
-      for (int k = 0; k < kMergeWarps; ++k) warp_topk_offer(all, lane < topk ? lists[k][lane] : 0ull, topk, lane);
+    const int n = kMergeWarps * topk;
+    if (threadIdx.x < n) {
+      const unsigned long long key = lists[threadIdx.x / topk][threadIdx.x % topk];
+      if (key != 0ull) {
+        int rank = 0;
+        for (int j = 0; j < n; ++j) rank += lists[j / topk][j % topk] > key ? 1 : 0;
+        if (rank < topk) ranked[rank] = key;
+      }
+    }
     __syncthreads();
-    return all;
+    return wib == 0 ? ranked[lane] : 0ull;
   };
-  // the ranges whose bound `field` reaches t, listed in shared memory (any order)
+  // the ranges whose bound `field` reaches t, listed in shared memory (any
+  // order), with the exclusive prefix of their entry counts; returns the
+  // number of listed entries
   auto list_ranges = [&](int field, float t) {
     if (threadIdx.x == 0) n_hit = 0;
     __syncthreads();
@@ -921,21 +935,48 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
       if ((field == 1 ? v.y : v.z) >= t) hit[atomicAdd(&n_hit, 1)] = sp;
     }
     __syncthreads();
-    return n_hit;
-  };
-  __syncthreads();
-  {  // the k-th largest of the ranges' largest lower bounds (each warp a share of the ranges)
-    unsigned long long top = 0ull;
-    for (int sp0 = wib * 32; sp0 < n_split; sp0 += kMergeWarps * 32) {
-      const int sp = sp0 + lane;
-      const unsigned long long key =
-          sp < n_split && rs[sp].y > -INFINITY ? ((unsigned long long)order_bits(rs[sp].y) << 32) | (uint32_t)sp : 0ull;
-      warp_topk_offer(top, key, topk, lane);
+    if (wib == 0) {  // lane l sums a run of the listed ranges, then a warp scan
+      const int nh = n_hit, per = (nh + 31) / 32, h0 = min(lane * per, nh), h1 = min(h0 + per, nh);
+      int sum = 0;
+      for (int h = h0; h < h1; ++h) sum += rn[hit[h]];
+      int incl = sum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += v;
+      }
+      int run = incl - sum;
+      for (int h = h0; h < h1; ++h) {
+        hpre[h] = run;
+        run += rn[hit[h]];
+      }
+      if (lane == 31) hpre[nh] = incl;
     }
-    const unsigned long long all = combine(top);
-    if (wib == 0) {
-      const unsigned long long kth = __shfl_sync(0xFFFFFFFFu, all, topk - 1);
-      if (lane == 0) lam_s = kth != 0ull ? order_bits_to_float((uint32_t)(kth >> 32)) : -INFINITY;
+    __syncthreads();
+    return hpre[n_hit];
+  };
+  // entry e of the listed ranges: (range, slot) through the prefix
+  auto entry_at = [&](int e, int& sp, int& j) {
+    int lo = 0, hi = n_hit;  // the last h with hpre[h] <= e
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (hpre[mid] <= e) lo = mid; else hi = mid;
+    }
+    sp = hit[lo];
+    j = e - hpre[lo];
+  };
+  for (int sp = threadIdx.x; sp < n_split; sp += kMergeWarps * 32)
+    rkey[sp] = rs[sp].y > -INFINITY ? ((unsigned long long)order_bits(rs[sp].y) << 32) | (uint32_t)sp : 0ull;
+  if (threadIdx.x == 0) lam_s = -INFINITY;
+  __syncthreads();
+  // the k-th largest of the ranges' largest lower bounds: each range key
+  // counts the range keys above it
+  for (int sp = threadIdx.x; sp < n_split; sp += kMergeWarps * 32) {
+    const unsigned long long key = rkey[sp];
+    if (key != 0ull) {
+      int rank = 0;
+      for (int j = 0; j < n_split; ++j) rank += rkey[j] > key ? 1 : 0;
+      if (rank == topk - 1) lam_s = rs[sp].y;
     }
   }
   __syncthreads();
@@ -947,16 +988,15 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
   // hold them: the entries of the listed ranges, one per thread
   unsigned long long lst = 0ull;
   {
-    const int nh = list_ranges(1, lam_star);
-    for (int base = wib * 32; base < nh * kbuf; base += kMergeWarps * 32) {
-      const int i = base + lane;
+    const int ne = list_ranges(1, lam_star);
+    for (int base = wib * 32; base < ne; base += kMergeWarps * 32) {
+      const int e = base + lane;
       unsigned long long key = 0ull;
-      if (i < nh * kbuf) {
-        const int sp = hit[i / kbuf], j = i % kbuf;
-        if (j < rn[sp]) {
-          const float l = cand_l[(cbase + sp) * kbuf + j];
-          if (l >= lam_star) key = ((unsigned long long)order_bits(l) << 32) | (uint32_t)(sp * kbuf + j);
-        }
+      if (e < ne) {
+        int sp, j;
+        entry_at(e, sp, j);
+        const float l = cand_l[(cbase + sp) * kbuf + j];
+        if (l >= lam_star) key = ((unsigned long long)order_bits(l) << 32) | (uint32_t)(sp * kbuf + j);
       }
       warp_topk_offer(lst, key, topk, lane);
     }
@@ -976,13 +1016,14 @@ __global__ void __launch_bounds__(kMergeWarps * 32) dtc_merge_kernel(
   // (past the list's capacity they are scored here, one per lane)
   unsigned long long fin = 0ull;
   {
-    const int nh = list_ranges(2, lam);
-    for (int base = wib * 32; base < nh * kbuf; base += kMergeWarps * 32) {
-      const int i = base + lane;
+    const int ne = list_ranges(2, lam);
+    for (int base = wib * 32; base < ne; base += kMergeWarps * 32) {
+      const int e = base + lane;
       unsigned long long key = 0ull;
-      if (i < nh * kbuf) {
-        const int sp = hit[i / kbuf], j = i % kbuf;
-        if (j < rn[sp] && cand_u[(cbase + sp) * kbuf + j] >= lam) {
+      if (e < ne) {
+        int sp, j;
+        entry_at(e, sp, j);
+        if (cand_u[(cbase + sp) * kbuf + j] >= lam) {
           const int c = cand_c[(cbase + sp) * kbuf + j];
           const int pos = atomicAdd(&n_cand, 1);
           if (pos < kMergeCand)

@@ -348,13 +348,13 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     float bm[KT];  // slots [KT-k, KT): the k largest terms (descending); +inf above
 #pragma unroll
     for (int i = 0; i < KT; ++i) bm[i] = i < KT - a.topk ? INFINITY : -INFINITY;
-    auto push = [&](float v) {  // branch-free insertion: bm keeps the k largest
+    // branch-free insertion: bm keeps the k largest. Slot i of the new list is
+    // the larger of the old slot i and min(old slot i-1, v), so every slot is
+    // formed independently (no chain through the list).
+    auto push = [&](float v) {
 #pragma unroll
-      for (int i = 0; i < KT; ++i) {
-        const float hi = fmaxf(bm[i], v);
-        v = fminf(bm[i], v);
-        bm[i] = hi;
-      }
+      for (int i = KT - 1; i > 0; --i) bm[i] = fmaxf(bm[i], fminf(bm[i - 1], v));
+      bm[0] = fmaxf(bm[0], v);
     };
     float lam_lo = -INFINITY;  // the final bound (second visits)
     int cnt = 0;  // collected entries
@@ -594,14 +594,14 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
         unsigned long long top[KT];
 #pragma unroll
         for (int i = 0; i < KT; ++i) top[i] = 0ull;
-        for (int j = 0; j < nc; ++j) {
-          unsigned long long v = rank_key(sm.bl[j][r], (uint32_t)sm.bi[j][r]);
+        for (int j = 0; j < nc; ++j) {  // insertion with every slot formed independently
+          const unsigned long long v = rank_key(sm.bl[j][r], (uint32_t)sm.bi[j][r]);
 #pragma unroll
-          for (int i = 0; i < KT; ++i) {
-            const unsigned long long hi = top[i] > v ? top[i] : v;
-            v = top[i] > v ? v : top[i];
-            top[i] = hi;
+          for (int i = KT - 1; i > 0; --i) {
+            const unsigned long long lo = top[i - 1] < v ? top[i - 1] : v;
+            top[i] = top[i] > lo ? top[i] : lo;
           }
+          top[0] = top[0] > v ? top[0] : v;
         }
         // the keff best, emitted by decreasing chunk index
 #pragma unroll

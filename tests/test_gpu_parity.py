@@ -282,6 +282,35 @@ def test_full_size_prefill_1m_needles():
     assert_close("O sampled", bf16_tensor_to_f64(fwd["O"][0, sample]), O[0, sample])
 
 
+# Rows longer than the selection's warm-up: once its bound holds 8k group terms
+# (after t_warm tiles of 64 chunks) the kernel collects candidates during its
+# one sweep against the bound built so far, and visits only the first t_warm
+# tiles again. k = 2 with groups of 32 columns warms up over 8 tiles, k = 12
+# (the kernel for k <= 16) over 48; these rows reach 25 and 55 tiles.
+@pytest.mark.parametrize("topk,Nc,G,d", [(2, 1600, 2, 64), (12, 3500, 4, 64)])
+def test_long_rows_collect_during_the_sweep(topk, Nc, G, d):
+    w = synth.Workload("long-rows", 80 + topk, B=1, L=64 * Nc + 13, S=64, Hq=G, Hkv=1, d=d, topk=topk,
+                       backward=False)
+    shape = shape_of(w)
+    dev = device_inputs(w, ("q", "K"))
+    kbar32_d, _ = hsa.chunk_pool(shape, dev["K"], want_bf16=False)
+    idx, s_sel = hsa.select_topk(shape, dev["q"], kbar32_d)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(topk)
+    sample = np.unique(np.concatenate([rng.choice(w.L, 256, replace=False), np.arange(w.L - 128, w.L)]))
+    K = synth.bf16_to_f64(synth.host_tensor(w, "K", (0, 0, 0, 0), w.dims("K")))
+    kbar32 = oracle.pool(K, w.S, f32=True)
+    assert np.array_equal(kbar32_d.cpu().numpy(), kbar32.astype(np.float32))
+    qb = np.zeros((1, w.L, w.Hq, w.d), np.uint16)
+    for t in sample:
+        qb[:, t:t + 1] = synth.host_tensor(w, "q", (0, t, 0, 0), (1, t + 1, w.Hq, w.d))
+    mask = np.zeros((1, w.L), np.uint8)
+    mask[0, sample] = 1
+    ridx, rs, _ = oracle.select(synth.bf16_to_f64(qb), kbar32, w.S, w.topk, f32=True, token_mask=mask)
+    assert np.array_equal(idx[0, sample].cpu().numpy(), ridx[0, sample])
+    assert np.array_equal(s_sel[0, sample].cpu().numpy(), rs[0, sample].astype(np.float32))
+
+
 def test_full_size_decode_64m_memory():
     w = synth.WORKLOADS[5]
     T, Nc, d = w.L, w.Nc, w.d

@@ -60,7 +60,8 @@ typedef enum {
     HSA_ERR_UNSUPPORTED = 2,
     HSA_ERR_WORKSPACE = 3,
     HSA_ERR_CUDA = 4,
-    HSA_ERR_TIMEOUT = 5
+    HSA_ERR_TIMEOUT = 5,
+    HSA_ERR_BOUNDS = 6
 } hsa_status_t;
 
 /* Variant flags (hsa_shape_t.flags, hsa_decode_shape_t.flags); 0 selects the
@@ -127,8 +128,17 @@ size_t hsa_status_bytes(void);
  * Waits for `stream` (the stream of those calls), reads and clears the
  * word, and returns HSA_ERR_TIMEOUT if a wait gave up in a call that used
  * this workspace since the word was last cleared (the results of those
- * calls are then invalid), HSA_ERR_CUDA if the stream reports an error,
+ * calls are then invalid), HSA_ERR_BOUNDS if such a call found an input
+ * index out of range (only a library built with the debug bounds checks,
+ * see below, looks), HSA_ERR_CUDA if the stream reports an error,
  * HSA_OK otherwise; HSA_ERR_INVALID_ARG for a bad workspace.
+ * Debug-bounds build (compiled with -DHSA_DEBUG_BOUNDS): every index the
+ * forward, backward and index kernels read from an input array (the chunk
+ * ids of idx, the offsets and slot ids of the inverse index) is checked
+ * against its range before use; an out-of-range value sets the status word
+ * and the access it would have made is skipped (no trap, no fault), so
+ * hsa_check then returns HSA_ERR_BOUNDS. Other builds skip the checks
+ * (out-of-range chunk ids still count as no selection there).
  * The word is sticky until checked, so a new workspace must start with it
  * cleared: zero its first hsa_status_bytes() bytes after allocating it (or
  * call hsa_check once and ignore the result).

@@ -3,6 +3,10 @@
 Each translation unit compiles in parallel; the shared library links against
 the shared CUDA runtime so that it shares the runtime (and therefore streams)
 with the host process. The result stays in-tree under _build/.
+
+build(debug_bounds=True) makes the debug-bounds variant (HSA_DEBUG_BOUNDS:
+input indices checked before use and reported through the status word that
+hsa_check reads) as _build_debug/libhsa_debug.so, beside the normal library.
 """
 from __future__ import annotations
 
@@ -17,6 +21,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libhsa.so")
+BUILD_DEBUG = os.path.join(HERE, "_build_debug")
+LIB_DEBUG = os.path.join(BUILD_DEBUG, "libhsa_debug.so")
 
 SOURCES = ["api.cu", "pool.cu", "select.cu", "select_tc.cu", "index.cu", "fwd.cu", "bwd.cu", "decode.cu", "decode_noalloc.cu",
            "selftest.cu", "memory.cu"]
@@ -45,20 +51,22 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(verbose: bool = False, jobs: int | None = None) -> str:
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose: bool = False, jobs: int | None = None, debug_bounds: bool = False) -> str:
+    out_dir, lib = (BUILD_DEBUG, LIB_DEBUG) if debug_bounds else (BUILD, LIB)
+    extra = ["-DHSA_DEBUG_BOUNDS"] if debug_bounds else []
+    os.makedirs(out_dir, exist_ok=True)
     headers = [os.path.join(CSRC, h) for h in HEADERS] + [os.path.join(INCLUDE, "hsa.h")]
     objs, todo = [], []
     for src in SOURCES:
         s = os.path.join(CSRC, src)
-        o = os.path.join(BUILD, src.replace(".cu", ".o"))
+        o = os.path.join(out_dir, src.replace(".cu", ".o"))
         objs.append(o)
         if _stale(o, [s, *headers]):
             todo.append((s, o))
 
     def compile_one(job):
         s, o = job
-        cmd = [nvcc(), *_flags(), "-c", s, "-o", o + ".tmp"]
+        cmd = [nvcc(), *_flags(), *extra, "-c", s, "-o", o + ".tmp"]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed for {s}:\n{r.stderr}")
@@ -70,15 +78,15 @@ def build(verbose: bool = False, jobs: int | None = None) -> str:
             for err in ex.map(compile_one, todo):
                 if verbose and err:
                     sys.stderr.write(err)
-    if todo or _stale(LIB, objs):
-        tmp = LIB + f".tmp{os.getpid()}"
+    if todo or _stale(lib, objs):
+        tmp = lib + f".tmp{os.getpid()}"
         cmd = [nvcc(), *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs,
                "-Xlinker", f"-rpath,{cuda_lib_dir()}"]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"link failed:\n{r.stderr}")
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":

@@ -89,6 +89,7 @@ const char* hsa_status_string(hsa_status_t status) {
     case HSA_ERR_WORKSPACE: return "HSA_ERR_WORKSPACE: workspace missing or too small";
     case HSA_ERR_CUDA: return "HSA_ERR_CUDA: a kernel launch failed";
     case HSA_ERR_TIMEOUT: return "HSA_ERR_TIMEOUT: a device-side wait gave up (results invalid)";
+    case HSA_ERR_BOUNDS: return "HSA_ERR_BOUNDS: an input index was out of range (debug-bounds build; results invalid)";
   }
   return "HSA_ERR_UNKNOWN";
 }
@@ -104,7 +105,7 @@ hsa_status_t hsa_check(void* ws, size_t ws_bytes, cudaStream_t stream) {
   if (cudaMemcpyAsync(&v, ws, sizeof(v), cudaMemcpyDeviceToHost, stream) != cudaSuccess ||
       cudaMemsetAsync(ws, 0, sizeof(v), stream) != cudaSuccess || cudaStreamSynchronize(stream) != cudaSuccess)
     return HSA_ERR_CUDA;
-  return v ? HSA_ERR_TIMEOUT : HSA_OK;
+  return (v & hsa::kStatusTimeout) ? HSA_ERR_TIMEOUT : (v ? HSA_ERR_BOUNDS : HSA_OK);
 }
 
 size_t hsa_status_bytes(void) { return kStatusBytes; }

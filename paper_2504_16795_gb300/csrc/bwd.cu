@@ -98,6 +98,7 @@ struct BwdArgs {
   float* dV;
   int L, Hq, Hkv, G, log2G, topk, Nc;
   int n_rows;   // B * L * Hq (a row index past it reads zeros)
+  long long n_slots;  // B * L * Hkv * topk (slot ids; debug builds check offsets and entries against it)
   int use_tma;  // G >= 8: each slot's G rows arrive as one swizzled TMA box
   float scale_log2, scale_attn, scale_sel;
   int softmax1;   // softmax-off-by-one inside the chunk
@@ -130,7 +131,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int key = bg * a.Nc + c;
   const int b = bg / a.Hkv, g = bg % a.Hkv;
   const int off = a.offsets[key];
-  const int cnt = a.offsets[key + 1] - off;
+  int cnt = a.offsets[key + 1] - off;
+  if (!(bounds_ok(off, 0, a.n_slots + 1, a.status) && bounds_ok(off + cnt, off, a.n_slots + 1, a.status)))
+    cnt = 0;  // debug: a list outside the entries is skipped
   const long long row0 = ((long long)b * a.L + (long long)c * kChunk) * a.Hkv + g;
   if (cnt <= 0) {  // a chunk nobody selected: no gradient
     for (int u = tid; u < kChunk * D; u += kThreads) {
@@ -199,16 +202,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int islot = item < epi ? item : item - epi;
     const uint32_t item_bytes = (uint32_t)((2 * epi - li + kLoaders - 1) / kLoaders) * a.G * D * 2;
     const uint64_t keep = tc::l2_evict_last();
+    auto checked = [&](int p) { return p < 0 || bounds_ok(p, 0, a.n_slots, status) ? p : -1; };
     auto load_ip = [&](int i) {
       const int e = i * epi + islot;
-      return (has_item && e < cnt) ? a.entries[off + e] : -1;
+      return checked((has_item && e < cnt) ? a.entries[off + e] : -1);
     };
     auto row_of = [&](int p) {  // past the list: rows past the tensor read zeros
       return p < 0 ? a.n_rows : ((b * a.L + (p / slot_div) % a.L) * a.Hq) + g * a.G;
     };
     auto load_p = [&](int i) {  // warp 8's slot tables: lane l holds slot l
       const int e = i * epi + lane;
-      return (li == 0 && epi <= 32 && lane < epi && e < cnt) ? a.entries[off + e] : -1;
+      return checked((li == 0 && epi <= 32 && lane < epi && e < cnt) ? a.entries[off + e] : -1);
     };
     int n_row = -1, n_p = -1;
     float n_w = 0.f, n_dl = 0.f;
@@ -256,8 +260,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               const int e = i * epi + sl;
               int row = -1, p = -1;
               float wv = 0.f, dl = 0.f;
-              if (e < cnt) {
-                p = a.entries[off + e];
+              if (e < cnt) p = checked(a.entries[off + e]);
+              if (p >= 0) {
                 const int t = (p / slot_div) % a.L;
                 row = ((b * a.L + t) * a.Hq) + g * a.G;
                 wv = a.w[p];
@@ -601,13 +605,15 @@ __global__ void __launch_bounds__(256) bwd_delta_kernel(const uint16_t* __restri
 // accumulate: ds += (layers sharing one selection add their score gradients).
 __global__ void __launch_bounds__(256) bwd_ds_kernel(const int32_t* __restrict__ idx, const float* __restrict__ w,
                                                      const float* __restrict__ dw, float* __restrict__ ds,
-                                                     long long n_rows, int topk, int Nc, int stick, int accumulate) {
+                                                     long long n_rows, int topk, int Nc, int stick, int accumulate,
+                                                     unsigned* __restrict__ status) {
   const long long row = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (row >= n_rows) return;
   const long long p0 = row * topk;
   int keff = 0;
   while (keff < topk) {
     const int c = idx[p0 + keff];
+    if (c >= 0) bounds_ok(c, 0, Nc, status);  // debug: a chunk id past the sequence is reported
     if (c < 0 || c >= Nc) break;
     ++keff;
   }
@@ -639,7 +645,7 @@ template <int D>
 __global__ void __launch_bounds__(256) sel_dq_kernel(const int32_t* __restrict__ idx, const float* __restrict__ ds,
                                                      const float* __restrict__ kbar32, float* __restrict__ dq,
                                                      long long n_rows, int G, int topk, int Nc, int L, int Hkv,
-                                                     float scale_sel) {
+                                                     float scale_sel, unsigned* __restrict__ status) {
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -650,6 +656,7 @@ __global__ void __launch_bounds__(256) sel_dq_kernel(const int32_t* __restrict__
   if (lane < topk) {  // lane j holds slot j's chunk and scaled score gradient
     cl = idx[p0 + lane];
     valid = cl >= 0 && cl < Nc;
+    if (cl >= 0) bounds_ok(cl, 0, Nc, status);
     sl = valid ? scale_sel * ds[p0 + lane] : 0.f;
   }
   const int keff = __popc(__ballot_sync(0xFFFFFFFFu, valid));
@@ -727,13 +734,18 @@ __global__ void __launch_bounds__(D * kDkbarGroups, 2) bwd_stick_dkbar_kernel(co
                                                                            const float* __restrict__ ds,
                                                                            const float* __restrict__ qhat,
                                                                            float* __restrict__ dK, int L, int Hkv,
-                                                                           int topk, int Nc, float scale_sel) {
+                                                                           int topk, int Nc, float scale_sel,
+                                                                           long long n_slots,
+                                                                           unsigned* __restrict__ status) {
   __shared__ float part[kDkbarGroups][D];
   int c, bg;
   block_key(Nc, (int)(gridDim.x / (unsigned)Nc), c, bg);
   const int key = bg * Nc + c;
   const int b = bg / Hkv, g = bg % Hkv;
-  const int off = offsets[key], cnt = offsets[key + 1] - off;
+  const int off = offsets[key];
+  int cnt = offsets[key + 1] - off;
+  if (!(bounds_ok(off, 0, n_slots + 1, status) && bounds_ok(off + cnt, off, n_slots + 1, status)))
+    cnt = 0;  // debug: a list outside the entries is skipped
   if (cnt <= 0) return;
   const int e = threadIdx.x % D, grp = threadIdx.x / D;
   const int slot_div = Hkv * topk;
@@ -747,15 +759,16 @@ __global__ void __launch_bounds__(D * kDkbarGroups, 2) bwd_stick_dkbar_kernel(co
     for (int u = 0; u < 8; ++u) p[u] = entries[off + n + u * kStep];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
-      dv[u] = ds[p[u]];
-      qv[u] = qhat[((long long)(p[u] / slot_div) * Hkv + g) * D + e];
+      const bool ok = bounds_ok(p[u], 0, n_slots, status);  // debug: a slot id out of range adds nothing
+      dv[u] = ok ? ds[p[u]] : 0.f;
+      qv[u] = ok ? qhat[((long long)(p[u] / slot_div) * Hkv + g) * D + e] : 0.f;
     }
 #pragma unroll
     for (int u = 0; u < 8; ++u) acc = fmaf(dv[u], qv[u], acc);
   }
   for (; n < cnt; n += kStep) {
     const int p = entries[off + n];
-    acc = fmaf(ds[p], qhat[((long long)(p / slot_div) * Hkv + g) * D + e], acc);
+    if (bounds_ok(p, 0, n_slots, status)) acc = fmaf(ds[p], qhat[((long long)(p / slot_div) * Hkv + g) * D + e], acc);
   }
   part[grp][e] = acc;
   __syncthreads();
@@ -777,7 +790,7 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
                                                            long long n_rows, int G, int topk, int Nc,
                                                            const float* __restrict__ ds,
                                                            const float* __restrict__ kbar32, int L, int Hkv,
-                                                           float scale_sel) {
+                                                           float scale_sel, unsigned* __restrict__ status) {
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -788,6 +801,7 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
   if (lane < topk) {  // lane j holds slot j's chunk (and, for the selection term, scaled ds)
     cl = idx[p0 + lane];
     valid = cl >= 0 && cl < Nc;
+    if (cl >= 0) bounds_ok(cl, 0, Nc, status);
     if (ds != nullptr && valid) sl = scale_sel * ds[p0 + lane];
   }
   const int keff = __popc(__ballot_sync(0xFFFFFFFFu, valid));
@@ -897,7 +911,8 @@ cudaError_t launch_dkbar(const Dims& Dm, const void* q, const int32_t* offsets, 
   const long long keys = Dm.keys();
   if (keys > 0) {
     bwd_stick_dkbar_kernel<D><<<(unsigned)keys, D * kDkbarGroups, 0, st>>>(offsets, entries, ds, qhat, dK, Dm.L,
-                                                                           Dm.Hkv, Dm.topk, Dm.Nc, Dm.scale_sel);
+                                                                           Dm.Hkv, Dm.topk, Dm.Nc, Dm.scale_sel,
+                                                                           Dm.slots(), Dm.status);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
@@ -964,6 +979,7 @@ cudaError_t run(const Dims& Dm, BwdMode mode, const void* q, const void* K, cons
     memset(&tdo, 0, sizeof(tdo));
     memset(&tdq, 0, sizeof(tdq));
     a.n_rows = Dm.B * Dm.L * Dm.Hq;
+    a.n_slots = Dm.slots();
     a.use_tma = Dm.G >= 8 ? 1 : 0;
     if (a.use_tma && (!tc::make_group8_tmap(&tq, q, (unsigned long long)a.n_rows, D) ||
                       !tc::make_group8_tmap(&tdo, dO, (unsigned long long)a.n_rows, D) ||
@@ -975,7 +991,7 @@ cudaError_t run(const Dims& Dm, BwdMode mode, const void* q, const void* K, cons
   }
   if (dw_mode) {
     bwd_ds_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(idx, w, dwb, dsb, rows, Dm.topk, Dm.Nc,
-                                                                   Dm.stick ? 1 : 0, full ? 0 : 1);
+                                                                   Dm.stick ? 1 : 0, full ? 0 : 1, Dm.status);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (full && (e = launch_dkbar<D>(Dm, q, offsets, entries, dsb, qhat, dK, st)) != cudaSuccess) return e;
@@ -983,7 +999,7 @@ cudaError_t run(const Dims& Dm, BwdMode mode, const void* q, const void* K, cons
   const bool sel_term = full && Dm.stick;
   bwd_dq_merge_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(idx, dqpart, dq, rows, Dm.G, Dm.topk, Dm.Nc,
                                                                       sel_term ? dsb : nullptr, kbar32, Dm.L, Dm.Hkv,
-                                                                      Dm.scale_sel);
+                                                                      Dm.scale_sel, Dm.status);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int tail0 = Dm.Nc * kChunk;
@@ -1007,7 +1023,7 @@ cudaError_t run_select_backward(const Dims& Dm, const void* q_sel, const float* 
   cudaError_t e;
   if ((e = cudaMemsetAsync(dK_sel, 0, (size_t)rows * D * sizeof(float), st)) != cudaSuccess) return e;
   sel_dq_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(idx, ds, kbar_sel, dq_sel, rows, Dm.G, Dm.topk, Dm.Nc,
-                                                               Dm.L, Dm.Hkv, Dm.scale_sel);
+                                                               Dm.L, Dm.Hkv, Dm.scale_sel, Dm.status);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return launch_dkbar<D>(Dm, q_sel, offsets, entries, ds, (float*)ws, dK_sel, st);

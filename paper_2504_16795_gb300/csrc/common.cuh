@@ -11,6 +11,28 @@ namespace hsa {
 
 constexpr int kChunk = 64;  // S: the only chunk size the kernels are built for
 
+// Bits of a call's device status word (the head of its workspace, read and
+// cleared by hsa_check): a bounded wait gave up; an index read from an input
+// array lay outside its range (checked only in builds with HSA_DEBUG_BOUNDS).
+enum : unsigned { kStatusTimeout = 1u, kStatusBounds = 2u };
+#ifdef HSA_DEBUG_BOUNDS
+constexpr bool kDebugBounds = true;
+#else
+constexpr bool kDebugBounds = false;
+#endif
+// Debug builds: whether lo <= v < hi, recording an out-of-range value in the
+// status word, so that the caller skips the access it would have made. Other
+// builds: true (the check compiles away).
+__device__ __forceinline__ bool bounds_ok(long long v, long long lo, long long hi, unsigned* status) {
+  if constexpr (kDebugBounds) {
+    if (v < lo || v >= hi) {
+      if (status) atomicOr(status, kStatusBounds);
+      return false;
+    }
+  }
+  return true;
+}
+
 // Block order of the chunk kernels. A chunk's list holds the slots of every
 // later token that chose it, so early chunks carry the longest lists. The
 // first kHeadChunks chunks of every (b, g) run first, chunk-major across the

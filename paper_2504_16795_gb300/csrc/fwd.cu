@@ -71,6 +71,7 @@ struct FwdArgs {
   uint16_t* Opart;  // [slots, G, D]
   int L, Hq, Hkv, G, log2G, topk, Nc;
   int n_rows;   // B * L * Hq (query rows; a row index past it reads zeros)
+  long long n_slots;  // B * L * Hkv * topk (slot ids; debug builds check entries against it)
   int use_tma;  // G >= 8: each slot's G rows arrive as one swizzled TMA box
   float scale_log2;  // c_att * log2(e)
   int softmax1;      // softmax-off-by-one inside the chunk
@@ -151,7 +152,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t keep = tc::l2_evict_last();
       auto load_p = [&](int i) {
         const int e = i * epi + my_slot;
-        return (a.use_tma && my_slot < epi && e < cnt) ? a.entries[off + e] : -1;
+        const int p = (a.use_tma && my_slot < epi && e < cnt) ? a.entries[off + e] : -1;
+        return p < 0 || bounds_ok(p, 0, a.n_slots, status) ? p : -1;
       };
       auto row_of = [&](int p) {  // past the list: rows past the tensor read zeros
         return p < 0 ? a.n_rows : ((b * a.L + (p / slot_div) % a.L) * a.Hq) + g * a.G;
@@ -180,8 +182,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           int row = -1;
           if (e < cnt) {
             const int p = a.entries[off + e];
-            const int t = (p / slot_div) % a.L;
-            row = ((b * a.L + t) * a.Hq) + g * a.G;
+            if (bounds_ok(p, 0, a.n_slots, status)) {
+              const int t = (p / slot_div) % a.L;
+              row = ((b * a.L + t) * a.Hq) + g * a.G;
+            }
           }
           sm.slot_row[st][sl] = row;
         }
@@ -314,11 +318,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     // slot's G rows with one TMA box per 8 rows. Otherwise rows go out directly.
     const bool issuer = a.use_tma && (r & (a.G - 1)) == 0;
     const uint64_t stream = tc::l2_evict_first();
-    int p_next = r >> a.log2G < cnt ? a.entries[off + (r >> a.log2G)] : -1;
+    auto entry = [&](int e) {  // slot id of list entry e (-1 past the list, or out of range)
+      const int p = e < cnt ? a.entries[off + e] : -1;
+      return p < 0 || bounds_ok(p, 0, a.n_slots, status) ? p : -1;
+    };
+    int p_next = entry(r >> a.log2G);
     for (int j = 0; j < niter; ++j) {
       const int pj = p_next;
       const int en = (j + 1) * epi + (r >> a.log2G);
-      p_next = en < cnt ? a.entries[off + en] : -1;  // prefetch the next step's slot
+      p_next = entry(en);  // prefetch the next step's slot
       const int ob = j & 1;
       const uint32_t stage = smem_u32(sm.Ostage[ob]);
       if (a.use_tma) {  // the stores of step j-2 have read this warp's part of the staging tile
@@ -390,7 +398,8 @@ __device__ __forceinline__ int key_in_order(int i, int Nc, int n_bg) {
 }
 __global__ void __launch_bounds__(1024) fwd_segments_kernel(const int32_t* __restrict__ offsets, int Nc, int n_bg,
                                                             int seg_slots, int4* __restrict__ segs,
-                                                            int* __restrict__ nseg) {
+                                                            int* __restrict__ nseg, long long n_slots,
+                                                            unsigned* __restrict__ status) {
   __shared__ int warp_sum[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int keys = Nc * n_bg;
@@ -399,7 +408,9 @@ __global__ void __launch_bounds__(1024) fwd_segments_kernel(const int32_t* __res
   int n = 0;
   for (int i = i0; i < i1; ++i) {
     const int key = key_in_order(i, Nc, n_bg);
-    const int len = offsets[key + 1] - offsets[key];
+    int o0 = offsets[key], o1 = offsets[key + 1];
+    if (!(bounds_ok(o0, 0, n_slots + 1, status) && bounds_ok(o1, o0, n_slots + 1, status))) o1 = o0;  // debug: skip
+    const int len = o1 - o0;
     n += len > 0 ? (len + seg_slots - 1) / seg_slots : 0;
   }
   int x = n;  // inclusive scan within the warp
@@ -423,7 +434,8 @@ __global__ void __launch_bounds__(1024) fwd_segments_kernel(const int32_t* __res
   int pos = (warp > 0 ? warp_sum[warp - 1] : 0) + x - n;
   for (int i = i0; i < i1; ++i) {
     const int key = key_in_order(i, Nc, n_bg);
-    const int o0 = offsets[key], o1 = offsets[key + 1];
+    int o0 = offsets[key], o1 = offsets[key + 1];
+    if (!(bounds_ok(o0, 0, n_slots + 1, nullptr) && bounds_ok(o1, o0, n_slots + 1, nullptr))) o1 = o0;
     for (int e = o0; e < o1; e += seg_slots) segs[pos++] = make_int4(key, e, min(e + seg_slots, o1), 0);
   }
   if (tid == 1023) *nseg = warp_sum[31];
@@ -435,7 +447,7 @@ __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict_
                                                         const int32_t* __restrict__ idx,
                                                         const uint16_t* __restrict__ Opart, uint16_t* __restrict__ O,
                                                         float* __restrict__ w, long long n_rows, int Hkv, int G,
-                                                        int topk, int Nc, int stick) {
+                                                        int topk, int Nc, int stick, unsigned* __restrict__ status) {
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -445,6 +457,7 @@ __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict_
   if (lane < topk) {
     const int c = idx[p0 + lane];
     valid = c >= 0 && c < Nc;
+    if (c >= 0) bounds_ok(c, 0, Nc, status);  // debug: a chunk id past the memory is reported
     if (valid) s = s_sel[p0 + lane];
   }
   const float wj = warp_chunk_weight(s, valid, stick != 0);
@@ -515,7 +528,8 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     int4* segs = (int4*)((char*)ws + lo.segs);
     int* nseg = (int*)((char*)ws + lo.nseg);
     const int seg_slots = kSegTiles * (kRows / Dm.G);
-    fwd_segments_kernel<<<1, 1024, 0, st>>>(offsets, Dm.Nc, Dm.B * Dm.Hkv, seg_slots, segs, nseg);
+    fwd_segments_kernel<<<1, 1024, 0, st>>>(offsets, Dm.Nc, Dm.B * Dm.Hkv, seg_slots, segs, nseg, Dm.slots(),
+                                            Dm.status);
     note_launches(1);
     cudaError_t e0 = cudaGetLastError();
     if (e0 != cudaSuccess) return e0;
@@ -544,6 +558,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     memset(&tq, 0, sizeof(tq));
     memset(&to, 0, sizeof(to));
     a.n_rows = Dm.B * Dm.L * Dm.Hq;
+    a.n_slots = Dm.slots();
     a.use_tma = Dm.G >= 8 ? 1 : 0;
     if (a.use_tma && !tc::make_group8_tmap(&tq, q, (unsigned long long)a.n_rows, D)) return cudaErrorNotSupported;
     if (a.use_tma && !tc::make_group8_tmap(&to, Opart, (unsigned long long)Dm.slots() * Dm.G, D))
@@ -554,7 +569,7 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
   }
   const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
   fwd_merge_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(s_sel, idx, Opart, (uint16_t*)O, w, rows, Dm.Hkv,
-                                                                  Dm.G, Dm.topk, Dm.Nc, Dm.stick ? 1 : 0);
+                                                                  Dm.G, Dm.topk, Dm.Nc, Dm.stick ? 1 : 0, Dm.status);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -25,8 +25,10 @@ struct KeyMap {
   const int32_t* idx;
   int L, Hkv, topk, Nc;
   uint32_t sentinel;
+  unsigned* status;  // the call's status word (debug builds report chunk ids past the sequence)
   __device__ __forceinline__ uint32_t key(long long p) const {
     const int c = idx[p];
+    if (c >= 0) bounds_ok(c, 0, Nc, status);
     if (c < 0 || c >= Nc) return sentinel;  // padding (or an out-of-range index) is never listed
     const long long g = (p / topk) % Hkv;
     const long long b = p / ((long long)topk * Hkv * L);
@@ -238,7 +240,7 @@ cudaError_t launch_index(const Dims& D, const int32_t* idx, int32_t* offsets, in
   int32_t* vals_buf[2] = {(int32_t*)(w + lo.off_vals_a), (int32_t*)(w + lo.off_vals_b)};
   uint32_t* hist = (uint32_t*)(w + lo.off_hist);
   uint32_t* sums = (uint32_t*)(w + lo.off_sums);
-  KeyMap km{idx, D.L, D.Hkv, D.topk, D.Nc, (uint32_t)lo.keys};
+  KeyMap km{idx, D.L, D.Hkv, D.topk, D.Nc, (uint32_t)lo.keys, D.status};
   cudaError_t e;
   const uint32_t* kin = nullptr;
   const int32_t* vin = nullptr;

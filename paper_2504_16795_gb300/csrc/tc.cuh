@@ -20,7 +20,6 @@ namespace tc {
 // block's abort flag and in a device status word, and returns false, so a
 // broken pipeline ends the kernel instead of hanging the GPU.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
-enum : unsigned { kStatusTimeout = 1u };
 
 // Programmatic dependent launch: a kernel launched as a dependent of the
 // previous kernel in its stream waits here until that grid has completed and

@@ -11,7 +11,7 @@ import synth
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
-OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA, TIMEOUT = 0, 1, 2, 3, 4, 5
+OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA, TIMEOUT, BOUNDS = 0, 1, 2, 3, 4, 5, 6
 
 
 def declared(header):
@@ -41,8 +41,18 @@ def test_synth_device_library_exports_its_header():
 
 
 def test_status_strings(lib):
-    for code in (OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA, TIMEOUT):
+    for code in (OK, INVALID, UNSUPPORTED, WORKSPACE, CUDA, TIMEOUT, BOUNDS):
         assert hsa.status_string(code).startswith("HSA_")
+    assert hsa.status_string(BOUNDS).startswith("HSA_ERR_BOUNDS")
+
+
+def test_debug_bounds_library_exports_every_declared_entry_point():
+    # the HSA_DEBUG_BOUNDS build: the same entry points, index checks inside
+    from paper_2504_16795_gb300.build import build as build_hsa
+
+    dbg = ctypes.CDLL(build_hsa(debug_bounds=True))
+    for n in declared(os.path.join(ROOT, "include", "hsa.h")):
+        assert hasattr(dbg, n), n
 
 
 def shape(**kw):

@@ -334,31 +334,32 @@ def run_gpu(args, rank, world, local_rank):
         h2d = sum(t.numel() * t.element_size() for t in host_in.values())
         d2h = sum(t.numel() * t.element_size() for t in host_out.values())
 
-        # two sets of device inputs and outputs: the next step's inputs go up on one copy stream and the
-        # previous step's outputs come down on another while the compute stream runs the current step
-        X2 = {n: torch.empty_like(X[n]) for n in host_in}
-        Y2 = dict(Y, **{n: torch.empty_like(Y[n]) for n in host_out})
-        sets = [(X, Y), (X2, Y2)]
+        # three sets of device inputs and outputs: the inputs of the next steps go up on one copy stream
+        # and the outputs of earlier steps come down on another while the compute stream runs the
+        # current step (the link, not the step, sets the pace, so the copies keep it busy throughout)
+        n_sets = 3
+        sets = [(X, Y)] + [({n: torch.empty_like(X[n]) for n in host_in},
+                            dict(Y, **{n: torch.empty_like(Y[n]) for n in host_out})) for _ in range(n_sets - 1)]
         main = torch.cuda.current_stream(dev)
         up, down = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
 
         def e2e_run(n):
-            comp_done, out_done = [None, None], [None, None]
+            comp_done, out_done = [None] * n_sets, [None] * n_sets
             up.wait_stream(main)
             down.wait_stream(main)
             for i in range(n):
-                b = i % 2
+                b = i % n_sets
                 Xb, Yb = sets[b]
                 with torch.cuda.stream(up):
                     if comp_done[b] is not None:
-                        up.wait_event(comp_done[b])  # step i-2 no longer reads these inputs
+                        up.wait_event(comp_done[b])  # step i - n_sets no longer reads these inputs
                     for nm, t in host_in.items():
                         Xb[nm].copy_(t, non_blocking=True)
                     ready = torch.cuda.Event()
                     ready.record(up)
                 main.wait_event(ready)
                 if out_done[b] is not None:
-                    main.wait_event(out_done[b])  # step i-2's outputs have left
+                    main.wait_event(out_done[b])  # the outputs of step i - n_sets have left
                 step(None, Xb, Yb)
                 comp_done[b] = torch.cuda.Event()
                 comp_done[b].record(main)
@@ -395,8 +396,8 @@ def run_gpu(args, rank, world, local_rank):
         e2e = {"value": world * tokens * K / (ms_e2e / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e / K,
                "h2d_gbs": round(h2d / (h2d_ms / 1e3) / 1e9, 1), "d2h_gbs": round(d2h / (d2h_ms / 1e3) / 1e9, 1),
-               "overlap": "inputs of step i+1 up and outputs of step i-1 down on two copy streams while step i runs"}
-        del host_in, host_out, X2, Y2, sets
+               "overlap": "three buffer sets: inputs of later steps up and outputs of earlier steps down on two copy streams while step i runs"}
+        del host_in, host_out, sets
 
     del X, Y, wss
     torch.cuda.empty_cache()

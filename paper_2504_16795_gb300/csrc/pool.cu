@@ -10,6 +10,8 @@
 namespace hsa {
 namespace {
 
+constexpr int kBatch = 16;
+
 __global__ void __launch_bounds__(256) pool_kernel(const uint4* __restrict__ K, float4* __restrict__ kbar32,
                                                    uint4* __restrict__ kbar16, int L, int Hkv, int d8, int S,
                                                    long long total) {
@@ -25,17 +27,26 @@ __global__ void __launch_bounds__(256) pool_kernel(const uint4* __restrict__ K, 
     float acc[8];
 #pragma unroll
     for (int c = 0; c < 8; ++c) acc[c] = 0.f;
-#pragma unroll 8
-    for (int s = 0; s < S; ++s) {
-      uint4 v = __ldg(src + (long long)s * row_vec);
-      acc[0] = acc[0] + bf16_lo(v.x);
-      acc[1] = acc[1] + bf16_hi(v.x);
-      acc[2] = acc[2] + bf16_lo(v.y);
-      acc[3] = acc[3] + bf16_hi(v.y);
-      acc[4] = acc[4] + bf16_lo(v.z);
-      acc[5] = acc[5] + bf16_hi(v.z);
-      acc[6] = acc[6] + bf16_lo(v.w);
-      acc[7] = acc[7] + bf16_hi(v.w);
+    // kBatch rows in flight per thread: all loads of a batch are issued before
+    // its sums, which still run in token order
+    for (int s0 = 0; s0 < S; s0 += kBatch) {
+      uint4 v[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j)
+        if (s0 + j < S) v[j] = __ldg(src + (long long)(s0 + j) * row_vec);
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        if (s0 + j < S) {
+          acc[0] = acc[0] + bf16_lo(v[j].x);
+          acc[1] = acc[1] + bf16_hi(v[j].x);
+          acc[2] = acc[2] + bf16_lo(v[j].y);
+          acc[3] = acc[3] + bf16_hi(v[j].y);
+          acc[4] = acc[4] + bf16_lo(v[j].z);
+          acc[5] = acc[5] + bf16_hi(v[j].z);
+          acc[6] = acc[6] + bf16_lo(v[j].w);
+          acc[7] = acc[7] + bf16_hi(v[j].w);
+        }
+      }
     }
     const float fs = (float)S;
 #pragma unroll

@@ -122,6 +122,7 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     bwd_chunk_kernel(BwdArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_do,
                      const __grid_constant__ CUtensorMap tmap_dq) {
+  griddep_wait();
   extern __shared__ unsigned char smem_raw[];
   BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
@@ -577,6 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <int D>
 __global__ void __launch_bounds__(256) bwd_delta_kernel(const uint16_t* __restrict__ O, const uint16_t* __restrict__ dO,
                                                         float* __restrict__ delta, long long n_rows, int G) {
+  griddep_wait();
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -607,6 +609,7 @@ __global__ void __launch_bounds__(256) bwd_ds_kernel(const int32_t* __restrict__
                                                      const float* __restrict__ dw, float* __restrict__ ds,
                                                      long long n_rows, int topk, int Nc, int stick, int accumulate,
                                                      unsigned* __restrict__ status) {
+  griddep_wait();
   const long long row = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (row >= n_rows) return;
   const long long p0 = row * topk;
@@ -646,6 +649,7 @@ __global__ void __launch_bounds__(256) sel_dq_kernel(const int32_t* __restrict__
                                                      const float* __restrict__ kbar32, float* __restrict__ dq,
                                                      long long n_rows, int G, int topk, int Nc, int L, int Hkv,
                                                      float scale_sel, unsigned* __restrict__ status) {
+  griddep_wait();
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -695,6 +699,7 @@ __global__ void __launch_bounds__(256) sel_dq_kernel(const int32_t* __restrict__
 template <int D>
 __global__ void __launch_bounds__(256) bwd_qhat_kernel(const uint16_t* __restrict__ q, float* __restrict__ qhat,
                                                        long long n_rows, int G) {
+  griddep_wait();
   constexpr int D8 = D / 8;
   const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (u >= n_rows * D8) return;
@@ -737,6 +742,7 @@ __global__ void __launch_bounds__(D * kDkbarGroups, 2) bwd_stick_dkbar_kernel(co
                                                                            int topk, int Nc, float scale_sel,
                                                                            long long n_slots,
                                                                            unsigned* __restrict__ status) {
+  griddep_wait();
   __shared__ float part[kDkbarGroups][D];
   int c, bg;
   block_key(Nc, (int)(gridDim.x / (unsigned)Nc), c, bg);
@@ -791,6 +797,7 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
                                                            const float* __restrict__ ds,
                                                            const float* __restrict__ kbar32, int L, int Hkv,
                                                            float scale_sel, unsigned* __restrict__ status) {
+  griddep_wait();
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -854,6 +861,7 @@ __global__ void __launch_bounds__(256) bwd_dq_merge_kernel(const int32_t* __rest
 // dK = dV = 0 on the rows of a trailing partial chunk.
 __global__ void zero_tail_kernel(float* __restrict__ dK, float* __restrict__ dV, int B, int L, int tail0,
                                  long long row_elems) {
+  griddep_wait();
   const long long per_b = (long long)(L - tail0) * row_elems;
   const long long total = per_b * B;
   const long long stride = (long long)gridDim.x * blockDim.x;
@@ -905,14 +913,14 @@ cudaError_t launch_dkbar(const Dims& Dm, const void* q, const int32_t* offsets, 
                          float* qhat, float* dK, cudaStream_t st) {
   const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
   cudaError_t e;
-  bwd_qhat_kernel<D><<<(unsigned)((rows * (D / 8) + 255) / 256), 256, 0, st>>>((const uint16_t*)q, qhat, rows, Dm.G);
+  (void)launch_dependent(bwd_qhat_kernel<D>, dim3((unsigned)((rows * (D / 8) + 255) / 256)), dim3(256), 0, st,
+                         (const uint16_t*)q, qhat, rows, Dm.G);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const long long keys = Dm.keys();
   if (keys > 0) {
-    bwd_stick_dkbar_kernel<D><<<(unsigned)keys, D * kDkbarGroups, 0, st>>>(offsets, entries, ds, qhat, dK, Dm.L,
-                                                                           Dm.Hkv, Dm.topk, Dm.Nc, Dm.scale_sel,
-                                                                           Dm.slots(), Dm.status);
+    (void)launch_dependent(bwd_stick_dkbar_kernel<D>, dim3((unsigned)keys), dim3(D * kDkbarGroups), 0, st, offsets,
+                           entries, ds, qhat, dK, Dm.L, Dm.Hkv, Dm.topk, Dm.Nc, Dm.scale_sel, Dm.slots(), Dm.status);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
@@ -937,8 +945,8 @@ cudaError_t run(const Dims& Dm, BwdMode mode, const void* q, const void* K, cons
   float* qhat = full && Dm.stick ? (float*)((char*)ws + lo.qhat) : nullptr;
   cudaError_t e;
   if (delta != nullptr) {  // Δ_t = sum_j w_j dw_j = dO · O feeds the softmax weights' ds inside the chunk kernel
-    bwd_delta_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>((const uint16_t*)O, (const uint16_t*)dO, delta,
-                                                                    rows, Dm.G);
+    (void)launch_dependent(bwd_delta_kernel<D>, dim3((unsigned)((rows + 7) / 8)), dim3(256), 0, st, (const uint16_t*)O,
+                           (const uint16_t*)dO, delta, rows, Dm.G);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
@@ -985,28 +993,28 @@ cudaError_t run(const Dims& Dm, BwdMode mode, const void* q, const void* K, cons
                       !tc::make_group8_tmap(&tdo, dO, (unsigned long long)a.n_rows, D) ||
                       !tc::make_rows_tmap(&tdq, dqpart, (unsigned long long)Dm.slots() * Dm.G, D, 8)))
       return cudaErrorNotSupported;
-    bwd_chunk_kernel<D><<<(unsigned)keys, kThreads, smem, st>>>(a, tq, tdo, tdq);
+    (void)launch_dependent(bwd_chunk_kernel<D>, dim3((unsigned)keys), dim3(kThreads), smem, st, a, tq, tdo, tdq);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (dw_mode) {
-    bwd_ds_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(idx, w, dwb, dsb, rows, Dm.topk, Dm.Nc,
-                                                                   Dm.stick ? 1 : 0, full ? 0 : 1, Dm.status);
+    (void)launch_dependent(bwd_ds_kernel, dim3((unsigned)((rows + 255) / 256)), dim3(256), 0, st, idx, w, dwb, dsb,
+                           rows, Dm.topk, Dm.Nc, Dm.stick ? 1 : 0, full ? 0 : 1, Dm.status);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (full && (e = launch_dkbar<D>(Dm, q, offsets, entries, dsb, qhat, dK, st)) != cudaSuccess) return e;
   }
   const bool sel_term = full && Dm.stick;
-  bwd_dq_merge_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(idx, dqpart, dq, rows, Dm.G, Dm.topk, Dm.Nc,
-                                                                      sel_term ? dsb : nullptr, kbar32, Dm.L, Dm.Hkv,
-                                                                      Dm.scale_sel, Dm.status);
+  (void)launch_dependent(bwd_dq_merge_kernel<D>, dim3((unsigned)((rows + 7) / 8)), dim3(256), 0, st, idx, dqpart, dq,
+                         rows, Dm.G, Dm.topk, Dm.Nc, sel_term ? dsb : nullptr, kbar32, Dm.L, Dm.Hkv, Dm.scale_sel,
+                         Dm.status);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int tail0 = Dm.Nc * kChunk;
   if (tail0 < Dm.L && Dm.B > 0) {
     const long long total = (long long)Dm.B * (Dm.L - tail0) * Dm.Hkv * D;
-    zero_tail_kernel<<<grid_cap((total + 255) / 256, 152LL * 8), 256, 0, st>>>(dK, dV, Dm.B, Dm.L, tail0,
-                                                                               (long long)Dm.Hkv * D);
+    (void)launch_dependent(zero_tail_kernel, dim3(grid_cap((total + 255) / 256, 152LL * 8)), dim3(256), 0, st, dK, dV,
+                           Dm.B, Dm.L, tail0, (long long)Dm.Hkv * D);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
@@ -1022,8 +1030,8 @@ cudaError_t run_select_backward(const Dims& Dm, const void* q_sel, const float* 
   const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
   cudaError_t e;
   if ((e = cudaMemsetAsync(dK_sel, 0, (size_t)rows * D * sizeof(float), st)) != cudaSuccess) return e;
-  sel_dq_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(idx, ds, kbar_sel, dq_sel, rows, Dm.G, Dm.topk, Dm.Nc,
-                                                               Dm.L, Dm.Hkv, Dm.scale_sel, Dm.status);
+  (void)launch_dependent(sel_dq_kernel<D>, dim3((unsigned)((rows + 7) / 8)), dim3(256), 0, st, idx, ds, kbar_sel,
+                         dq_sel, rows, Dm.G, Dm.topk, Dm.Nc, Dm.L, Dm.Hkv, Dm.scale_sel, Dm.status);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return launch_dkbar<D>(Dm, q_sel, offsets, entries, ds, (float*)ws, dK_sel, st);

@@ -180,6 +180,16 @@ __device__ __forceinline__ int warp_emit_selection(unsigned long long mine, int 
   return keff;
 }
 
+// ------------------------------------------------------------------ programmatic dependent launch
+// A kernel launched with launch_dependent (below) is set up while the previous
+// kernel in its stream finishes: griddep_wait returns once that grid has
+// completed and its writes are visible (for a kernel launched the ordinary way
+// it returns at once). Every such kernel calls it before it reads or writes
+// global memory. No kernel signals its dependents early: letting the next
+// grid's blocks onto the SMs during a chunk kernel's last wave made the
+// backward slower.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ------------------------------------------------------------------ async copies / tensor-core fragments
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
@@ -288,7 +298,7 @@ struct DecodeDims {
   unsigned* status = nullptr;  // as in Dims
 };
 // Launch `kernel` as a programmatic dependent of the previous kernel in `st`
-// (it must call tc::griddep_wait before reading that kernel's results).
+// (it must call griddep_wait before it touches global memory).
 template <typename... KArgs, typename... Args>
 cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
                              Args&&... args) {

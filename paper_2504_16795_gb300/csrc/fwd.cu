@@ -81,6 +81,7 @@ struct FwdArgs {
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     fwd_chunk_kernel(FwdArgs a, const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_o) {
+  griddep_wait();
   extern __shared__ unsigned char smem_raw[];
   FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>(smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u));
   constexpr int D8 = D / 8;
@@ -400,6 +401,7 @@ __global__ void __launch_bounds__(1024) fwd_segments_kernel(const int32_t* __res
                                                             int seg_slots, int4* __restrict__ segs,
                                                             int* __restrict__ nseg, long long n_slots,
                                                             unsigned* __restrict__ status) {
+  griddep_wait();
   __shared__ int warp_sum[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int keys = Nc * n_bg;
@@ -448,6 +450,7 @@ __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict_
                                                         const uint16_t* __restrict__ Opart, uint16_t* __restrict__ O,
                                                         float* __restrict__ w, long long n_rows, int Hkv, int G,
                                                         int topk, int Nc, int stick, unsigned* __restrict__ status) {
+  griddep_wait();
   const int lane = threadIdx.x & 31;
   const long long row = (long long)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
   if (row >= n_rows) return;
@@ -528,8 +531,8 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     int4* segs = (int4*)((char*)ws + lo.segs);
     int* nseg = (int*)((char*)ws + lo.nseg);
     const int seg_slots = kSegTiles * (kRows / Dm.G);
-    fwd_segments_kernel<<<1, 1024, 0, st>>>(offsets, Dm.Nc, Dm.B * Dm.Hkv, seg_slots, segs, nseg, Dm.slots(),
-                                            Dm.status);
+    (void)launch_dependent(fwd_segments_kernel, dim3(1), dim3(1024), 0, st, offsets, Dm.Nc, Dm.B * Dm.Hkv, seg_slots,
+                           segs, nseg, Dm.slots(), Dm.status);
     note_launches(1);
     cudaError_t e0 = cudaGetLastError();
     if (e0 != cudaSuccess) return e0;
@@ -563,13 +566,13 @@ cudaError_t run(const Dims& Dm, const void* q, const void* K, const void* V, con
     if (a.use_tma && !tc::make_group8_tmap(&tq, q, (unsigned long long)a.n_rows, D)) return cudaErrorNotSupported;
     if (a.use_tma && !tc::make_group8_tmap(&to, Opart, (unsigned long long)Dm.slots() * Dm.G, D))
       return cudaErrorNotSupported;
-    fwd_chunk_kernel<D><<<(unsigned)lo.max_segs, kThreads, smem, st>>>(a, tq, to);
+    (void)launch_dependent(fwd_chunk_kernel<D>, dim3((unsigned)lo.max_segs), dim3(kThreads), smem, st, a, tq, to);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   const long long rows = (long long)Dm.B * Dm.L * Dm.Hkv;
-  fwd_merge_kernel<D><<<(unsigned)((rows + 7) / 8), 256, 0, st>>>(s_sel, idx, Opart, (uint16_t*)O, w, rows, Dm.Hkv,
-                                                                  Dm.G, Dm.topk, Dm.Nc, Dm.stick ? 1 : 0, Dm.status);
+  (void)launch_dependent(fwd_merge_kernel<D>, dim3((unsigned)((rows + 7) / 8)), dim3(256), 0, st, s_sel, idx, Opart,
+                         (uint16_t*)O, w, rows, Dm.Hkv, Dm.G, Dm.topk, Dm.Nc, Dm.stick ? 1 : 0, Dm.status);
   note_launches(1);
   return cudaGetLastError();
 }

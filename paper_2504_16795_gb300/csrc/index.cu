@@ -40,6 +40,7 @@ struct KeyMap {
 __global__ void __launch_bounds__(kThreads) radix_hist_kernel(KeyMap km, const uint32_t* __restrict__ keys_in,
                                                               long long n, int shift, uint32_t* __restrict__ hist,
                                                               int n_tiles) {
+  griddep_wait();
   __shared__ uint32_t h[256];
   h[threadIdx.x] = 0;
   __syncthreads();
@@ -65,6 +66,7 @@ __global__ void __launch_bounds__(kThreads) radix_scatter_kernel(KeyMap km, cons
                                                                  int shift, const uint32_t* __restrict__ base_off,
                                                                  int n_tiles, uint32_t* __restrict__ keys_out,
                                                                  int32_t* __restrict__ vals_out) {
+  griddep_wait();
   __shared__ uint32_t run[256];
   __shared__ uint32_t cnt[kThreads / 32][256];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -108,6 +110,7 @@ __global__ void __launch_bounds__(kThreads) radix_scatter_kernel(KeyMap km, cons
 // keys in (key[i-1], key[i]]; position n closes the range up to n_keys.
 __global__ void offsets_from_sorted_kernel(const uint32_t* __restrict__ sorted, long long n, long long n_keys,
                                            int32_t* __restrict__ offsets) {
+  griddep_wait();
   const long long stride = (long long)gridDim.x * blockDim.x;
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i <= n; i += stride) {
     const long long cur = i < n ? (long long)sorted[i] : n_keys;
@@ -146,6 +149,7 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* w
 
 __global__ void __launch_bounds__(kScanThreads) scan_tiles_kernel(uint32_t* __restrict__ a, long long n,
                                                                   uint32_t* __restrict__ tile_sums) {
+  griddep_wait();
   __shared__ uint32_t ws[32];
   const long long base = (long long)blockIdx.x * kScanTile + (long long)threadIdx.x * kScanItems;
   uint32_t v[kScanItems], s = 0;
@@ -166,6 +170,7 @@ __global__ void __launch_bounds__(kScanThreads) scan_tiles_kernel(uint32_t* __re
 
 __global__ void __launch_bounds__(kScanThreads) add_tile_base_kernel(uint32_t* __restrict__ a, long long n,
                                                                      const uint32_t* __restrict__ tile_base) {
+  griddep_wait();
   const long long base = (long long)blockIdx.x * kScanTile + (long long)threadIdx.x * kScanItems;
   const uint32_t add = tile_base[blockIdx.x];
 #pragma unroll
@@ -177,16 +182,16 @@ __global__ void __launch_bounds__(kScanThreads) add_tile_base_kernel(uint32_t* _
 cudaError_t exclusive_scan(uint32_t* a, long long n, uint32_t* tile_sums, cudaStream_t st) {
   const long long tiles = (n + kScanTile - 1) / kScanTile;
   if (tiles <= 1) {
-    scan_tiles_kernel<<<1, kScanThreads, 0, st>>>(a, n, nullptr);
+    (void)launch_dependent(scan_tiles_kernel, dim3(1), dim3(kScanThreads), 0, st, a, n, nullptr);
     note_launches(1);
     return cudaGetLastError();
   }
   if (tiles > kScanTile) return cudaErrorInvalidValue;
-  scan_tiles_kernel<<<(unsigned)tiles, kScanThreads, 0, st>>>(a, n, tile_sums);
+  (void)launch_dependent(scan_tiles_kernel, dim3((unsigned)tiles), dim3(kScanThreads), 0, st, a, n, tile_sums);
   note_launches(1);
-  scan_tiles_kernel<<<1, kScanThreads, 0, st>>>(tile_sums, tiles, nullptr);
+  (void)launch_dependent(scan_tiles_kernel, dim3(1), dim3(kScanThreads), 0, st, tile_sums, tiles, nullptr);
   note_launches(1);
-  add_tile_base_kernel<<<(unsigned)tiles, kScanThreads, 0, st>>>(a, n, tile_sums);
+  (void)launch_dependent(add_tile_base_kernel, dim3((unsigned)tiles), dim3(kScanThreads), 0, st, a, n, tile_sums);
   note_launches(1);
   return cudaGetLastError();
 }
@@ -248,19 +253,21 @@ cudaError_t launch_index(const Dims& D, const int32_t* idx, int32_t* offsets, in
     const bool last = pass == lo.passes - 1;
     uint32_t* kout = keys_buf[pass & 1];
     int32_t* vout = last ? entries : vals_buf[pass & 1];
-    radix_hist_kernel<<<(unsigned)lo.n_tiles, kThreads, 0, st>>>(km, kin, lo.n, 8 * pass, hist, (int)lo.n_tiles);
+    (void)launch_dependent(radix_hist_kernel, dim3((unsigned)lo.n_tiles), dim3(kThreads), 0, st, km, kin, lo.n,
+                           8 * pass, hist, (int)lo.n_tiles);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if ((e = exclusive_scan(hist, lo.hist_len, sums, st)) != cudaSuccess) return e;
-    radix_scatter_kernel<<<(unsigned)lo.n_tiles, kThreads, 0, st>>>(km, kin, vin, lo.n, 8 * pass, hist,
-                                                                   (int)lo.n_tiles, kout, vout);
+    (void)launch_dependent(radix_scatter_kernel, dim3((unsigned)lo.n_tiles), dim3(kThreads), 0, st, km, kin, vin, lo.n,
+                           8 * pass, hist, (int)lo.n_tiles, kout, vout);
     note_launches(1);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     kin = kout;
     vin = vout;
   }
   // offsets from the sorted keys of the last pass
-  offsets_from_sorted_kernel<<<grid_cap((lo.n + 256) / 256, 152LL * 8), 256, 0, st>>>(kin, lo.n, lo.keys, offsets);
+  (void)launch_dependent(offsets_from_sorted_kernel, dim3(grid_cap((lo.n + 256) / 256, 152LL * 8)), dim3(256), 0, st,
+                         kin, lo.n, lo.keys, offsets);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -15,6 +15,7 @@ constexpr int kBatch = 16;
 __global__ void __launch_bounds__(256) pool_kernel(const uint4* __restrict__ K, float4* __restrict__ kbar32,
                                                    uint4* __restrict__ kbar16, int L, int Hkv, int d8, int S,
                                                    long long total) {
+  griddep_wait();
   const long long stride = (long long)gridDim.x * blockDim.x;
   const int Nc = L / S;
   const long long row_vec = (long long)Hkv * d8;  // uint4 per token row
@@ -71,7 +72,8 @@ cudaError_t launch_pool(const Dims& D, const void* K, float* kbar32, void* kbar1
   const long long total = (long long)D.B * D.Nc * D.Hkv * d8;
   if (total == 0) return cudaSuccess;
   const int grid = grid_cap((total + 255) / 256, 152LL * 16);
-  pool_kernel<<<grid, 256, 0, st>>>((const uint4*)K, (float4*)kbar32, (uint4*)kbar16, D.L, D.Hkv, d8, D.S, total);
+  (void)launch_dependent(pool_kernel, dim3(grid), dim3(256), 0, st, (const uint4*)K, (float4*)kbar32, (uint4*)kbar16,
+                         D.L, D.Hkv, d8, D.S, total);
   note_launches(1);
   return cudaGetLastError();
 }

@@ -272,7 +272,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
-  tc::griddep_wait();  // decode: the query rows and norms of the kernel before
+  tc::griddep_wait();  // the kernel before: the query rows and norms (decode), the bf16 summaries (prefill)
   const uint32_t tmem = sm.tmem_base;
   const uint32_t abase = smem_u32(sm.A), ubase = smem_u32(sm.B);
   constexpr uint32_t kStageBytes = kCt * D * 2;
@@ -639,6 +639,7 @@ template <int D>
 __global__ void __launch_bounds__(256) sel_qhat_kernel(const uint16_t* __restrict__ q, uint16_t* __restrict__ qh16,
                                                        float* __restrict__ qh32t, float* __restrict__ qn, int L,
                                                        int Lp, int Hq, int Hkv, int G) {
+  griddep_wait();
   __shared__ float qs[32][D + 1];
   constexpr int D8 = D / 8;
   const int bg = blockIdx.y;
@@ -694,6 +695,7 @@ template <int D>
 __global__ void __launch_bounds__(256) sel_kbar_kernel(const float* __restrict__ kbar32, uint16_t* __restrict__ kb16,
                                                        float* __restrict__ kn, unsigned* __restrict__ ktmax,
                                                        long long rows, int Nc, int Ncp, int Hkv, int c0, int Nrow) {
+  griddep_wait();
   constexpr int D8 = D / 8;
   const long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   const long long row = u / D8;  // input row (b, i, g)
@@ -739,6 +741,7 @@ __global__ void __launch_bounds__(kExactWarps * 32) sel_exact_rows_kernel(
     const float* __restrict__ qh32t, const float* __restrict__ kbar32, const unsigned* __restrict__ nflag,
     const int32_t* __restrict__ flags, int32_t* __restrict__ idx, float* __restrict__ s_sel, int L, int Lp, int Hkv,
     int Nc, int topk, float scale_sel) {
+  griddep_wait();
   extern __shared__ __align__(16) unsigned char ex_smem[];
   float* stage_all = reinterpret_cast<float*>(ex_smem);                    // [warps][32 rows][D]
   float* qsh = stage_all + kExactWarps * 32 * D;                             // [D]
@@ -1148,13 +1151,13 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
   if ((e = cudaMemsetAsync(ktmax, 0, lo.flags - lo.ktmax, st)) != cudaSuccess) return e;
   constexpr int D8 = DD / 8;
   const int Lp = padded_tokens(Dm);
-  sel_qhat_kernel<DD><<<dim3((unsigned)((Dm.L + 31) / 32), (unsigned)BH), 256, 0, st>>>((const uint16_t*)q, qh16, qh32,
-                                                                                      qn, Dm.L, Lp, Dm.Hq, Dm.Hkv, Dm.G);
+  (void)launch_dependent(sel_qhat_kernel<DD>, dim3((unsigned)((Dm.L + 31) / 32), (unsigned)BH), dim3(256), 0, st,
+                         (const uint16_t*)q, qh16, qh32, qn, Dm.L, Lp, Dm.Hq, Dm.Hkv, Dm.G);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int Ncp = padded_chunks(Dm);
-  sel_kbar_kernel<DD><<<(unsigned)((krows * D8 + 255) / 256), 256, 0, st>>>(kbar32, kb16, kn, ktmax, krows, Dm.Nc,
-                                                                           Ncp, Dm.Hkv, 0, Dm.Nc);
+  (void)launch_dependent(sel_kbar_kernel<DD>, dim3((unsigned)((krows * D8 + 255) / 256)), dim3(256), 0, st, kbar32,
+                         kb16, kn, ktmax, krows, Dm.Nc, Ncp, Dm.Hkv, 0, Dm.Nc);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
@@ -1191,15 +1194,16 @@ cudaError_t run_tc(const Dims& Dm, const void* q, const float* kbar32, int32_t* 
                                 (int)smem)) != cudaSuccess)
     return e;
   const long long blocks = (long long)a.n_qt * BH;
-  sel_tc_kernel<DD, KT, false><<<(unsigned)blocks, kThreads, smem, st>>>(a, tq, tk, tq32t);
+  (void)launch_dependent(sel_tc_kernel<DD, KT, false>, dim3((unsigned)blocks), dim3(kThreads), smem, st, a, tq, tk,
+                         tq32t);
   note_launches(1);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const size_t ex_smem = ((size_t)kExactWarps * 32 * DD + DD) * 4 + (size_t)kExactWarps * 32 * 8;
   if ((e = cudaFuncSetAttribute(sel_exact_rows_kernel<DD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)ex_smem)) != cudaSuccess)
     return e;
-  sel_exact_rows_kernel<DD><<<152, kExactWarps * 32, ex_smem, st>>>(qh32, kbar32, nflag, flags, idx, s_sel, Dm.L, Lp,
-                                                                    Dm.Hkv, Dm.Nc, Dm.topk, Dm.scale_sel);
+  (void)launch_dependent(sel_exact_rows_kernel<DD>, dim3(152), dim3(kExactWarps * 32), ex_smem, st, qh32, kbar32, nflag,
+                         flags, idx, s_sel, Dm.L, Lp, Dm.Hkv, Dm.Nc, Dm.topk, Dm.scale_sel);
   note_launches(1);
   return cudaGetLastError();
 }
@@ -1366,13 +1370,13 @@ cudaError_t launch_index_rows(const DecodeDims& Dm, const float* kbar32, void* i
   const long long krows = (c1 - c0) * Dm.Hkv;  // input rows (i, g) of the one-batch memory, chunk c0 first
   const float* src = kbar32 + c0 * Dm.Hkv * Dm.d;
   if (Dm.d == 64)
-    sel_kbar_kernel<64><<<(unsigned)((krows * 8 + 255) / 256), 256, 0, st>>>(
-        src, (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows,
-        (int)(c1 - c0), Ncp, Dm.Hkv, (int)c0, (int)Dm.cap);
+    (void)launch_dependent(sel_kbar_kernel<64>, dim3((unsigned)((krows * 8 + 255) / 256)), dim3(256), 0, st, src,
+                           (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows,
+                           (int)(c1 - c0), Ncp, Dm.Hkv, (int)c0, (int)Dm.cap);
   else
-    sel_kbar_kernel<128><<<(unsigned)((krows * 16 + 255) / 256), 256, 0, st>>>(
-        src, (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows,
-        (int)(c1 - c0), Ncp, Dm.Hkv, (int)c0, (int)Dm.cap);
+    (void)launch_dependent(sel_kbar_kernel<128>, dim3((unsigned)((krows * 16 + 255) / 256)), dim3(256), 0, st, src,
+                           (uint16_t*)(base + ix.kb16), (float*)(base + ix.kn), (unsigned*)(base + ix.ktmax), krows,
+                           (int)(c1 - c0), Ncp, Dm.Hkv, (int)c0, (int)Dm.cap);
   note_launches(1);
   return cudaGetLastError();
 }

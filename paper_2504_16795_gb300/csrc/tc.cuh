@@ -21,12 +21,10 @@ namespace tc {
 // broken pipeline ends the kernel instead of hanging the GPU.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
 
-// Programmatic dependent launch: a kernel launched as a dependent of the
-// previous kernel in its stream waits here until that grid has completed and
-// its writes are visible; for a kernel launched the ordinary way it returns at
-// once. The work before it (barrier setup, tensor-memory allocation) overlaps
-// the previous grid's tail.
-__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Programmatic dependent launch (common.cuh): the work a kernel does before
+// griddep_wait (barrier setup, tensor-memory allocation) overlaps the previous
+// grid's tail.
+using ::hsa::griddep_wait;
 
 __device__ __forceinline__ unsigned long long globaltimer() {
   unsigned long long t;

@@ -220,8 +220,10 @@ hsa_status_t hsa_select_topk(const hsa_shape_t* shape, const void* q, const floa
  *           entries[offsets[k] .. offsets[k+1]).
  *   entries [B*L*Hkv*topk] int32, output (capacity): the flat slot index
  *           p = ((b*L + t)*Hkv + g)*topk + j of idx, in increasing p (so in
- *           increasing token order) within each key.
- * Deterministic (a stable radix sort); needs workspace HSA_OP_INDEX.
+ *           increasing token order) within each key. Positions from
+ *           offsets[B*Hkv*(L/S)] on are unspecified.
+ * Deterministic (a stable counting sort when Hkv*(L/S) <= 4096, else a stable
+ * radix sort); needs workspace HSA_OP_INDEX.
  */
 hsa_status_t hsa_build_index(const hsa_shape_t* shape, const int32_t* idx, int32_t* offsets, int32_t* entries,
                              void* ws, size_t ws_bytes, cudaStream_t stream);

@@ -232,7 +232,12 @@ def test_workspace_sizes_scale_with_the_problem(lib):
     # the forward keeps one bf16 partial per slot and head, and the list of slot-list segments
     assert hsa.workspace_size(hsa.HSA_OP_FORWARD, s) >= hsa.status_bytes() + slots * 8 * 128 * 2
     assert hsa.workspace_size(hsa.HSA_OP_BACKWARD, s) >= slots * 8 * 128 * 2
-    assert hsa.workspace_size(hsa.HSA_OP_INDEX, s) >= slots * 16
+    # the index: with Hkv * Nc <= 4096 keys per batch row, one count per (key, tile of 8192 slots)
+    n_tiles = -(-32768 // (8192 // (4 * 8)))
+    assert hsa.workspace_size(hsa.HSA_OP_INDEX, s) >= 2 * 4 * 512 * n_tiles * 4
+    # with more keys per row, the radix sort's two key and value buffers
+    long_row = shape(B=1, L=1 << 20, Hq=16, Hkv=1, topk=16)
+    assert hsa.workspace_size(hsa.HSA_OP_INDEX, long_row) >= (1 << 20) * 16 * 16
     assert hsa.workspace_size(hsa.HSA_OP_FORWARD, shape(d=96)) == 0
 
 

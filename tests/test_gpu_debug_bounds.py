@@ -5,8 +5,9 @@ It runs in a child process that loads _build_debug/libhsa_debug.so:
   library's bit for bit, and hsa_check reports HSA_OK.
 - With a planted out-of-range index, the call still completes, and the next
   hsa_check reports HSA_ERR_BOUNDS. The planted indices are:
-  a chunk id past the sequence in idx; an inverted pair of offsets (a list
-  that ends before it starts); a slot id past the end in entries.
+  a chunk id past the sequence in idx (seen by the forward, the backward and
+  the inverse index); an inverted pair of offsets (a list that ends before it
+  starts); a slot id past the end in entries.
 
 Every planted value is harmless even to the normal build. Out-of-range chunk
 ids count as no selection; an inverted list is empty; with G = 8 the query
@@ -59,9 +60,12 @@ def run_case(lib_path, case):
     hsa.forward(shape, X["q"], X["K"], X["V"], idx, fwd["s_sel"], offsets, entries, O, wts, ws=wss.forward)
     dq, dK, dV = hsa.backward(shape, X["q"], X["K"], X["V"], fwd["kbar32"], idx, wts, O, X["dO"], offsets, entries,
                               ws=wss.backward)
+    # the inverse index of the (possibly planted) selection, in its own workspace
+    hsa.check(wss.index)
+    hsa.build_index(shape, idx, ws=wss.index)
     torch.cuda.synchronize()
     codes = {}
-    for name in ("forward", "backward"):
+    for name in ("forward", "backward", "index"):
         ws = getattr(wss, name)
         codes[name] = int(hsa.load().hsa_check(ws.data_ptr(), ws.numel(), None))
     h = hashlib.sha256()
@@ -95,9 +99,9 @@ def debug_results():
 def test_debug_build_matches_the_normal_build_on_clean_inputs(debug_results):
     hsa.build()
     codes, digest = run_case(None, "clean")
-    assert codes == {"forward": 0, "backward": 0}
+    assert codes == {"forward": 0, "backward": 0, "index": 0}
     dbg_codes, dbg_digest = debug_results["clean"]
-    assert dbg_codes == {"forward": 0, "backward": 0}
+    assert dbg_codes == {"forward": 0, "backward": 0, "index": 0}
     assert dbg_digest == digest
 
 
@@ -109,3 +113,5 @@ def test_debug_build_reports_planted_indices(debug_results, case):
     # kernel reads offsets and entries) and the backward (the same inputs)
     assert codes["forward"] == BOUNDS, codes
     assert codes["backward"] == BOUNDS, codes
+    # the index reads idx alone: only a chunk id past the sequence reaches it
+    assert codes["index"] == (BOUNDS if case == "idx" else 0), codes

@@ -149,7 +149,7 @@ struct CountGeom {
   __device__ __forceinline__ int tile_slots(int tile) const {
     return min(tile_tokens, L - tile * tile_tokens) * Hkv * topk;
   }
-  // the row-local key of slot p (the tile's base excluded), -1 if not listed
+  // the key of slot p within its batch row (g * Nc + chunk), -1 if the slot is not listed
   __device__ __forceinline__ int local_key(const int32_t* idx, long long p, unsigned* status) const {
     const int c = idx[p];
     if (c >= 0) bounds_ok(c, 0, Nc, status);

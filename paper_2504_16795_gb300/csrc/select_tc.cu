@@ -336,6 +336,7 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     // through shared memory (named barrier 1), so both hold the row's bound.
     // Each keeps its own buffer, and thread r exports both.
     const bool pair = DEC && a.Bq <= kTok / 2 && gsz >= 8;
+    constexpr bool kBothHalves = !DEC && KT > 8;
     const int r = tid;
     const int t = t0 + (pair ? (r & (kTok / 2 - 1)) : r);
     const bool row_ok = DEC ? t < a.Bq : t < a.L;
@@ -362,6 +363,42 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
     auto scan_barrier = [&]() { asm volatile("barrier.sync 1, 128;" ::: "memory"); };
 
     const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    // The candidates of a half tile: each set bit c of m (a column whose score
+    // reaches thr - the tile's largest eps) whose own upper bound reaches thr
+    // enters the buffer, as chunk cbase + c.
+    auto insert_hits = [&](uint32_t m, const float (&xh)[32], const float* knh, int cbase, float thr) {
+      while (m) {
+        const int c = __ffs(m) - 1;
+        m &= m - 1;
+        const float xc = pick32(xh, c);
+        const float e = fmaf(cq, knh[c], kEpsAbs);
+        if (xc + e >= thr) {
+          const float lv = xc - e, uv = xc + e;
+          int slot = cnt;
+          if (cnt < kBuf) {
+            ++cnt;
+          } else {  // full: replace the entry with the smallest upper bound, if smaller
+            float um = sm.bu[0][r];
+            slot = 0;
+            for (int j = 1; j < kBuf; ++j) {
+              const float uj = sm.bu[j][r];
+              if (uj < um) um = uj, slot = j;
+            }
+            if (uv > um) {
+              u_drop = fmaxf(u_drop, um);
+            } else {
+              u_drop = fmaxf(u_drop, uv);
+              slot = -1;
+            }
+          }
+          if (slot >= 0) {
+            sm.bl[slot][r] = lv;
+            sm.bu[slot][r] = uv;
+            sm.bi[slot][r] = cbase + c;
+          }
+        }
+      }
+    };
     bool dead = false;  // a wait gave up; in pair mode the warp still meets every barrier
     for (int it = 0; it < n_iter; ++it) {
       const bool sweep = it < ntiles;     // first visit: the bound's terms
@@ -378,6 +415,66 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       if (!dead) tc::fence_after_sync();
       const float* knt = sm.knt[kq];
       const float emax = dead ? 0.f : fmaf(cq, knt[kCt], kEpsAbs);  // the tile's largest eps_i
+      if constexpr (kBothHalves) {
+        // Long rows (k > 8: one block per SM, registers to spare): both halves
+        // of the tile leave tensor memory together and go through the sweep and
+        // the candidate mask side by side, so their dependent chains interleave.
+        // Half 0's candidates are tested against a bound that already holds half
+        // 1's terms: still at most lam_lo, so the collection stays complete.
+        float x0[32], x1[32];
+        const int c0 = n * kCt, lim0 = vis - c0, lim1 = lim0 - 32;
+        __syncwarp();
+        tc::tmem_ld32(tmem + lane_base + ab * kCt, x0);
+        tc::tmem_ld32(tmem + lane_base + ab * kCt + 32, x1);
+        tc::tmem_wait_ld();
+        if (sweep && lim0 > 0) {
+          if (lim0 < 2 * 32) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              x0[c] = c < lim0 ? x0[c] : -INFINITY;
+              x1[c] = c < lim1 ? x1[c] : -INFINITY;
+            }
+          }
+          if (gsz == 1) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) push(x0[c] - emax);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) push(x1[c] - emax);
+          } else {
+            float g0[4], g1[4];  // maxima of the groups of 8 columns
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              g0[j] = fmaxf(fmaxf(fmaxf(x0[8 * j], x0[8 * j + 1]), fmaxf(x0[8 * j + 2], x0[8 * j + 3])),
+                            fmaxf(fmaxf(x0[8 * j + 4], x0[8 * j + 5]), fmaxf(x0[8 * j + 6], x0[8 * j + 7])));
+              g1[j] = fmaxf(fmaxf(fmaxf(x1[8 * j], x1[8 * j + 1]), fmaxf(x1[8 * j + 2], x1[8 * j + 3])),
+                            fmaxf(fmaxf(x1[8 * j + 4], x1[8 * j + 5]), fmaxf(x1[8 * j + 6], x1[8 * j + 7])));
+            }
+            if (gsz == 8) {
+#pragma unroll
+              for (int j = 0; j < 4; ++j) push(g0[j] - emax);
+#pragma unroll
+              for (int j = 0; j < 4; ++j) push(g1[j] - emax);
+            } else {
+              push(fmaxf(fmaxf(g0[0], g0[1]), fmaxf(g0[2], g0[3])) - emax);
+              push(fmaxf(fmaxf(g1[0], g1[1]), fmaxf(g1[2], g1[3])) - emax);
+            }
+          }
+        }
+        if (collect && lim0 > 0) {
+          const float thr = sweep ? bm[KT - 1] : lam_lo;
+          const float lo = thr - emax;
+          uint32_t m0 = 0, m1 = 0;
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            m0 |= x0[c] >= lo ? (1u << c) : 0u;
+            m1 |= x1[c] >= lo ? (1u << c) : 0u;
+          }
+          if (lim0 < 32) m0 &= (1u << lim0) - 1u;
+          if (lim1 < 32) m1 = lim1 > 0 ? m1 & ((1u << lim1) - 1u) : 0u;
+          insert_hits(m0, x0, knt, c_begin + c0, thr);
+          insert_hits(m1, x1, knt + 32, c_begin + c0 + 32, thr);
+        }
+      } else {
 #pragma unroll 1
       for (int h = h_begin; h < h_end; ++h) {
         float x[32];
@@ -433,39 +530,10 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
 #pragma unroll
           for (int c = 0; c < 32; ++c) m |= x[c] >= lo ? (1u << c) : 0u;
           if (lim < 32) m &= (1u << lim) - 1u;
-          while (m) {
-            const int c = __ffs(m) - 1;
-            m &= m - 1;
-            const float xc = pick32(x, c);
-            const float e = fmaf(cq, knt[h * 32 + c], kEpsAbs);
-            if (xc + e >= thr) {
-              const float lv = xc - e, uv = xc + e;
-              int slot = cnt;
-              if (cnt < kBuf) {
-                ++cnt;
-              } else {  // full: replace the entry with the smallest upper bound, if smaller
-                float um = sm.bu[0][r];
-                slot = 0;
-                for (int j = 1; j < kBuf; ++j) {
-                  const float uj = sm.bu[j][r];
-                  if (uj < um) um = uj, slot = j;
-                }
-                if (uv > um) {
-                  u_drop = fmaxf(u_drop, um);
-                } else {
-                  u_drop = fmaxf(u_drop, uv);
-                  slot = -1;
-                }
-              }
-              if (slot >= 0) {
-                sm.bl[slot][r] = lv;
-                sm.bu[slot][r] = uv;
-                sm.bi[slot][r] = c_begin + c0 + c;
-              }
-            }
-          }
+          insert_hits(m, x, knt + h * 32, c_begin + c0, thr);
         }
       }
+      }  // one half at a time
       if (!dead) {
         tc::fence_before_sync();
         tc::mbar_arrive(bar(BAR_ACC_EMPTY + ab));

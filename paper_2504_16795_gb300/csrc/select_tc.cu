@@ -92,7 +92,12 @@ struct SelTcSmem {
   uint32_t tmem_base;
   int abort_flag;
 };
-// the rescoring stages 32 fp32 K̄ rows per scan warp in A and B
+// the rescoring stages 32 fp32 K̄ rows per scan warp in A and B (with K_T = 16, a second buffer
+// per warp: two more in A and B, two in bu)
+static_assert(sizeof(SelTcSmem<128, 16>::A) + sizeof(SelTcSmem<128, 16>::B) >= 6 * 32 * 128 * 4, "staging");
+static_assert(sizeof(SelTcSmem<64, 16>::A) + sizeof(SelTcSmem<64, 16>::B) >= 6 * 32 * 64 * 4, "staging");
+static_assert(sizeof(SelTcSmem<128, 16>::bu) >= 2 * 32 * 128 * 4, "staging");
+static_assert(sizeof(SelTcSmem<64, 16>::bu) >= 2 * 32 * 64 * 4, "staging");
 static_assert(sizeof(SelTcSmem<128, 8>::A) + sizeof(SelTcSmem<128, 8>::B) >= 4 * 32 * 128 * 4, "staging");
 static_assert(sizeof(SelTcSmem<64, 8>::A) + sizeof(SelTcSmem<64, 8>::B) >= 4 * 32 * 64 * 4, "staging");
 // two blocks per SM with K_T = 8 (228 KB of shared memory, 1 KB reserved per block)
@@ -145,7 +150,7 @@ __device__ __forceinline__ float pick32(const float (&x)[32], int c) {
 // with float4 j at slot j ^ (l & 7), so that the lanes' reads of their own
 // rows below hit distinct banks.
 template <int D>
-__device__ __forceinline__ void stage_kbar_rows(uint32_t stage, const float* kb, long long row_stride, int c,
+__device__ __forceinline__ void issue_kbar_rows(uint32_t stage, const float* kb, long long row_stride, int c,
                                                 int lane) {
 #pragma unroll 4
   for (int l = 0; l < 32; ++l) {
@@ -154,6 +159,11 @@ __device__ __forceinline__ void stage_kbar_rows(uint32_t stage, const float* kb,
       cp_async16(stage + (uint32_t)(l * D + ((lane ^ (l & 7)) << 2)) * 4u, kb + (long long)cl * row_stride + lane * 4);
   }
   cp_async_commit();
+}
+template <int D>
+__device__ __forceinline__ void stage_kbar_rows(uint32_t stage, const float* kb, long long row_stride, int c,
+                                                int lane) {
+  issue_kbar_rows<D>(stage, kb, row_stride, c, lane);
   cp_async_wait<0>();
   __syncwarp();
 }
@@ -632,21 +642,54 @@ __global__ void __launch_bounds__(kThreads, SelCfg<KT>::kBlocksPerSm)
       const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
       const float* kb = a.kbar32 + ((long long)b * a.Nc * a.Hkv + g) * D;
       const uint32_t stage = abase + (uint32_t)(warp * 32 * D) * 4u;  // 32 rows per warp inside A and B
-      for (int base = 0; base < total; base += 32) {
+      // lane l's entry of the round starting at base: its row (owning lane src), index j, chunk c (-1: none)
+      auto locate = [&](int base, int& src, int& j, int& c) {
         const int e = base + lane;
-        int src = 0;  // the owning lane: the number of lanes whose prefix ends at or before e
+        src = 0;  // the owning lane: the number of lanes whose prefix ends at or before e
 #pragma unroll
         for (int step = 16; step >= 1; step >>= 1) {
           const int v = __shfl_sync(0xFFFFFFFFu, incl, src + step - 1);
           if (v <= e) src += step;
         }
-        const int j = e - (__shfl_sync(0xFFFFFFFFu, incl, src) - __shfl_sync(0xFFFFFFFFu, my_n, src));
-        const int rs = warp * 32 + src;
-        const int c = e < total ? sm.bi[j][rs] : -1;
-        stage_kbar_rows<D>(stage, kb, (long long)a.Hkv * D, c, lane);
-        const float v = staged_dot_from<D>(qr, src, stage, lane);
-        if (c >= 0) sm.bl[j][rs] = v * a.scale_sel;
-        __syncwarp();
+        j = e - (__shfl_sync(0xFFFFFFFFu, incl, src) - __shfl_sync(0xFFFFFFFFu, my_n, src));
+        c = e < total ? sm.bi[j][warp * 32 + src] : -1;
+      };
+      if constexpr (!DEC && KT > 8) {
+        // One block per SM leaves room for a second staging buffer per warp (the
+        // rest of A and B for warps 0-1, the freed upper bounds for warps 2-3):
+        // the next round's K̄ rows are in flight while this round's chains run.
+        const uint32_t stage1 = warp < 2 ? abase + (uint32_t)((4 + warp) * 32 * D) * 4u
+                                         : smem_u32(&sm.bu[0][0]) + (uint32_t)((warp - 2) * 32 * D) * 4u;
+        int src, j, c;
+        locate(0, src, j, c);
+        if (total > 0) issue_kbar_rows<D>(stage, kb, (long long)a.Hkv * D, c, lane);
+        for (int base = 0, round = 0; base < total; base += 32, ++round) {
+          const uint32_t cur = (round & 1) ? stage1 : stage;
+          int src_n = 0, j_n = 0, c_n = -1;
+          if (base + 32 < total) {
+            locate(base + 32, src_n, j_n, c_n);
+            issue_kbar_rows<D>((round & 1) ? stage : stage1, kb, (long long)a.Hkv * D, c_n, lane);
+            cp_async_wait<1>();
+          } else {
+            cp_async_wait<0>();
+          }
+          __syncwarp();
+          const float v = staged_dot_from<D>(qr, src, cur, lane);
+          if (c >= 0) sm.bl[j][warp * 32 + src] = v * a.scale_sel;
+          __syncwarp();  // the buffer is refilled two rounds on
+          src = src_n;
+          j = j_n;
+          c = c_n;
+        }
+      } else {
+        for (int base = 0; base < total; base += 32) {
+          int src, j, c;
+          locate(base, src, j, c);
+          stage_kbar_rows<D>(stage, kb, (long long)a.Hkv * D, c, lane);
+          const float v = staged_dot_from<D>(qr, src, stage, lane);
+          if (c >= 0) sm.bl[j][warp * 32 + src] = v * a.scale_sel;
+          __syncwarp();
+        }
       }
     }
     if (live) {

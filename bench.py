@@ -672,14 +672,18 @@ def run_prefill_1m(args, dev, pk, hsa, barrier, max_over_ranks):
         n = hsa.workspace_size(op, shape)
         return torch.empty(n, dtype=torch.uint8, device=dev) if n else None
 
-    wsel, widx, wfwd = ws(hsa.HSA_OP_SELECT), ws(hsa.HSA_OP_INDEX), ws(hsa.HSA_OP_FORWARD)
+    # pooling and selection alone (profiling captures that must keep the device memory small)
+    select_only = getattr(args, "select_only", False)
+    wsel = ws(hsa.HSA_OP_SELECT)
+    widx, wfwd = (None, None) if select_only else (ws(hsa.HSA_OP_INDEX), ws(hsa.HSA_OP_FORWARD))
     Y = dict(kbar32=torch.empty((w.B, w.Nc, w.Hkv, w.d), dtype=f32, device=dev),
              kbar16=torch.empty((w.B, w.Nc, w.Hkv, w.d), dtype=torch.bfloat16, device=dev),
-             idx=torch.empty(sel, dtype=i32, device=dev), s_sel=torch.empty(sel, dtype=f32, device=dev),
-             offsets=torch.empty(w.B * w.Hkv * w.Nc + 1, dtype=i32, device=dev),
-             entries=torch.empty(w.B * w.L * w.Hkv * w.topk, dtype=i32, device=dev),
-             O=torch.empty_like(X["q"]), w=torch.empty(sel, dtype=f32, device=dev))
-    calls = ["hsa_chunk_pool", "hsa_select_topk", "hsa_build_index", "hsa_forward"]
+             idx=torch.empty(sel, dtype=i32, device=dev), s_sel=torch.empty(sel, dtype=f32, device=dev))
+    if not select_only:
+        Y.update(offsets=torch.empty(w.B * w.Hkv * w.Nc + 1, dtype=i32, device=dev),
+                 entries=torch.empty(w.B * w.L * w.Hkv * w.topk, dtype=i32, device=dev),
+                 O=torch.empty_like(X["q"]), w=torch.empty(sel, dtype=f32, device=dev))
+    calls = ["hsa_chunk_pool", "hsa_select_topk"] + ([] if select_only else ["hsa_build_index", "hsa_forward"])
 
     def step(ev=None):
         def mark(i):
@@ -690,6 +694,8 @@ def run_prefill_1m(args, dev, pk, hsa, barrier, max_over_ranks):
         mark(1)
         hsa.select_topk(shape, X["q"], Y["kbar32"], Y["idx"], Y["s_sel"], ws=wsel)
         mark(2)
+        if select_only:
+            return
         hsa.build_index(shape, Y["idx"], Y["offsets"], Y["entries"], ws=widx)
         mark(3)
         hsa.forward(shape, X["q"], X["K"], X["V"], Y["idx"], Y["s_sel"], Y["offsets"], Y["entries"], Y["O"], Y["w"],
@@ -707,7 +713,7 @@ def run_prefill_1m(args, dev, pk, hsa, barrier, max_over_ranks):
             step(evs[i])
         barrier()
     clocks = clk.summary()
-    ms_total = max_over_ranks(sum(evs[i][0].elapsed_time(evs[i][4]) for i in range(K)))
+    ms_total = max_over_ranks(sum(evs[i][0].elapsed_time(evs[i][len(calls)]) for i in range(K)))
     per_call = {c: statistics.mean(evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(K))
                 for j, c in enumerate(calls)}
     ms_step = ms_total / K
@@ -979,6 +985,8 @@ def main():
                     help="run only the decode sub-benchmark and print its object (profiling)")
     ap.add_argument("--prefill-1m-only", action="store_true",
                     help="run only the forward-only 2^20-token prefill and print its object (profiling)")
+    ap.add_argument("--select-only", action="store_true",
+                    help="with --prefill-1m-only: pooling and selection alone (profiling captures)")
     ap.add_argument("--prefill-tokens", type=int, default=None,
                     help="sequence length of that prefill (default 2^20); for profiling captures")
     args = ap.parse_args()

@@ -445,7 +445,7 @@ __global__ void __launch_bounds__(1024) fwd_segments_kernel(const int32_t* __res
 
 // O_t = sum_j w_j O'_{t,j}; w = softmax over the selected scores or stick-breaking. One warp per (b, t, g).
 template <int D>
-__global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict__ s_sel,
+__global__ void __launch_bounds__(256, 4) fwd_merge_kernel(const float* __restrict__ s_sel,
                                                         const int32_t* __restrict__ idx,
                                                         const uint16_t* __restrict__ Opart, uint16_t* __restrict__ O,
                                                         float* __restrict__ w, long long n_rows, int Hkv, int G,
@@ -470,25 +470,38 @@ __global__ void __launch_bounds__(256) fwd_merge_kernel(const float* __restrict_
   const uint4* src = reinterpret_cast<const uint4*>(Opart) + p0 * GD8;
   uint4* dst = reinterpret_cast<uint4*>(O) + row * GD8;  // heads of group g are contiguous in O
   // every lane runs every iteration (the weight broadcast needs the full warp);
-  // lanes past the row's last 16-byte chunk only skip the memory accesses
+  // lanes past the row's last 16-byte chunk only skip the memory accesses.
+  // Slots go in batches of kMergeBatch: their weights are broadcast first, then
+  // all their partial rows are requested, then summed in slot order.
+  constexpr int kMergeBatch = 4;
   for (int base = 0; base < GD8; base += 32) {
     const int ch = base + lane;
     const bool active = ch < GD8;
     float acc[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-    for (int j = 0; j < keff; ++j) {
-      const float wb = __shfl_sync(0xFFFFFFFFu, wj, j);
-      if (!active) continue;
-      const uint4 v = src[(long long)j * GD8 + ch];
-      acc[0] += wb * bf16_lo(v.x);
-      acc[1] += wb * bf16_hi(v.x);
-      acc[2] += wb * bf16_lo(v.y);
-      acc[3] += wb * bf16_hi(v.y);
-      acc[4] += wb * bf16_lo(v.z);
-      acc[5] += wb * bf16_hi(v.z);
-      acc[6] += wb * bf16_lo(v.w);
-      acc[7] += wb * bf16_hi(v.w);
+    for (int j0 = 0; j0 < keff; j0 += kMergeBatch) {
+      float wb[kMergeBatch];
+      uint4 v[kMergeBatch];
+#pragma unroll
+      for (int u = 0; u < kMergeBatch; ++u) {
+        const int j = j0 + u;
+        wb[u] = __shfl_sync(0xFFFFFFFFu, wj, j & 31);
+        v[u] = (active && j < keff) ? src[(long long)j * GD8 + ch] : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < kMergeBatch; ++u) {
+        if (j0 + u < keff) {
+          acc[0] += wb[u] * bf16_lo(v[u].x);
+          acc[1] += wb[u] * bf16_hi(v[u].x);
+          acc[2] += wb[u] * bf16_lo(v[u].y);
+          acc[3] += wb[u] * bf16_hi(v[u].y);
+          acc[4] += wb[u] * bf16_lo(v[u].z);
+          acc[5] += wb[u] * bf16_hi(v[u].z);
+          acc[6] += wb[u] * bf16_lo(v[u].w);
+          acc[7] += wb[u] * bf16_hi(v[u].w);
+        }
+      }
     }
     if (!active) continue;
     uint4 out;
